@@ -1,0 +1,170 @@
+"""CPU oracle for the OSD verify and distill operations (test infrastructure).
+
+TEST INFRASTRUCTURE ONLY: tests/, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` leg of ``bench.py`` (plus ``--impl reference``) may import
+this package.  The product path (``paper_2310_07177_gb300``) never does.
+
+The arithmetic lives in ``osd_oracle.c`` (plain C, double precision); this
+module only compiles it with gcc and marshals numpy arrays through ctypes.
+Inputs of any float dtype are converted to float64, which is exact for bf16
+and fp32 logits.  ``torch`` tensors are accepted and converted on the CPU.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "osd_oracle.c")
+LIB_PATH = os.path.join(_HERE, "libosd_oracle.so")
+
+LOSS_KINDS = {"fkl": 0, "rkl": 1, "jsd": 2, "tvd": 3}
+
+_lib = None
+_lock = threading.Lock()
+
+
+GCC_FLAGS = ["-O2", "-std=c99", "-fPIC", "-shared", "-ffp-contract=off", "-fno-fast-math"]
+
+
+def compile_source(src: str, out: str) -> str:
+    """gcc one oracle source file into a shared library (IEEE double, no FMA
+    contraction, so x86 and aarch64 round identically)."""
+    tmp = out + f".tmp{os.getpid()}"
+    subprocess.run(["gcc", *GCC_FLAGS, "-o", tmp, src, "-lm"], check=True)
+    os.replace(tmp, out)
+    return out
+
+
+def build(force: bool = False) -> str:
+    """Compile osd_oracle.c into libosd_oracle.so unless it is up to date."""
+    if (not force and os.path.exists(LIB_PATH)
+            and os.path.getmtime(LIB_PATH) >= os.path.getmtime(_SRC)):
+        return LIB_PATH
+    return compile_source(_SRC, LIB_PATH)
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        # OSD_ORACLE_LIB lets tests/test_oracle_mutants.py load a copy of the
+        # oracle compiled with a planted mistake, to show the pins catch it.
+        path = os.environ.get("OSD_ORACLE_LIB")
+        if not path:
+            path = build()
+        lib = ctypes.CDLL(path)
+        dp = ctypes.POINTER(ctypes.c_double)
+        i32p = ctypes.POINTER(ctypes.c_int32)
+        u8p = ctypes.POINTER(ctypes.c_uint8)
+        L = ctypes.c_long
+        lib.osd_oracle_verify.restype = ctypes.c_int
+        lib.osd_oracle_verify.argtypes = [dp, dp, L, L, L, i32p, dp, ctypes.c_double,
+                                          i32p, i32p, u8p, dp, dp, dp]
+        lib.osd_oracle_distill.restype = ctypes.c_int
+        lib.osd_oracle_distill.argtypes = [dp, dp, L, L, u8p, ctypes.c_int,
+                                           ctypes.c_double, dp, dp]
+        lib.osd_oracle_log_softmax.restype = None
+        lib.osd_oracle_log_softmax.argtypes = [dp, L, ctypes.c_double, dp]
+        _lib = lib
+        return lib
+
+
+def _np(x, dtype):
+    if hasattr(x, "detach"):  # torch tensor
+        x = x.detach().to("cpu")
+        if dtype is np.float64:
+            x = x.double()
+        x = x.numpy()
+    return np.ascontiguousarray(np.asarray(x, dtype=dtype))
+
+
+def _ptr(a, ctype):
+    return a.ctypes.data_as(ctypes.POINTER(ctype))
+
+
+def log_softmax(x, temperature: float = 1.0) -> np.ndarray:
+    """Row-wise log softmax(x / T) in double precision."""
+    lib = _load()
+    x = _np(x, np.float64)
+    out = np.empty_like(x)
+    V = x.shape[-1]
+    xf = x.reshape(-1, V)
+    of = out.reshape(-1, V)
+    for r in range(xf.shape[0]):
+        lib.osd_oracle_log_softmax(_ptr(xf[r], ctypes.c_double), V,
+                                   float(temperature), _ptr(of[r], ctypes.c_double))
+    return out
+
+
+def verify(draft_logits, target_logits, draft_tokens, uniforms, temperature):
+    """Speculative-sampling verification (Appendix A.1), double precision.
+
+    draft_logits [B, k, V], target_logits [B, k+1, V], draft_tokens [B, k],
+    uniforms [B, k+1], temperature a float (pass the exact fp32 value the GPU
+    sees, e.g. ``float(np.float32(0.7))``).  Returns a dict with accepted [B],
+    out_tokens [B, k+1], mismatch_mask [B, k], margin [B, k], cdf_gap [B],
+    ratio [B, k].
+    """
+    lib = _load()
+    z = _np(draft_logits, np.float64)
+    t = _np(target_logits, np.float64)
+    y = _np(draft_tokens, np.int32)
+    u = _np(uniforms, np.float64)
+    B, k, V = z.shape
+    assert t.shape == (B, k + 1, V) and y.shape == (B, k) and u.shape == (B, k + 1)
+    acc = np.empty(B, np.int32)
+    out = np.empty((B, k + 1), np.int32)
+    mask = np.empty((B, k), np.uint8)
+    margin = np.empty((B, k), np.float64)
+    gap = np.empty(B, np.float64)
+    ratio = np.empty((B, k), np.float64)
+    rc = lib.osd_oracle_verify(_ptr(z, ctypes.c_double), _ptr(t, ctypes.c_double), B, k, V,
+                               _ptr(y, ctypes.c_int32), _ptr(u, ctypes.c_double),
+                               float(temperature), _ptr(acc, ctypes.c_int32),
+                               _ptr(out, ctypes.c_int32), _ptr(mask, ctypes.c_uint8),
+                               _ptr(margin, ctypes.c_double), _ptr(gap, ctypes.c_double),
+                               _ptr(ratio, ctypes.c_double))
+    if rc != 0:
+        raise ValueError("osd_oracle_verify rejected its arguments")
+    return {"accepted": acc, "out_tokens": out, "mismatch_mask": mask,
+            "margin": margin, "cdf_gap": gap, "ratio": ratio}
+
+
+def distill(draft_logits, target_logits, mask=None, loss_kind="fkl", beta=0.5,
+            dlogits_init=None):
+    """Per-position distillation loss and d loss / d draft_logits (Eq. 2-3).
+
+    draft_logits, target_logits [N, V] (any leading shape is flattened to
+    rows); mask [N] of 0/1 or None.  Returns (loss [N], dlogits [N, V]) in
+    float64.  Rows with mask 0 get loss 0 and keep ``dlogits_init`` (NaN by
+    default) in their gradient row.
+    """
+    lib = _load()
+    z = _np(draft_logits, np.float64)
+    t = _np(target_logits, np.float64)
+    V = z.shape[-1]
+    lead = z.shape[:-1]
+    z = z.reshape(-1, V)
+    t = t.reshape(-1, V)
+    N = z.shape[0]
+    assert t.shape == (N, V)
+    m = None if mask is None else _np(mask, np.uint8).reshape(-1)
+    loss = np.empty(N, np.float64)
+    if dlogits_init is None:
+        g = np.full((N, V), np.nan, np.float64)
+    else:
+        g = _np(dlogits_init, np.float64).reshape(N, V).copy()
+    kind = LOSS_KINDS[loss_kind] if isinstance(loss_kind, str) else int(loss_kind)
+    rc = lib.osd_oracle_distill(_ptr(z, ctypes.c_double), _ptr(t, ctypes.c_double), N, V,
+                                None if m is None else _ptr(m, ctypes.c_uint8),
+                                kind, float(beta), _ptr(loss, ctypes.c_double),
+                                _ptr(g, ctypes.c_double))
+    if rc != 0:
+        raise ValueError("osd_oracle_distill rejected its arguments")
+    return loss.reshape(lead), g.reshape(*lead, V)
