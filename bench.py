@@ -1,0 +1,496 @@
+#!/usr/bin/env python
+"""Benchmark of the OSD hot path: speculative-sampling verification and the
+distillation loss/gradient, at vocabulary 32000 (bf16 logits).
+
+One step is one pass of the whole hot path over synthetic inputs:
+  verify   B=32 sequences, k=5 draft tokens, V=32000, T=1.0, then the greedy
+           (T=0) pass over the same logits            -> 2 x 160 verified positions
+  distill  a buffer flush of N=65536 positions x V=32000, reverse KL then TVD,
+           loss and d loss / d draft logits           -> 2 x 65536 distilled positions
+The value is positions (verified + distilled) per second for the whole job.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload serving-32k|large-vocab]
+
+`--workload large-vocab` times verify at B=256, k=8, V=128256, T=0.7 followed
+by forward-KL distill of its mismatch rows (the 128k-vocabulary serving step).
+`--impl reference` times the CPU oracle (the correctness reference) on a
+bounded sample of the same workload, on the host cores.
+Prints one JSON line (rank 0).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "verified positions/s and distilled positions/s at V=32000; % of HBM peak"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def _peak_hbm():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def _source_hash(files):
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+DISTILL_SOURCES = ["paper_2310_07177_gb300/csrc/osd_distill.cu", "paper_2310_07177_gb300/csrc/osd_device.cuh"]
+VERIFY_SOURCES = ["paper_2310_07177_gb300/csrc/osd_verify.cu", "paper_2310_07177_gb300/csrc/osd_device.cuh"]
+
+
+def _traffic(kernel: str, files):
+    """DRAM bytes per launch from the committed ncu summary, if it still matches the source."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)[kernel]
+    except Exception:
+        return None
+    if rec.get("source_sha") != _source_hash(files):
+        return None
+    return rec.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """Samples nvidia-smi clocks and throttle reasons while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = float(parts[1])
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[3:7]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- workloads
+def _setup_serving_32k(dev, distill_rows=None):
+    import dataclasses
+
+    from paper_2310_07177_gb300 import workloads as W
+    spec_v, spec_d = W.VERIFY[2], W.DISTILL[4]
+    if distill_rows:
+        spec_d = dataclasses.replace(spec_d, N=distill_rows)
+    v = W.verify_inputs(spec_v, seed=W.seed_for(2), device=dev)
+    d = W.distill_inputs(spec_d, seed=W.seed_for(4), device=dev)
+    return {"v": v, "d": d, "spec_v": spec_v, "spec_d": spec_d,
+            "desc": "serving-32k: verify B=32 k=5 V=32000 bf16 T=1.0 + greedy T=0 pass; "
+                    f"distill flush N={spec_d.N} V=32000 bf16 reverse-KL + TVD"}
+
+
+def _setup_large_vocab(dev):
+    from paper_2310_07177_gb300 import workloads as W
+    v = W.verify_inputs(W.VERIFY[5], seed=W.seed_for(5), device=dev)
+    return {"v": v, "spec_v": W.VERIFY[5],
+            "desc": "large-vocab: verify B=256 k=8 V=128256 bf16 T=0.7 -> forward-KL distill of "
+                    "the mismatch rows against target[:, :k]"}
+
+
+def _bytes_verify(B, k, V, s_in, greedy):
+    return (B * (k + 1) * V * s_in) if greedy else ((B * k + B * (k + 1)) * V * s_in)
+
+
+# ----------------------------------------------------------------------------- our arm
+def run_ours(args):
+    import torch
+    import paper_2310_07177_gb300 as osd
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    osd.build_library()
+    osd.load_library()
+
+    wl = args.workload
+    setup = _setup_serving_32k(dev, args.distill_rows) if wl == "serving-32k" else _setup_large_vocab(dev)
+    stream = torch.cuda.current_stream(dev)
+    v = setup["v"]
+    sv = setup["spec_v"]
+    s_in = 2 if sv.dtype == torch.bfloat16 else 4
+    ws = torch.empty(osd.osd_verify_workspace_size(sv.B, sv.k, sv.V), dtype=torch.uint8, device=dev)
+    vout = osd.osd_verify(v["draft"], v["target"], v["tokens"], v["uniforms"], sv.temperature, workspace=ws)
+    vout0 = osd.osd_verify(v["draft"], v["target"], v["greedy_tokens"], v["uniforms"], 0.0, workspace=ws)
+    l2_flush = torch.empty(2 * 128 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+
+    if wl == "serving-32k":
+        d = setup["d"]
+        sd = setup["spec_d"]
+        dl = torch.empty(sd.N, sd.V, dtype=torch.float32, device=dev)
+        loss = torch.empty(sd.N, dtype=torch.float32, device=dev)
+        kinds = ["rkl", "tvd"]
+        dist_pos = 2 * sd.N
+        dist_bytes = sd.N * sd.V * (2 * 2 + 4)  # per launch
+    else:
+        dl = torch.empty(sv.B, sv.k, sv.V, dtype=torch.float32, device=dev)
+        loss = torch.empty(sv.B, sv.k, dtype=torch.float32, device=dev)
+        kinds = ["fkl"]
+
+    ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    n_ver = 2 if wl == "serving-32k" else 1
+
+    def step(record):
+        l2_flush.zero_()
+        e = [ev() for _ in range(1 + n_ver + len(kinds))]
+        e[0].record(stream)
+        osd.osd_verify(v["draft"], v["target"], v["tokens"], v["uniforms"], sv.temperature,
+                       workspace=ws, out=vout)
+        e[1].record(stream)
+        if wl == "serving-32k":
+            osd.osd_verify(None, v["target"], v["greedy_tokens"], None, 0.0, workspace=ws, out=vout0)
+            e[2].record(stream)
+            for i, kind in enumerate(kinds):
+                osd.osd_distill(d["draft"], d["target"], d["mask"], kind, 0.5, loss=loss, dlogits=dl)
+                e[3 + i].record(stream)
+        else:
+            osd.osd_distill(v["draft"], v["target"][:, :sv.k], vout.mismatch_mask, "fkl", 0.5,
+                            loss=loss, dlogits=dl)
+            e[2].record(stream)
+        record.append(e)
+
+    warm = []
+    for _ in range(args.warmup):
+        step(warm)
+    torch.cuda.synchronize()
+
+    props = torch.cuda.get_device_properties(dev)
+    gpu_id = str(getattr(props, "uuid", local))
+    if gpu_id and not gpu_id.startswith("GPU-") and len(gpu_id) == 36:
+        gpu_id = "GPU-" + gpu_id
+    recs = []
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(gpu_id) as clk:
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            step(recs)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+    if world > 1:
+        torch.distributed.barrier()
+
+    step_ms = [r[0].elapsed_time(r[-1]) for r in recs]
+    verify_ms = [r[0].elapsed_time(r[1]) for r in recs]
+    if wl == "serving-32k":
+        greedy_ms = [r[1].elapsed_time(r[2]) for r in recs]
+        dist_ms = [r[2 + i].elapsed_time(r[3 + i]) for r in recs for i in range(len(kinds))]
+        n_active = sd.N
+    else:
+        dist_ms = [r[1].elapsed_time(r[2]) for r in recs]
+        n_active = int(vout.mismatch_mask.sum().item())
+    total_ms = sum(step_ms)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = t.item()
+    ms_step = total_ms / args.steps
+
+    if wl == "serving-32k":
+        ver_pos = 2 * sv.B * sv.k
+        positions = ver_pos + dist_pos
+        launches = 2 * 2 + len(kinds)
+        bytes_v = _bytes_verify(sv.B, sv.k, sv.V, s_in, False)
+        bytes_g = _bytes_verify(sv.B, sv.k, sv.V, s_in, True)
+    else:
+        ver_pos = sv.B * sv.k
+        positions = ver_pos + n_active
+        launches = 2 + 1
+        bytes_v = _bytes_verify(sv.B, sv.k, sv.V, s_in, False)
+        dist_bytes = n_active * sv.V * (2 * s_in + 4)
+    value = world * positions / (ms_step / 1e3)
+    peak, peak_src = _peak_hbm()
+    avg_dist = statistics.mean(dist_ms)
+    avg_ver = statistics.mean(verify_ms)
+    kernels = {
+        "verify": {"us_per_call": avg_ver * 1e3, "alg_bytes": bytes_v,
+                   "gbs": bytes_v / (avg_ver / 1e3) / 1e9,
+                   "positions_per_s": sv.B * sv.k / (avg_ver / 1e3)},
+        "distill": {"us_per_call": avg_dist * 1e3, "alg_bytes": dist_bytes,
+                    "gbs": dist_bytes / (avg_dist / 1e3) / 1e9,
+                    "positions_per_s": (sd.N if wl == "serving-32k" else n_active) / (avg_dist / 1e3)},
+    }
+    if wl == "serving-32k":
+        avg_g = statistics.mean(greedy_ms)
+        kernels["verify_greedy"] = {"us_per_call": avg_g * 1e3, "alg_bytes": bytes_g,
+                                    "gbs": bytes_g / (avg_g / 1e3) / 1e9,
+                                    "positions_per_s": sv.B * sv.k / (avg_g / 1e3)}
+    for kv in kernels.values():
+        kv["frac_of_peak"] = kv["gbs"] / peak
+    achieved = kernels["distill"]["gbs"]
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": _traffic("distill", DISTILL_SOURCES),
+                "kernel": "distill_kernel", "peak_source": peak_src}
+
+    e2e = None
+    if not args.no_e2e and (world == 1 or rank == 0):
+        e2e = run_e2e(args, osd, setup, dev, stream, positions, wl)
+    cpu = cpu_baseline(args, setup) if (rank == 0 and world == 1 and not args.no_cpu_baseline) else None
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 1), "unit": "positions/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded random logits shaped like 32k/128k-vocabulary LLM outputs; no model weights)",
+            "config": {"workload": setup["desc"], "l2": "flushed (256 MiB write) before every step",
+                       "parallelism": f"replicas x{world} (rows sharded, no collective)"},
+            "roofline": roofline,
+            "kernels": {k2: {kk: (round(vv, 3) if isinstance(vv, float) else vv) for kk, vv in kv.items()}
+                        for k2, kv in kernels.items()},
+            "clocks": clk.summary(),
+            "gpu_launches": launches * args.steps,
+            "wall_s_timed": round(wall, 3),
+            "e2e": e2e,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+def run_e2e(args, osd, setup, dev, stream, positions, wl):
+    """Same step through the public API from pinned host buffers: inputs copied
+    host->device and results device->host inside the timed region."""
+    import torch
+    v = setup["v"]
+    sv = setup["spec_v"]
+    host = {k: v[k].cpu().pin_memory() for k in ("draft", "target", "tokens", "greedy_tokens", "uniforms")}
+    dv = {k: torch.empty_like(v[k]) for k in host}
+    h_out = {"acc": torch.empty(sv.B, dtype=torch.int32).pin_memory(),
+             "tok": torch.empty(sv.B, sv.k + 1, dtype=torch.int32).pin_memory(),
+             "mask": torch.empty(sv.B, sv.k, dtype=torch.uint8).pin_memory()}
+    ws = torch.empty(osd.osd_verify_workspace_size(sv.B, sv.k, sv.V), dtype=torch.uint8, device=dev)
+    h2d = sum(t.numel() * t.element_size() for k, t in host.items()
+              if wl == "serving-32k" or k != "greedy_tokens")
+    if wl == "serving-32k":
+        d = setup["d"]
+        sd = setup["spec_d"]
+        hd = {"draft": d["draft"].cpu().pin_memory(), "target": d["target"].cpu().pin_memory()}
+        dd = {k: torch.empty_like(d[k]) for k in hd}
+        loss = torch.empty(sd.N, dtype=torch.float32, device=dev)
+        dl = torch.empty(sd.N, sd.V, dtype=torch.float32, device=dev)
+        h_loss = torch.empty(2, sd.N, dtype=torch.float32).pin_memory()
+        h2d += sum(t.numel() * t.element_size() for t in hd.values())
+        d2h = 2 * (h_out["acc"].numel() * 4 + h_out["tok"].numel() * 4 + h_out["mask"].numel()) + h_loss.numel() * 4
+    else:
+        loss = torch.empty(sv.B, sv.k, dtype=torch.float32, device=dev)
+        dl = torch.empty(sv.B, sv.k, sv.V, dtype=torch.float32, device=dev)
+        h_loss = torch.empty(1, sv.B * sv.k, dtype=torch.float32).pin_memory()
+        d2h = h_out["acc"].numel() * 4 + h_out["tok"].numel() * 4 + h_out["mask"].numel() + h_loss.numel() * 4
+
+    def step():
+        for k in host:
+            dv[k].copy_(host[k], non_blocking=True)
+        r = osd.osd_verify(dv["draft"], dv["target"], dv["tokens"], dv["uniforms"], sv.temperature, workspace=ws)
+        h_out["acc"].copy_(r.accepted, non_blocking=True)
+        h_out["tok"].copy_(r.out_tokens, non_blocking=True)
+        h_out["mask"].copy_(r.mismatch_mask, non_blocking=True)
+        if wl == "serving-32k":
+            r0 = osd.osd_verify(None, dv["target"], dv["greedy_tokens"], None, 0.0, workspace=ws)
+            h_out["acc"].copy_(r0.accepted, non_blocking=True)
+            h_out["tok"].copy_(r0.out_tokens, non_blocking=True)
+            h_out["mask"].copy_(r0.mismatch_mask, non_blocking=True)
+            for k in hd:
+                dd[k].copy_(hd[k], non_blocking=True)
+            for i, kind in enumerate(("rkl", "tvd")):
+                osd.osd_distill(dd["draft"], dd["target"], None, kind, 0.5, loss=loss, dlogits=dl)
+                h_loss[i].copy_(loss, non_blocking=True)
+        else:
+            osd.osd_distill(dv["draft"], dv["target"][:, :sv.k], r.mismatch_mask, "fkl", 0.5, loss=loss, dlogits=dl)
+            h_loss[0].copy_(loss.reshape(-1), non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    n = max(3, args.steps // 2)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(n):
+        step()
+    e1.record(stream)
+    e1.synchronize()
+    ms = e0.elapsed_time(e1) / n
+    if wl != "serving-32k":
+        positions = sv.B * sv.k + int(h_out["mask"].sum())
+    return {"value": round(positions / (ms / 1e3), 1), "unit": "positions/s", "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h), "ms_per_step": round(ms, 3), "steps": n,
+            "note": "dlogits stays on the device, where the draft model's backward pass consumes it"}
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+def _oracle_step_time(setup, n_rows, threads):
+    """Time the oracle on the verify batch (whole) and on n_rows distill rows per
+    loss kind; returns (seconds, positions) of that bounded sample."""
+    import concurrent.futures as cf
+
+    import numpy as np
+    import oracle
+
+    v = setup["v"]
+    sv = setup["spec_v"]
+    z = v["draft"].cpu()
+    t = v["target"].cpu()
+    y = v["tokens"].cpu()
+    yg = v["greedy_tokens"].cpu()
+    u = v["uniforms"].cpu()
+    T = float(np.float32(sv.temperature))
+
+    def chunks(n, parts):
+        step = max(1, (n + parts - 1) // parts)
+        return [(i, min(n, i + step)) for i in range(0, n, step)]
+
+    jobs = []
+    for (a, b) in chunks(sv.B, threads):
+        jobs.append(lambda a=a, b=b: oracle.verify(z[a:b], t[a:b], y[a:b], u[a:b], T))
+        if "d" in setup:
+            jobs.append(lambda a=a, b=b: oracle.verify(z[a:b], t[a:b], yg[a:b], u[a:b], 0.0))
+    positions = sv.B * sv.k * (2 if "d" in setup else 1)
+    if "d" in setup:
+        d = setup["d"]
+        zd = d["draft"][:n_rows].cpu()
+        td = d["target"][:n_rows].cpu()
+        for kind in ("rkl", "tvd"):
+            for (a, b) in chunks(n_rows, threads):
+                jobs.append(lambda a=a, b=b, kind=kind: oracle.distill(zd[a:b], td[a:b], None, kind, 0.5))
+        positions += 2 * n_rows
+    t0 = time.perf_counter()
+    with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+        list(ex.map(lambda f: f(), jobs))
+    return time.perf_counter() - t0, positions
+
+
+def cpu_baseline(args, setup):
+    threads = os.cpu_count() or 1
+    n_rows = args.cpu_rows
+    secs, pos = _oracle_step_time(setup, n_rows, threads)
+    return {"value": round(pos / secs, 2), "unit": "positions/s", "cores": threads, "kind": "oracle",
+            "sample": f"whole verify batch (both passes) + {n_rows} distill rows per loss kind, "
+                      f"{secs:.1f} s on {threads} host threads (double-precision C oracle)"}
+
+
+def run_reference(args):
+    """The oracle (plain double-precision C) as the reference arm, on host cores."""
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    import torch
+    dev = "cpu"
+    setup = (_setup_serving_32k(dev, args.distill_rows) if args.workload == "serving-32k"
+             else _setup_large_vocab(dev))
+    threads = os.cpu_count() or 1
+    for _ in range(args.warmup):
+        _oracle_step_time(setup, max(16, args.cpu_rows // 8), threads)
+    times, pos = [], 0
+    for _ in range(args.steps):
+        s, pos = _oracle_step_time(setup, args.cpu_rows, threads)
+        times.append(s)
+    ms = 1e3 * sum(times) / len(times)
+    value = pos / (ms / 1e3)
+    sample = (f"per step: whole verify batch (both passes) + {args.cpu_rows} distill rows per loss kind "
+              f"of the same workload, {threads} host threads")
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 2), "unit": "positions/s",
+            "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded random logits)", "config": {"workload": setup["desc"]},
+            "cpu_baseline": {"value": round(value, 2), "unit": "positions/s", "cores": threads,
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 2), "unit": "positions/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0},
+            "torch": torch.__version__}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=["serving-32k", "large-vocab"], default="serving-32k")
+    ap.add_argument("--cpu-rows", type=int, default=4096, help="distill rows per loss kind in the oracle sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
+    ap.add_argument("--distill-rows", type=int, default=None,
+                    help="override the distill buffer size N (small cases for profiling)")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,158 @@
+/*
+ * osd.h -- C ABI of the GB300 (sm_103a) hot path of Online Speculative
+ * Decoding (Liu et al., "Online Speculative Decoding", ICML 2024).
+ *
+ * Two operations run every serving step of the paper's Algorithm 1:
+ *
+ *   osd_verify   speculative-sampling verification of k draft tokens against
+ *                k+1 target distributions (Section 3 and Appendix A.1; the
+ *                "determine number of accepted tokens and sample one more
+ *                token" step of Algorithm 1), which also emits the mismatch
+ *                mask that feeds the temporary buffer R of Algorithm 1.
+ *   osd_distill  the per-position distillation loss D(p || q_theta) of Eq. 2
+ *                with D one of the distances of Eq. 3 (forward KL, reverse
+ *                KL, JSD[beta]) or total variation distance, and its gradient
+ *                with respect to the draft logits (the analytic update step
+ *                of Algorithm 1).
+ *
+ * Conventions shared by every entry point:
+ *   - All array arguments are DEVICE pointers to caller-owned memory on the
+ *     current CUDA device; the library keeps no allocation between calls and
+ *     allocates nothing itself.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Work is enqueued asynchronously on it; outputs are valid once
+ *     the stream reaches that point.  Argument errors are detected on the
+ *     host and returned before anything is enqueued.
+ *   - No C++ exception crosses this boundary.  Functions are thread-safe as
+ *     long as concurrent calls do not share output or workspace buffers.
+ *   - Logits are row-major with the vocabulary innermost and contiguous, in
+ *     fp32 or bf16 (OSD_F32 / OSD_BF16).  Any alignment to the element size
+ *     is accepted; rows that start on 16-byte boundaries take the fast
+ *     vectorised path.
+ *   - Accumulation is fp32 inside a thread with fp64 where it decides a
+ *     sample position; exponentials use the hardware ex2 unit.
+ */
+#ifndef OSD_H_
+#define OSD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum osd_status {
+    OSD_OK = 0,
+    OSD_ERR_INVALID_ARG = 1,  /* a null pointer, size, alignment or value out of range */
+    OSD_ERR_UNSUPPORTED = 2,  /* valid arguments beyond this build's limits (e.g. V)   */
+    OSD_ERR_CUDA = 3,         /* a CUDA launch or API call failed                        */
+    OSD_ERR_TIMEOUT = 4       /* a bounded device-side wait gave up (see osd_distill)    */
+} osd_status;
+
+typedef enum osd_dtype { OSD_F32 = 0, OSD_BF16 = 1 } osd_dtype;
+
+/* Distances of Eq. 3 (Section 4.1) plus total variation distance. */
+typedef enum osd_loss {
+    OSD_FKL = 0,  /* KL(p || q)                                               */
+    OSD_RKL = 1,  /* KL(q || p)                                               */
+    OSD_JSD = 2,  /* beta KL(p || m) + (1 - beta) KL(q || m), m = beta p + (1-beta) q */
+    OSD_TVD = 3   /* 1/2 sum |p - q|                                          */
+} osd_loss;
+
+/* Largest vocabulary osd_verify accepts. */
+#define OSD_VERIFY_MAX_V (1 << 21)
+/* Largest number of draft tokens osd_verify accepts. */
+#define OSD_VERIFY_MAX_K 64
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char *osd_status_string(osd_status status);
+
+/* ABI version of this library: (major << 16) | minor. */
+int osd_abi_version(void);
+
+/*
+ * Bytes of device workspace osd_verify needs for B sequences of k draft
+ * tokens over a vocabulary of V (per-row softmax statistics).  Writes the
+ * size to *bytes.  Returns OSD_ERR_INVALID_ARG for a null `bytes` or sizes
+ * out of range, OSD_ERR_UNSUPPORTED beyond OSD_VERIFY_MAX_K/_MAX_V.
+ */
+osd_status osd_verify_workspace_size(int B, int k, int V, size_t *bytes);
+
+/*
+ * Speculative-sampling verification (Section 3, Appendix A.1, Algorithm 1).
+ *
+ * For each sequence b, with q_i = softmax(draft_logits[b,i,:] / T) and
+ * p_i = softmax(target_logits[b,i,:] / T):
+ *   - tests i = 0..k-1 in order and accepts draft_tokens[b,i] iff
+ *     uniforms[b,i] < p_i(y_i) / q_i(y_i) (strict; q(y) = 0 < p(y) accepts),
+ *     stopping at the first rejection; a = number accepted;
+ *   - samples one more token by inverse CDF with uniforms[b,k]: from
+ *     norm(max(0, p_a - q_a)) if a < k, from p_k if a = k.  The CDF runs in
+ *     ascending vocabulary order and picks min{ j : C_j > u W }.
+ *   - T == 0 is greedy: accept while y_i == argmax p_i (lowest index on
+ *     ties), then emit argmax p_a; uniforms and draft logits are not read.
+ *
+ * draft_logits   [B, k, V]    dtype, contiguous (not read when T == 0)
+ * target_logits  [B, k+1, V]  dtype, contiguous
+ * draft_tokens   [B, k]       int32
+ * uniforms       [B, k+1]     fp32 in [0, 1) (not read when T == 0)
+ * temperature    >= 0 and finite, else OSD_ERR_INVALID_ARG
+ * accepted       [B]          out: a in 0..k; -1 if any draft token of the
+ *                             sequence lies outside [0, V)
+ * out_tokens     [B, k+1]     out: y_0..y_{a-1}, the sampled token at a, then -1
+ * mismatch_mask  [B, k]       out: 1 at i == a when a < k, else 0 (the first
+ *                             rejected position, the rows Algorithm 1 keeps
+ *                             for distillation)
+ * diag_margin    [B, k]       out, nullable: |u_i - r_i| for decided
+ *                             positions, NaN after the decision and when T == 0
+ * diag_cdf_gap   [B]          out, nullable: distance of u W to the nearest
+ *                             edge of the chosen CDF step, divided by W (NaN
+ *                             when T == 0)
+ * workspace      device scratch of at least osd_verify_workspace_size()
+ *                bytes, 16-byte aligned; contents need no initialisation and
+ *                are garbage afterwards.  Calls that overlap on the GPU
+ *                must not share it.
+ * Limits: 1 <= k <= OSD_VERIFY_MAX_K, 1 <= V <= OSD_VERIFY_MAX_V, B >= 0.
+ */
+osd_status osd_verify(const void *draft_logits, const void *target_logits,
+                      osd_dtype dtype, int B, int k, int V,
+                      const int32_t *draft_tokens, const float *uniforms,
+                      float temperature,
+                      int32_t *accepted, int32_t *out_tokens, uint8_t *mismatch_mask,
+                      float *diag_margin, float *diag_cdf_gap,
+                      void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * Per-position distillation loss and gradient (Eq. 2-3, Section 4.1), at
+ * temperature 1, over rows laid out as [G, P, V] with element strides
+ * (the [N, V] case is G = N, P = 1, d_stride_g = t_stride_g = V).
+ * q = softmax(draft row), p = softmax(target row).
+ *
+ * draft_logits, target_logits  row (g, p) starts at base + g*stride_g +
+ *                p*stride_p elements; the V entries of a row are contiguous.
+ * mask           [G, P] uint8, nullable (NULL = every row active).
+ * kind, beta     the distance; beta in [0, 1] is used by OSD_JSD only.
+ * loss           [G, P] fp32 out: the per-position loss (the 1/n_B batch
+ *                mean of Eq. 2 is left to the caller); 0 for inactive rows.
+ * dlogits        [G, P, V] fp32 contiguous out: d loss / d draft logits,
+ *                unscaled; rows of inactive positions are NOT written.
+ * status         nullable device int32: set to 0 by this call, then to
+ *                OSD_ERR_TIMEOUT if a bounded wait for a bulk copy gave up
+ *                (that row's loss is then NaN and its gradient not written).
+ * Limits: V <= 393216 (bf16) or 196608 (fp32), else OSD_ERR_UNSUPPORTED.
+ * Rows whose logits are all -inf, or that hold +inf or NaN, are outside the
+ * domain: their results are unspecified.
+ */
+osd_status osd_distill(const void *draft_logits, const void *target_logits,
+                       osd_dtype dtype, int G, int P, int V,
+                       int64_t d_stride_g, int64_t d_stride_p,
+                       int64_t t_stride_g, int64_t t_stride_p,
+                       const uint8_t *mask, osd_loss kind, float beta,
+                       float *loss, float *dlogits, int32_t *status, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OSD_H_ */

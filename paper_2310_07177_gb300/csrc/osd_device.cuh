@@ -1,0 +1,231 @@
+// osd_device.cuh -- device-side building blocks shared by the verify and
+// distill kernels: element loads for fp32/bf16, hardware ex2/lg2, online
+// (max, sum-exp) merging, mbarrier + bulk-copy wrappers with bounded waits,
+// and thread-block-cluster primitives (rank, DSMEM map/load, barriers).
+#pragma once
+
+#include <cstdint>
+#include <cuda_bf16.h>
+
+namespace osd {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kNegInf = -__builtin_huge_valf();
+
+// ---------------------------------------------------------------- elements
+template <typename In> struct Elem;
+template <> struct Elem<float> {
+    static constexpr int kVec = 4;  // elements per 16-byte vector
+    __device__ static float load(const float* p) { return __ldg(p); }
+    __device__ static float lds(const float* p) { return *p; }
+    __device__ static void store(float* p, float v) { *p = v; }
+    __device__ static void unpack(const uint4& r, float* x) {
+        x[0] = __uint_as_float(r.x); x[1] = __uint_as_float(r.y);
+        x[2] = __uint_as_float(r.z); x[3] = __uint_as_float(r.w);
+    }
+};
+template <> struct Elem<__nv_bfloat16> {
+    static constexpr int kVec = 8;
+    __device__ static float load(const __nv_bfloat16* p) {
+        return __uint_as_float(uint32_t(__ldg(reinterpret_cast<const unsigned short*>(p))) << 16);
+    }
+    __device__ static float lds(const __nv_bfloat16* p) {
+        return __uint_as_float(uint32_t(*reinterpret_cast<const unsigned short*>(p)) << 16);
+    }
+    __device__ static void store(__nv_bfloat16* p, float v) {  // only for copying exact bf16 values
+        *reinterpret_cast<unsigned short*>(p) = (unsigned short)(__float_as_uint(v) >> 16);
+    }
+    // bf16 -> fp32 is exact: the bf16 bits are the top half of the fp32 bits.
+    __device__ static void unpack(const uint4& r, float* x) {
+        const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            x[2 * i] = __uint_as_float(w[i] << 16);
+            x[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+        }
+    }
+};
+
+// 16-byte streaming global load that bypasses L1 (read-once data).
+__device__ __forceinline__ uint4 ldg_stream(const void* p) {
+    uint4 r;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w) : "l"(p));
+    return r;
+}
+__device__ __forceinline__ uint4 lds_v4(const void* p) {
+    return *reinterpret_cast<const uint4*>(p);
+}
+__device__ __forceinline__ void stg_v4(float* p, float a, float b, float c, float d) {
+    asm volatile("st.global.v4.f32 [%0], {%1,%2,%3,%4};" :: "l"(p), "f"(a), "f"(b), "f"(c), "f"(d)
+                 : "memory");
+}
+
+// ---------------------------------------------------------------- math
+// Hardware base-2 exponential / logarithm (PTX ex2.approx / lg2.approx).
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float lg2(float x) {
+    float y;
+    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+// d * c with c = c_hi + c_lo held as a pair of floats: removes the rounding of
+// log2(e)/T from every exponent argument (it would otherwise bias all terms).
+__device__ __forceinline__ float mul2(float d, float c_hi, float c_lo) {
+    return fmaf(d, c_hi, d * c_lo);
+}
+
+// Online softmax statistics of one set of values: m = max, s = sum 2^((x-m)c).
+struct MaxSum {
+    float m;
+    float s;
+};
+__device__ __forceinline__ MaxSum merge_ms(MaxSum a, MaxSum b, float c_hi, float c_lo) {
+    if (b.m > a.m) { MaxSum t = a; a = b; b = t; }
+    if (b.m != kNegInf) a.s += b.s * ex2(mul2(b.m - a.m, c_hi, c_lo));
+    return a;
+}
+// Argmax with the lowest index on ties.
+struct MaxIdx {
+    float m;
+    int i;
+};
+__device__ __forceinline__ MaxIdx merge_mi(MaxIdx a, MaxIdx b) {
+    if (b.m > a.m || (b.m == a.m && b.i < a.i)) return b;
+    return a;
+}
+
+template <typename T, typename F>
+__device__ __forceinline__ T warp_reduce(T v, F f) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        T w;
+        if constexpr (sizeof(T) == 8) {
+            unsigned long long bits = *reinterpret_cast<unsigned long long*>(&v);
+            bits = __shfl_xor_sync(0xffffffffu, bits, o);
+            w = *reinterpret_cast<T*>(&bits);
+        } else if constexpr (sizeof(T) == 4) {
+            unsigned bits = *reinterpret_cast<unsigned*>(&v);
+            bits = __shfl_xor_sync(0xffffffffu, bits, o);
+            w = *reinterpret_cast<T*>(&bits);
+        } else {
+            static_assert(sizeof(T) % 4 == 0, "warp_reduce needs 4-byte multiples");
+            unsigned* vb = reinterpret_cast<unsigned*>(&v);
+            unsigned wb[sizeof(T) / 4];
+#pragma unroll
+            for (int k = 0; k < int(sizeof(T) / 4); ++k) wb[k] = __shfl_xor_sync(0xffffffffu, vb[k], o);
+            w = *reinterpret_cast<T*>(wb);
+        }
+        v = f(v, w);
+    }
+    return v;
+}
+
+// Block-wide reduction through shared scratch (one slot per warp); result is
+// returned to every thread.  `scratch` holds at least kThreads/32 values.
+template <int kThreads, typename T, typename F>
+__device__ __forceinline__ T block_reduce(T v, F f, T* scratch) {
+    constexpr int kWarps = kThreads / 32;
+    v = warp_reduce(v, f);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    __syncthreads();  // scratch may still be read by a previous reduction
+    if (lane == 0) scratch[warp] = v;
+    __syncthreads();
+    T r = scratch[0];
+#pragma unroll
+    for (int w = 1; w < kWarps; ++w) r = f(r, scratch[w]);
+    return r;
+}
+
+// ---------------------------------------------------------------- timers / errors
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// ---------------------------------------------------------------- mbarrier + bulk copy
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" :: "r"(smem_addr(bar)), "r"(count) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;"
+                 :: "r"(smem_addr(bar)), "r"(bytes) : "memory");
+}
+// One-dimensional bulk copy global -> this CTA's shared memory, completing
+// `bytes` transactions on `bar`.  dst, src 16-byte aligned; bytes % 16 == 0.
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+        :: "r"(smem_addr(dst)), "l"(src), "r"(bytes), "r"(smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok) : "r"(smem_addr(bar)), "r"(parity) : "memory");
+    return ok != 0;
+}
+// Wait for phase `parity` of `bar`, giving up after `limit_ns` of wall time.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = global_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (global_ns() - t0 > limit_ns) return false;
+    }
+    return true;
+}
+
+// ---------------------------------------------------------------- clusters
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+// The .aligned forms need a converged warp, hence the __syncwarp() first.
+__device__ __forceinline__ void cluster_sync() {
+    __syncwarp();
+    asm volatile("barrier.cluster.arrive.release.aligned;\n"
+                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_arrive() {
+    __syncwarp();
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+    __syncwarp();
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Address of `p` (in this CTA's shared memory) inside CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_rank(const void* p, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr(p)), "r"(rank));
+    return r;
+}
+__device__ __forceinline__ float ld_dsmem_f32(uint32_t addr) {
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+    return v;
+}
+__device__ __forceinline__ double ld_dsmem_f64(uint32_t addr) {
+    double v;
+    asm volatile("ld.shared::cluster.f64 %0, [%1];" : "=d"(v) : "r"(addr) : "memory");
+    return v;
+}
+__device__ __forceinline__ int ld_dsmem_s32(uint32_t addr) {
+    int v;
+    asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+
+}  // namespace osd

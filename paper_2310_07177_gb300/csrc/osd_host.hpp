@@ -1,0 +1,57 @@
+// osd_host.hpp -- host-side helpers shared by the launchers: status mapping,
+// argument checks and cluster launches through cudaLaunchKernelEx.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+
+#include "osd.h"
+
+namespace osd {
+
+inline osd_status from_cuda(cudaError_t e) { return e == cudaSuccess ? OSD_OK : OSD_ERR_CUDA; }
+
+inline bool aligned_to(const void* p, size_t a) {
+    return (reinterpret_cast<uintptr_t>(p) % a) == 0;
+}
+
+inline size_t dtype_size(osd_dtype d) { return d == OSD_BF16 ? 2 : 4; }
+
+// exp(x / T) = 2^(x * c) with c = log2(e) / T, carried as c_hi + c_lo where both
+// halves are positive floats: the pair removes the rounding of c from every
+// exponent argument, and positive halves keep -inf inputs at -inf.
+inline void split_scale(float temperature, float* c_hi, float* c_lo) {
+    const double c = 1.4426950408889634074 / static_cast<double>(temperature);
+    float hi = static_cast<float>(c);
+    if (static_cast<double>(hi) > c) hi = std::nextafter(hi, 0.0f);
+    float lo = static_cast<float>(c - static_cast<double>(hi));
+    if (!(lo > 0.0f)) lo = 1e-30f;
+    *c_hi = hi;
+    *c_lo = lo;
+}
+
+// Launch `kernel` with an optional thread-block cluster of `cluster` CTAs
+// along x (cluster == 1 launches without the attribute).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                          cudaStream_t stream, int cluster, Args&&... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    if (cluster > 1) {
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = static_cast<unsigned>(cluster);
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+    }
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
+}  // namespace osd

@@ -1,0 +1,86 @@
+"""The C-ABI library builds, loads and exports every function include/osd.h
+declares; host-side argument checks answer without touching a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "osd.h")
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(osd_[a-z_0-9]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    import paper_2310_07177_gb300 as osd
+    osd.build_library()
+    return osd.load_library()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    import paper_2310_07177_gb300 as osd
+    names = _declared()
+    assert set(names) == set(osd.EXPORTS), names
+    for name in names:
+        assert hasattr(lib, name), f"{name} missing from libosd.so"
+
+
+def test_status_strings_and_version(lib):
+    import paper_2310_07177_gb300 as osd
+    assert osd.osd_abi_version() >> 16 == 1
+    for code in range(5):
+        assert osd.osd_status_string(code).startswith("OSD_")
+    assert osd.osd_status_string(99) == "OSD_ERR_UNKNOWN"
+
+
+def test_workspace_size_host_checks(lib):
+    import paper_2310_07177_gb300 as osd
+    n = ctypes.c_size_t(0)
+    assert lib.osd_verify_workspace_size(256, 8, 128256, ctypes.byref(n)) == osd.OSD_OK
+    assert n.value >= 256 * 17 * 16 * 16 and n.value % 256 == 0
+    assert lib.osd_verify_workspace_size(-1, 8, 100, ctypes.byref(n)) == osd.OSD_ERR_INVALID_ARG
+    assert lib.osd_verify_workspace_size(4, 8, 0, ctypes.byref(n)) == osd.OSD_ERR_INVALID_ARG
+    assert lib.osd_verify_workspace_size(4, 65, 100, ctypes.byref(n)) == osd.OSD_ERR_UNSUPPORTED
+    assert lib.osd_verify_workspace_size(4, 8, 100, None) == osd.OSD_ERR_INVALID_ARG
+
+
+def test_argument_errors_return_before_any_launch(lib):
+    """Invalid arguments are rejected on the host (no device pointer is touched)."""
+    import paper_2310_07177_gb300 as osd
+    fake = ctypes.c_void_p(0x1000)  # never dereferenced: every call below fails validation first
+    # bad dtype, bad temperature
+    assert lib.osd_verify(fake, fake, 7, 2, 2, 16, fake, fake, 1.0, fake, fake, fake, None, None,
+                          fake, 1 << 20, None) == osd.OSD_ERR_INVALID_ARG
+    assert lib.osd_verify(fake, fake, 0, 2, 2, 16, fake, fake, -1.0, fake, fake, fake, None, None,
+                          fake, 1 << 20, None) == osd.OSD_ERR_INVALID_ARG
+    # workspace too small
+    assert lib.osd_verify(fake, fake, 0, 2, 2, 16, fake, fake, 1.0, fake, fake, fake, None, None,
+                          fake, 8, None) == osd.OSD_ERR_INVALID_ARG
+    # empty batch is a no-op
+    assert lib.osd_verify(None, None, 0, 0, 2, 16, None, None, 1.0, None, None, None, None, None,
+                          None, 0, None) == osd.OSD_OK
+    # distill: bad beta, bad kind, vocabulary beyond the limit, negative stride
+    assert lib.osd_distill(fake, fake, 1, 2, 1, 16, 16, 0, 16, 0, None, 2, 1.5, fake, fake, None,
+                           None) == osd.OSD_ERR_INVALID_ARG
+    assert lib.osd_distill(fake, fake, 1, 2, 1, 16, 16, 0, 16, 0, None, 9, 0.5, fake, fake, None,
+                           None) == osd.OSD_ERR_INVALID_ARG
+    assert lib.osd_distill(fake, fake, 1, 1, 1, 500000, 0, 0, 0, 0, None, 0, 0.5, fake, fake, None,
+                           None) == osd.OSD_ERR_UNSUPPORTED
+    assert lib.osd_distill(fake, fake, 1, 2, 1, 16, -16, 0, 16, 0, None, 0, 0.5, fake, fake, None,
+                           None) == osd.OSD_ERR_INVALID_ARG
+    assert lib.osd_distill(None, None, 1, 0, 4, 16, 16, 0, 16, 0, None, 0, 0.5, None, None, None,
+                           None) == osd.OSD_OK
+
+
+def test_product_path_fails_loudly_without_library(tmp_path, monkeypatch):
+    import paper_2310_07177_gb300 as osd
+    monkeypatch.setattr(osd, "LIB_PATH", str(tmp_path / "missing.so"))
+    monkeypatch.setattr(osd, "_lib", None)
+    with pytest.raises(RuntimeError, match="missing"):
+        osd.load_library()

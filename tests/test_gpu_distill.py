@@ -1,0 +1,241 @@
+"""GPU parity of osd_distill (C ABI through the Python binding) against the
+oracle, for every loss kind, both dtypes, strided views, masks, ragged and
+unaligned vocabularies, and the full-size buffer-flush workloads."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2310_07177_gb300 import workloads as W
+from tests.parity import check_distill
+
+pytestmark = pytest.mark.gpu
+KINDS = ["fkl", "rkl", "jsd", "tvd"]
+
+
+@pytest.fixture(scope="module")
+def osd():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    import paper_2310_07177_gb300 as pkg
+    pkg.build_library()
+    pkg.load_library()
+    return pkg
+
+
+def _tvd_ambiguous(z, t):
+    """Entries where sign(q - p) is not decided by fp32: |ln q - ln p| < 1e-5."""
+    lq = oracle.log_softmax(z.reshape(-1, z.shape[-1]))
+    lp = oracle.log_softmax(t.reshape(-1, t.shape[-1]))
+    return np.abs(lq - lp) < 1e-5
+
+
+def _run(osd, z, t, mask, kind, beta, dev="cuda"):
+    zd, td = z.to(dev), t.to(dev)
+    md = None if mask is None else mask.to(dev)
+    V = z.shape[-1]
+    lead = tuple(z.shape[:-1])
+    dl = torch.full(lead + (V,), float("nan"), dtype=torch.float32, device=dev)
+    loss, g = osd.osd_distill(zd, td, md, kind, beta, dlogits=dl)
+    torch.cuda.synchronize()
+    return loss.cpu().numpy().reshape(-1), g.cpu().numpy().reshape(-1, V)
+
+
+def _oracle(z, t, mask, kind, beta):
+    V = z.shape[-1]
+    zc = z.reshape(-1, V)
+    tc = t.reshape(-1, V)
+    m = None if mask is None else mask.reshape(-1)
+    return oracle.distill(zc, tc, m, kind, beta)
+
+
+SHAPES = [  # (N, V, dtype)
+    (3, 1, torch.float32),
+    (5, 7, torch.bfloat16),
+    (6, 100, torch.float32),
+    (4, 8200, torch.bfloat16),
+    (3, 32000, torch.bfloat16),
+    (2, 32000, torch.float32),
+    (3, 33001, torch.bfloat16),
+    (2, 32128, torch.float32),
+    (2, 128256, torch.bfloat16),
+]
+
+
+@pytest.mark.parametrize("kind", KINDS)
+@pytest.mark.parametrize("N,V,dtype", SHAPES)
+def test_distill_matches_oracle(osd, kind, N, V, dtype):
+    spec = W.DistillSpec(N, V, dtype, 2.0, "draft+noise", 1.5, 1.0)
+    inp = W.distill_inputs(spec, seed=77 + V + N)
+    z, t = inp["draft"], inp["target"]
+    mask = torch.ones(N, dtype=torch.uint8)
+    if N >= 3:
+        mask[1] = 0
+    beta = 0.3 if kind == "jsd" else 0.5
+    lg, gg = _run(osd, z, t, mask, kind, beta)
+    lr, gr = _oracle(z, t, mask, kind, beta)
+    skip = _tvd_ambiguous(z, t) if kind == "tvd" else None
+    rep = check_distill(lg, gg, lr, gr, mask.numpy() == 1, skip)
+    print(f"{kind} N={N} V={V} {dtype}: {rep}")
+
+
+@pytest.mark.parametrize("kind", KINDS)
+def test_strided_target_view(osd, kind):
+    """Distill the [B,k] draft rows against target[:, :k] of a [B,k+1,V] tensor (no copy)."""
+    spec = W.VerifySpec(3, 4, 5000, torch.bfloat16, 2.0, 1.0, 1.0, 1.0)
+    inp = W.verify_inputs(spec, seed=3)
+    z, t = inp["draft"], inp["target"]
+    dev = torch.device("cuda")
+    td = t.to(dev)
+    view = td[:, :4, :]
+    assert not view.is_contiguous()
+    mask = torch.tensor([[1, 0, 1, 1], [0, 0, 1, 0], [1, 1, 1, 1]], dtype=torch.uint8)
+    dl = torch.full((3, 4, 5000), float("nan"), device=dev)
+    loss, g = osd.osd_distill(z.to(dev), view, mask.to(dev), kind, 0.5, dlogits=dl)
+    torch.cuda.synchronize()
+    lr, gr = _oracle(z, t[:, :4].contiguous(), mask, kind, 0.5)
+    skip = _tvd_ambiguous(z, t[:, :4].contiguous()) if kind == "tvd" else None
+    check_distill(loss.cpu().numpy().reshape(-1), g.cpu().numpy().reshape(-1, 5000), lr, gr,
+                  mask.numpy().reshape(-1) == 1, skip)
+
+
+def test_unaligned_rows(osd):
+    """Rows starting off a 16-byte boundary take the element-wise path."""
+    base = torch.randn(4 * 1001 + 3, generator=torch.Generator().manual_seed(1)) * 2
+    z = base[3:].view(4, 1001)
+    t = (z + 0.5 * torch.randn(4, 1001, generator=torch.Generator().manual_seed(2)))
+    dev = torch.device("cuda")
+    zd = base.to(dev)[3:].view(4, 1001)
+    for kind in KINDS:
+        dl = torch.full((4, 1001), float("nan"), device=dev)
+        loss, g = osd.osd_distill(zd, t.to(dev), None, kind, 0.5, dlogits=dl)
+        torch.cuda.synchronize()
+        lr, gr = _oracle(z, t, None, kind, 0.5)
+        skip = _tvd_ambiguous(z, t) if kind == "tvd" else None
+        check_distill(loss.cpu().numpy(), g.cpu().numpy(), lr, gr, np.ones(4, bool), skip)
+
+
+def test_identical_rows_and_jsd_endpoints(osd):
+    dev = torch.device("cuda")
+    z = (torch.randn(4, 3000) * 3).to(torch.bfloat16).to(dev)
+    for kind in KINDS:
+        loss, g = osd.osd_distill(z, z, None, kind, 0.5)
+        assert loss.abs().max().item() < 1e-6
+        assert g.abs().max().item() < 1e-7
+    t = (torch.randn(4, 3000) * 3).to(torch.bfloat16).to(dev)
+    for beta in (0.0, 1.0):
+        loss, g = osd.osd_distill(z, t, None, "jsd", beta)
+        assert loss.abs().max().item() == 0.0 and g.abs().max().item() == 0.0
+
+
+def test_extreme_and_neg_inf_logits(osd):
+    g0 = torch.Generator().manual_seed(9)
+    z = torch.randn(5, 3000, generator=g0) * 3
+    t = torch.randn(5, 3000, generator=g0) * 3
+    z[0] *= 30
+    t[1, 500:] = float("-inf")
+    z[2, :100] = float("-inf")
+    t[2, :100] = float("-inf")
+    t[3, 7] = 60.0
+    for kind in KINDS:
+        lg, gg = _run(osd, z, t, None, kind, 0.4)
+        lr, gr = _oracle(z, t, None, kind, 0.4)
+        skip = _tvd_ambiguous(z, t) if kind == "tvd" else None
+        check_distill(lg, gg, lr, gr, np.ones(5, bool), skip)
+
+
+def test_invalid_arguments_are_rejected(osd):
+    dev = torch.device("cuda")
+    z = torch.zeros(2, 16, device=dev)
+    with pytest.raises(osd.OsdError) as ei:
+        osd.osd_distill(z, z, None, "jsd", 1.5)
+    assert ei.value.status == osd.OSD_ERR_INVALID_ARG
+    with pytest.raises(osd.OsdError) as ei:
+        osd.osd_distill(z, z, None, 7, 0.5)
+    assert ei.value.status == osd.OSD_ERR_INVALID_ARG
+    big = torch.zeros(1, 500000, dtype=torch.bfloat16, device=dev)
+    with pytest.raises(osd.OsdError) as ei:
+        osd.osd_distill(big, big, None, "fkl", 0.5)
+    assert ei.value.status == osd.OSD_ERR_UNSUPPORTED
+    st = torch.full((1,), 123, dtype=torch.int32, device=dev)
+    e = torch.zeros(0, 16, device=dev)
+    osd.osd_distill(e, e, None, "fkl", 0.5, status=st)
+    assert st.item() == 0
+
+
+# ----------------------------------------------------------------- full-size workloads
+def test_workload_tiny_config_full(osd):
+    """Forward-KL of the 16 draft rows against target rows 0..k-1 (strided view)."""
+    spec = W.VERIFY[1]
+    inp = W.verify_inputs(spec, seed=W.seed_for(1))
+    z, t = inp["draft"], inp["target"]
+    dev = torch.device("cuda")
+    td = t.to(dev)
+    status = torch.full((1,), -1, dtype=torch.int32, device=dev)
+    dl = torch.full((4, 4, spec.V), float("nan"), device=dev)
+    loss, g = osd.osd_distill(z.to(dev), td[:, :4], None, "fkl", 0.5, dlogits=dl, status=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    lr, gr = _oracle(z, t[:, :4].contiguous(), None, "fkl", 0.5)
+    check_distill(loss.cpu().numpy().reshape(-1), g.cpu().numpy().reshape(-1, spec.V), lr, gr,
+                  np.ones(16, bool))
+
+
+def _sampled_full(osd, cfg, kind, beta, n_sample=48):
+    spec = W.DISTILL[cfg]
+    inp = W.distill_inputs(spec, seed=W.seed_for(cfg), device="cuda")
+    z, t, mask = inp["draft"], inp["target"], inp["mask"]
+    dl = torch.full((spec.N, spec.V), float("nan"), device="cuda")
+    status = torch.full((1,), -1, dtype=torch.int32, device="cuda")
+    loss, g = osd.osd_distill(z, t, mask, kind, beta, dlogits=dl, status=status)
+    torch.cuda.synchronize()
+    assert status.item() == 0
+    idx = torch.tensor(sorted(np.random.default_rng(cfg).choice(spec.N, n_sample, replace=False)),
+                       device="cuda")
+    zs, ts = z[idx].cpu(), t[idx].cpu()
+    ms = None if mask is None else mask[idx].cpu()
+    lr, gr = _oracle(zs, ts, ms, kind, beta)
+    skip = _tvd_ambiguous(zs, ts) if kind == "tvd" else None
+    act = np.ones(n_sample, bool) if ms is None else ms.numpy() == 1
+    rep = check_distill(loss[idx].cpu().numpy(), g[idx].cpu().numpy(), lr, gr, act, skip)
+    # properties over every row: loss >= 0, gradient rows sum to zero, inactive rows untouched
+    active = torch.ones(spec.N, dtype=torch.bool, device="cuda") if mask is None else mask.bool()
+    la = loss[active]
+    assert torch.isfinite(la).all() and (la >= -1e-6).all()
+    assert (loss[~active] == 0).all()
+    # softmax invariance: each gradient row sums to 0, up to fp32 rounding of its entries
+    ga = g[active].double()
+    assert (ga.sum(1).abs() <= 1e-5 * ga.abs().sum(1) + 1e-9).all()
+    assert torch.isnan(g[~active]).all()
+    return rep
+
+
+def test_workload_flush_jsd_sampled(osd):
+    print(_sampled_full(osd, 3, "jsd", 0.5))
+
+
+@pytest.mark.parametrize("kind", ["rkl", "tvd"])
+def test_workload_flush_large_sampled(osd, kind):
+    print(_sampled_full(osd, 4, kind, 0.5))
+
+
+def test_workload_large_vocab_chain(osd):
+    """Verify (B=256, k=8, V=128256, T=0.7), then forward-KL distill of the
+    rejected draft rows against target[:, :k], on one stream with no host sync."""
+    spec = W.VERIFY[5]
+    inp = W.verify_inputs(spec, seed=W.seed_for(5), device="cuda")
+    res = osd.osd_verify(inp["draft"], inp["target"], inp["tokens"], inp["uniforms"], spec.temperature)
+    dl = torch.full((spec.B, spec.k, spec.V), float("nan"), device="cuda")
+    loss, g = osd.osd_distill(inp["draft"], inp["target"][:, :spec.k], res.mismatch_mask, "fkl", 0.5,
+                              dlogits=dl)
+    torch.cuda.synchronize()
+    mask = res.mismatch_mask.cpu()
+    rows = torch.nonzero(mask.reshape(-1)).reshape(-1)
+    assert rows.numel() == int((res.accepted.cpu() < spec.k).sum())
+    sel = rows[torch.randperm(rows.numel(), generator=torch.Generator().manual_seed(0))[:16]]
+    zf = inp["draft"].reshape(-1, spec.V)[sel.cuda()].cpu()
+    tf = inp["target"][:, :spec.k].reshape(-1, spec.V)[sel.cuda()].cpu()
+    lr, gr = _oracle(zf, tf, None, "fkl", 0.5)
+    check_distill(loss.reshape(-1)[sel.cuda()].cpu().numpy(), g.reshape(-1, spec.V)[sel.cuda()].cpu().numpy(),
+                  lr, gr, np.ones(sel.numel(), bool))
+    assert (loss.reshape(-1).cpu()[mask.reshape(-1) == 0] == 0).all()

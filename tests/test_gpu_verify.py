@@ -1,0 +1,221 @@
+"""GPU parity of osd_verify (C ABI through the Python binding) against the
+oracle, plus a chi-square test of the GPU path's output distribution."""
+import math
+
+import numpy as np
+import pytest
+import torch
+from scipy.special import softmax
+from scipy.stats import chisquare
+
+import oracle
+from paper_2310_07177_gb300 import workloads as W
+from tests.parity import check_margins, check_verify
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def osd():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    import paper_2310_07177_gb300 as pkg
+    pkg.build_library()
+    pkg.load_library()
+    return pkg
+
+
+def _t32(T):
+    return float(np.float32(T))
+
+
+def _run(osd, inp, T, greedy_tokens=False):
+    dev = torch.device("cuda")
+    z = inp["draft"].to(dev)
+    t = inp["target"].to(dev)
+    y = (inp["greedy_tokens"] if greedy_tokens else inp["tokens"]).to(dev)
+    u = inp["uniforms"].to(dev)
+    res = osd.osd_verify(z, t, y, u, T)
+    torch.cuda.synchronize()
+    ref = oracle.verify(inp["draft"], inp["target"], y.cpu(), inp["uniforms"], _t32(T))
+    return res, ref
+
+
+CASES = [  # (B, k, V, dtype, T)
+    (3, 1, 1, torch.float32, 1.0),
+    (5, 2, 7, torch.bfloat16, 1.0),
+    (4, 3, 100, torch.float32, 0.7),
+    (6, 4, 4097, torch.bfloat16, 1.0),
+    (2, 5, 8193, torch.float32, 1.3),
+    (4, 4, 33001, torch.bfloat16, 0.7),
+    (3, 6, 32000, torch.bfloat16, 1.0),
+    (8, 2, 65539, torch.float32, 1.0),
+]
+
+
+@pytest.mark.parametrize("B,k,V,dtype,T", CASES)
+def test_verify_matches_oracle(osd, B, k, V, dtype, T):
+    spec = W.VerifySpec(B, k, V, dtype, 2.0, 0.8, 1.2, T)
+    inp = W.verify_inputs(spec, seed=1234 + V + k)
+    res, ref = _run(osd, inp, T)
+    rep = check_verify(res, ref, k, V)
+    check_margins(res, ref)
+    print(f"B={B} k={k} V={V} {dtype} T={T}: {rep}")
+
+
+@pytest.mark.parametrize("B,k,V,dtype", [(16, 3, 1, torch.float32), (32, 4, 1001, torch.bfloat16),
+                                         (12, 5, 32000, torch.bfloat16), (9, 2, 40000, torch.float32)])
+def test_greedy_matches_oracle(osd, B, k, V, dtype):
+    spec = W.VerifySpec(B, k, V, dtype, 2.0, 1.0, 0.3, 0.0)
+    inp = W.verify_inputs(spec, seed=99 + V)
+    # round logits to a coarse grid so argmax ties occur
+    for key in ("draft", "target"):
+        inp[key] = (inp[key].float() * 2).round().div(2).to(dtype)
+    inp["greedy_tokens"] = torch.argmax(inp["draft"].float(), -1).to(torch.int32)
+    res, ref = _run(osd, inp, 0.0, greedy_tokens=True)
+    np.testing.assert_array_equal(res.accepted.cpu().numpy(), ref["accepted"])
+    np.testing.assert_array_equal(res.out_tokens.cpu().numpy(), ref["out_tokens"])
+    np.testing.assert_array_equal(res.mismatch_mask.cpu().numpy(), ref["mismatch_mask"])
+    assert torch.isnan(res.diag_margin).all() and torch.isnan(res.diag_cdf_gap).all()
+    # greedy needs neither draft logits nor uniforms
+    dev = torch.device("cuda")
+    res2 = osd.osd_verify(None, inp["target"].to(dev), inp["greedy_tokens"].to(dev), None, 0.0)
+    assert torch.equal(res2.out_tokens, res.out_tokens)
+
+
+def test_identical_logits_accept_all(osd):
+    spec = W.VerifySpec(16, 5, 5000, torch.bfloat16, 2.0, 1.0, 0.0, 1.0)
+    inp = W.verify_inputs(spec, seed=5)
+    inp["target"] = torch.cat([inp["draft"], inp["target"][:, -1:]], dim=1).contiguous()
+    res, ref = _run(osd, inp, 1.0)
+    assert (res.accepted.cpu() == 5).all()
+    check_verify(res, ref, 5, 5000)
+
+
+def test_extreme_and_neg_inf_logits(osd):
+    B, k, V = 6, 3, 2000
+    g = torch.Generator().manual_seed(7)
+    z = torch.randn(B, k, V, generator=g) * 3
+    t = torch.randn(B, k + 1, V, generator=g) * 3
+    z[0, 0, :] = -1e4
+    z[0, 0, 5] = 1e4
+    t[1, :, 100:] = float("-inf")
+    z[2, 1, :50] = float("-inf")
+    t[3, 0, :] = torch.linspace(-1e4, 1e4, V)
+    y = torch.randint(0, 100, (B, k), generator=g).to(torch.int32)
+    y[0, 0] = 5
+    inp = {"draft": z, "target": t, "tokens": y, "uniforms": torch.rand(B, k + 1, generator=g)}
+    res, ref = _run(osd, inp, 1.0)
+    check_verify(res, ref, k, V)
+
+
+def test_bad_tokens_and_empty_batch(osd):
+    spec = W.VerifySpec(5, 3, 300, torch.float32, 2.0, 1.0, 1.0, 1.0)
+    inp = W.verify_inputs(spec, seed=8)
+    inp["tokens"][1, 2] = 300
+    inp["tokens"][3, 0] = -5
+    res, ref = _run(osd, inp, 1.0)
+    check_verify(res, ref, 3, 300)
+    assert res.accepted[1].item() == -1 and res.accepted[3].item() == -1
+    dev = torch.device("cuda")
+    e = osd.osd_verify(torch.empty(0, 3, 10, device=dev), torch.empty(0, 4, 10, device=dev),
+                       torch.empty(0, 3, dtype=torch.int32, device=dev),
+                       torch.empty(0, 4, device=dev), 1.0)
+    assert e.accepted.numel() == 0
+
+
+def test_invalid_arguments_are_rejected(osd):
+    import ctypes
+    lib = osd.load_library()
+    n = ctypes.c_size_t(0)
+    assert lib.osd_verify_workspace_size(4, 0, 100, ctypes.byref(n)) == osd.OSD_ERR_INVALID_ARG
+    assert lib.osd_verify_workspace_size(4, 65, 100, ctypes.byref(n)) == osd.OSD_ERR_UNSUPPORTED
+    assert lib.osd_verify_workspace_size(4, 2, (1 << 21) + 1, ctypes.byref(n)) == osd.OSD_ERR_UNSUPPORTED
+    dev = torch.device("cuda")
+    z = torch.zeros(2, 2, 16, device=dev)
+    t = torch.zeros(2, 3, 16, device=dev)
+    y = torch.zeros(2, 2, dtype=torch.int32, device=dev)
+    u = torch.zeros(2, 3, device=dev)
+    for T in (-1.0, float("nan"), float("inf")):
+        with pytest.raises(osd.OsdError) as ei:
+            osd.osd_verify(z, t, y, u, T)
+        assert ei.value.status == osd.OSD_ERR_INVALID_ARG
+    small = torch.empty(8, dtype=torch.uint8, device=dev)
+    with pytest.raises(osd.OsdError):
+        osd.osd_verify(z, t, y, u, 1.0, workspace=small)
+
+
+def _mc(osd, z1, t1, T, n, seed):
+    k, V = z1.shape
+    rng = np.random.default_rng(seed)
+    q = softmax(z1 / T, axis=1)
+    y = np.empty((n, k), np.int32)
+    for i in range(k):
+        c = np.cumsum(q[i]); c[-1] = 1.0
+        y[:, i] = np.searchsorted(c, rng.random(n), side="right")
+    dev = torch.device("cuda")
+    zt = torch.tensor(z1, dtype=torch.float32, device=dev).expand(n, k, V).contiguous()
+    tt = torch.tensor(t1, dtype=torch.float32, device=dev).expand(n, k + 1, V).contiguous()
+    u = torch.tensor(rng.random((n, k + 1)), dtype=torch.float32, device=dev)
+    res = osd.osd_verify(zt, tt, torch.tensor(y, device=dev), u, T, diagnostics=False)
+    return res.accepted.cpu().numpy(), res.out_tokens.cpu().numpy()
+
+
+@pytest.mark.parametrize("T,V,k", [(1.0, 5, 3), (0.6, 8, 2)])
+def test_gpu_output_distribution_equals_target(osd, T, V, k):
+    """Section 3: the emitted tokens follow p exactly; chi-square over 10^6 sequences."""
+    rng = np.random.default_rng(4000 + V)
+    z1 = rng.normal(0, 1.5, (k, V))
+    t1 = rng.normal(0, 1.5, (k + 1, V))
+    a, out = _mc(osd, z1, t1, T, 1_000_000, seed=4100 + V)
+    p = softmax(t1 / T, axis=1)
+    q = softmax(z1 / T, axis=1)
+    for i in range(k + 1):
+        tok = out[a >= i, i]
+        obs = np.bincount(tok, minlength=V)
+        pv = chisquare(obs, p[i] * tok.size).pvalue
+        assert pv > 1e-3, (i, pv)
+    for i in range(k):
+        reach, acc = np.sum(a >= i), np.sum(a >= i + 1)
+        alpha = np.minimum(p[i], q[i]).sum()
+        assert abs(acc / reach - alpha) < 5 * math.sqrt(alpha * (1 - alpha) / reach)
+
+
+# ----------------------------------------------------------------- full-size workloads
+@pytest.mark.parametrize("cfg", [1, 2])
+def test_workload_small_configs_full(osd, cfg):
+    spec = W.VERIFY[cfg]
+    inp = W.verify_inputs(spec, seed=W.seed_for(cfg))
+    res, ref = _run(osd, inp, spec.temperature)
+    rep = check_verify(res, ref, spec.k, spec.V)
+    check_margins(res, ref)
+    print(f"config {cfg}: {rep}, alpha={np.mean(ref['accepted']) / spec.k:.3f}")
+    if cfg == 2:  # greedy pass on the same logits with argmax proposals
+        res0, ref0 = _run(osd, inp, 0.0, greedy_tokens=True)
+        np.testing.assert_array_equal(res0.out_tokens.cpu().numpy(), ref0["out_tokens"])
+        np.testing.assert_array_equal(res0.accepted.cpu().numpy(), ref0["accepted"])
+
+
+def test_workload_large_vocab_sampled(osd):
+    """B=256, k=8, V=128256 bf16, T=0.7 at full size on the GPU, exactly as the
+    benchmark launches it; 24 sampled sequences are checked against the oracle."""
+    spec = W.VERIFY[5]
+    inp = W.verify_inputs(spec, seed=W.seed_for(5), device="cuda")
+    res = osd.osd_verify(inp["draft"], inp["target"], inp["tokens"], inp["uniforms"], spec.temperature)
+    torch.cuda.synchronize()
+    idx = torch.tensor(sorted(np.random.default_rng(0).choice(spec.B, 24, replace=False)))
+    ref = oracle.verify(inp["draft"][idx].cpu(), inp["target"][idx].cpu(), inp["tokens"][idx].cpu(),
+                        inp["uniforms"][idx].cpu(), _t32(spec.temperature))
+
+    class Sub:
+        pass
+    sub = Sub()
+    for f in ("accepted", "out_tokens", "mismatch_mask", "diag_margin", "diag_cdf_gap"):
+        setattr(sub, f, getattr(res, f)[idx.to(res.accepted.device)])
+    rep = check_verify(sub, ref, spec.k, spec.V)
+    check_margins(sub, ref)
+    # properties over every sequence
+    acc = res.accepted.cpu()
+    assert ((acc >= 0) & (acc <= spec.k)).all()
+    assert (res.mismatch_mask.sum(1).cpu() == (acc < spec.k).to(torch.uint8)).all()
+    print(f"config 5 sampled: {rep}, mean accepted {acc.float().mean():.3f}")
