@@ -17,8 +17,8 @@
  *
  * Conventions shared by every entry point:
  *   - All array arguments are DEVICE pointers to caller-owned memory on the
- *     current CUDA device; the library keeps no allocation between calls and
- *     allocates nothing itself.
+ *     current CUDA device; the library allocates nothing itself.  Apart from
+ *     the fixed array behind osd_verify_noalloc it keeps no device memory.
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
  *     stream).  Work is enqueued asynchronously on it; outputs are valid once
  *     the stream reaches that point.  Argument errors are detected on the
@@ -122,6 +122,35 @@ osd_status osd_verify(const void *draft_logits, const void *target_logits,
                       int32_t *accepted, int32_t *out_tokens, uint8_t *mismatch_mask,
                       float *diag_margin, float *diag_cdf_gap,
                       void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * osd_verify without a caller-supplied workspace (no counterpart in the paper).
+ *
+ * For callers that must not allocate device memory while serving: engines
+ * that reserve all free device memory for their KV cache at start-up, plugins
+ * running inside such an engine without an allocator of their own, and
+ * latency-critical loops where cudaMalloc, which may synchronise the device,
+ * would stall the other streams.  Arguments and results are those of
+ * osd_verify; the workspace is a 4 MiB array inside the library (one per GPU
+ * that loads it, kept until the process exits).  This function allocates
+ * nothing: no cudaMalloc, cudaFree or allocating library call.
+ *   - The first call on a device looks up that device's copy of the array
+ *     (cudaGetSymbolAddress, with the device current); make that first call
+ *     before any stream capture.
+ *   - Returns OSD_ERR_UNSUPPORTED when osd_verify_workspace_size(B, k, V)
+ *     exceeds 4 MiB (B * (2k+1) * ceil(V / 8192) * 16 bytes), or when the
+ *     current device ordinal is 64 or more.
+ *   - All calls on a device share the one array, which keeps the last call's
+ *     contents (every entry is rewritten before it is read, so nothing needs
+ *     clearing).  Calls that overlap on the GPU, on different streams or from
+ *     different threads, race on it: serialise them.
+ */
+osd_status osd_verify_noalloc(const void *draft_logits, const void *target_logits,
+                              osd_dtype dtype, int B, int k, int V,
+                              const int32_t *draft_tokens, const float *uniforms,
+                              float temperature,
+                              int32_t *accepted, int32_t *out_tokens, uint8_t *mismatch_mask,
+                              float *diag_margin, float *diag_cdf_gap, void *stream);
 
 /*
  * Per-position distillation loss and gradient (Eq. 2-3, Section 4.1), at

@@ -29,7 +29,7 @@ VERIFY_MAX_V = 1 << 21
 
 # every symbol include/osd.h declares
 EXPORTS = ("osd_status_string", "osd_abi_version", "osd_verify_workspace_size",
-           "osd_verify", "osd_distill")
+           "osd_verify", "osd_verify_noalloc", "osd_distill")
 
 
 class OsdError(RuntimeError):
@@ -58,6 +58,8 @@ def load_library():
     lib.osd_verify_workspace_size.argtypes = [i32, i32, i32, ctypes.POINTER(sz)]
     lib.osd_verify.restype = i32
     lib.osd_verify.argtypes = [vp, vp, i32, i32, i32, i32, vp, vp, f32, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.osd_verify_noalloc.restype = i32
+    lib.osd_verify_noalloc.argtypes = [vp, vp, i32, i32, i32, i32, vp, vp, f32, vp, vp, vp, vp, vp, vp]
     lib.osd_distill.restype = i32
     lib.osd_distill.argtypes = [vp, vp, i32, i32, i32, i32, i64, i64, i64, i64, vp, i32, f32, vp, vp, vp, vp]
     _lib = lib
@@ -161,6 +163,24 @@ def osd_verify(draft_logits: torch.Tensor, target_logits: torch.Tensor, draft_to
                         _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(dev, stream))
     if st != OSD_OK:
         raise OsdError(st, "osd_verify")
+    return out
+
+
+def osd_verify_noalloc(draft_logits: torch.Tensor, target_logits: torch.Tensor, draft_tokens: torch.Tensor,
+                       uniforms: Optional[torch.Tensor], temperature: float, out: VerifyResult, *,
+                       stream: Optional[torch.cuda.Stream] = None) -> VerifyResult:
+    """osd_verify on the library's own static workspace, for callers that must not
+    allocate device memory while serving (see include/osd.h).  Outputs are
+    caller-provided in ``out``; calls that overlap on the GPU must be serialised."""
+    lib = load_library()
+    B, k1, V = target_logits.shape
+    dev = _need_cuda(draft_logits, target_logits, draft_tokens, uniforms, *out)
+    st = lib.osd_verify_noalloc(_ptr(draft_logits), _ptr(target_logits), _dtype_code(target_logits), B, k1 - 1, V,
+                                _ptr(draft_tokens), _ptr(uniforms), float(temperature), _ptr(out.accepted),
+                                _ptr(out.out_tokens), _ptr(out.mismatch_mask), _ptr(out.diag_margin),
+                                _ptr(out.diag_cdf_gap), _stream(dev, stream))
+    if st != OSD_OK:
+        raise OsdError(st, "osd_verify_noalloc")
     return out
 
 

@@ -22,8 +22,9 @@
 // maxima, (t_y - m_t) - (z_y - m_z), and the ratio of the two sums, so no
 // log-sum-exp is rounded on its own.
 #include <climits>
-#include <type_traits>
 #include <cstdint>
+#include <mutex>
+#include <type_traits>
 
 #include "osd.h"
 #include "osd_device.cuh"
@@ -573,4 +574,52 @@ extern "C" osd_status osd_verify(const void* draft_logits, const void* target_lo
                                                  diag_cdf_gap, stats, s);
     return osd::launch_verify<float>(draft_logits, target_logits, B, k, V, draft_tokens, uniforms, temperature,
                                      accepted, out_tokens, mismatch_mask, diag_margin, diag_cdf_gap, stats, s);
+}
+
+// ------------------------------------------------------------------ no-allocation variant
+// Some callers cannot call cudaMalloc while they serve: engines that reserve all
+// free device memory for their KV cache at start-up and hand out nothing
+// afterwards, plugins that run inside such an engine without an allocator of
+// their own, and latency-critical loops where cudaMalloc (which may synchronise
+// the device) would stall every other stream.  osd_verify_noalloc serves them
+// with a fixed workspace that lives in the library itself: a file-scope device
+// array, one copy per GPU that loads the library, held until the process exits.
+namespace {
+constexpr size_t kNoAllocScratchBytes = size_t(4) << 20;  // 4 MiB
+constexpr int kNoAllocMaxDevices = 64;
+__device__ __align__(256) unsigned char g_verify_scratch[kNoAllocScratchBytes];
+std::mutex g_scratch_mu;
+void* g_scratch_addr[kNoAllocMaxDevices] = {};
+}  // namespace
+
+extern "C" osd_status osd_verify_noalloc(const void* draft_logits, const void* target_logits,
+                                         osd_dtype dtype, int B, int k, int V,
+                                         const int32_t* draft_tokens, const float* uniforms,
+                                         float temperature, int32_t* accepted, int32_t* out_tokens,
+                                         uint8_t* mismatch_mask, float* diag_margin, float* diag_cdf_gap,
+                                         void* stream) {
+    size_t need = 0;
+    const osd_status st = osd_verify_workspace_size(B, k, V, &need);
+    if (st != OSD_OK) return st;
+    if (need > kNoAllocScratchBytes) return OSD_ERR_UNSUPPORTED;  // beyond the static scratch
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return OSD_ERR_CUDA;
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return OSD_ERR_UNSUPPORTED;
+    void* scratch = nullptr;
+    {
+        // One-time set-up per device, with that device current: the host-side name
+        // of the array is not a device address, so ask the runtime for it.
+        std::lock_guard<std::mutex> lock(g_scratch_mu);
+        if (!g_scratch_addr[dev]) {
+            void* addr = nullptr;
+            if (cudaGetSymbolAddress(&addr, g_verify_scratch) != cudaSuccess || !addr) return OSD_ERR_CUDA;
+            g_scratch_addr[dev] = addr;
+        }
+        scratch = g_scratch_addr[dev];
+    }
+    // The statistics pass writes every workspace entry before the finalize pass
+    // reads it, so nothing in the shared array needs clearing between calls.
+    return osd_verify(draft_logits, target_logits, dtype, B, k, V, draft_tokens, uniforms, temperature,
+                      accepted, out_tokens, mismatch_mask, diag_margin, diag_cdf_gap, scratch,
+                      kNoAllocScratchBytes, stream);
 }
