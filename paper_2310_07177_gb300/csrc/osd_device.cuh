@@ -15,8 +15,27 @@ constexpr float kNegInf = -__builtin_huge_valf();
 
 // ---------------------------------------------------------------- elements
 template <typename In> struct Elem;
+// Raw 16-byte chunks: max and clamp work on the packed representation.
+// kClampBits / kClamp is -1e30 (rounded to the type): below it every logit
+// already has probability 0, and clamped entries keep exp() at exactly 0 while
+// differences of logits stay finite.
 template <> struct Elem<float> {
     static constexpr int kVec = 4;  // elements per 16-byte vector
+    __device__ static float max_raw(const uint4& r) {
+        return fmaxf(fmaxf(__uint_as_float(r.x), __uint_as_float(r.y)),
+                     fmaxf(__uint_as_float(r.z), __uint_as_float(r.w)));
+    }
+    __device__ static void clamp_raw(uint4& r) {
+        r.x = __float_as_uint(fmaxf(__uint_as_float(r.x), -1e30f));
+        r.y = __float_as_uint(fmaxf(__uint_as_float(r.y), -1e30f));
+        r.z = __float_as_uint(fmaxf(__uint_as_float(r.z), -1e30f));
+        r.w = __float_as_uint(fmaxf(__uint_as_float(r.w), -1e30f));
+    }
+    __device__ static float clamp1(float x) { return fmaxf(x, -1e30f); }
+    __device__ static float min_raw(const uint4& r) {
+        return fminf(fminf(__uint_as_float(r.x), __uint_as_float(r.y)),
+                     fminf(__uint_as_float(r.z), __uint_as_float(r.w)));
+    }
     __device__ static float load(const float* p) { return __ldg(p); }
     __device__ static float lds(const float* p) { return *p; }
     __device__ static void store(float* p, float v) { *p = v; }
@@ -27,6 +46,11 @@ template <> struct Elem<float> {
 };
 template <> struct Elem<__nv_bfloat16> {
     static constexpr int kVec = 8;
+    static constexpr uint32_t kClampBits = 0xF149F149u;  // bf16 pair of -1.0e30
+    __device__ static float max_raw(const uint4& r);
+    __device__ static float min_raw(const uint4& r);
+    __device__ static void clamp_raw(uint4& r);
+    __device__ static float clamp1(float x) { return fmaxf(x, __uint_as_float(0xF1490000u)); }
     __device__ static float load(const __nv_bfloat16* p) {
         return __uint_as_float(uint32_t(__ldg(reinterpret_cast<const unsigned short*>(p))) << 16);
     }
@@ -76,8 +100,70 @@ __device__ __forceinline__ float lg2(float x) {
 }
 // d * c with c = c_hi + c_lo held as a pair of floats: removes the rounding of
 // log2(e)/T from every exponent argument (it would otherwise bias all terms).
-__device__ __forceinline__ float mul2(float d, float c_hi, float c_lo) {
+__device__ __forceinline__ float mul_c(float d, float c_hi, float c_lo) {
     return fmaf(d, c_hi, d * c_lo);
+}
+
+// ---------------------------------------------------------------- packed f32x2 (sm_100+)
+// Two fp32 lanes per instruction; the pack/unpack moves vanish in register allocation.
+__device__ __forceinline__ unsigned long long pk2(float a, float b) {
+    unsigned long long r;
+    asm("mov.b64 %0, {%1,%2};" : "=l"(r) : "f"(a), "f"(b));
+    return r;
+}
+__device__ __forceinline__ float2 upk2(unsigned long long r) {
+    float2 v;
+    asm("mov.b64 {%0,%1}, %2;" : "=f"(v.x), "=f"(v.y) : "l"(r));
+    return v;
+}
+__device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
+    unsigned long long d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(pk2(a.x, a.y)), "l"(pk2(b.x, b.y)), "l"(pk2(c.x, c.y)));
+    return upk2(d);
+}
+__device__ __forceinline__ float2 add2(float2 a, float2 b) {
+    unsigned long long d;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(pk2(a.x, a.y)), "l"(pk2(b.x, b.y)));
+    return upk2(d);
+}
+__device__ __forceinline__ float2 sub2(float2 a, float2 b) {
+    unsigned long long d;
+    asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(pk2(a.x, a.y)), "l"(pk2(b.x, b.y)));
+    return upk2(d);
+}
+__device__ __forceinline__ float2 mul2(float2 a, float2 b) {
+    unsigned long long d;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(pk2(a.x, a.y)), "l"(pk2(b.x, b.y)));
+    return upk2(d);
+}
+__device__ __forceinline__ float2 f2(float a) { return make_float2(a, a); }
+
+// ---------------------------------------------------------------- packed bf16 pairs
+__device__ __forceinline__ uint32_t bmax2(uint32_t a, uint32_t b) {
+    uint32_t d;
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+__device__ __forceinline__ uint32_t bmin2(uint32_t a, uint32_t b) {
+    uint32_t d;
+    asm("min.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+__device__ __forceinline__ float Elem<__nv_bfloat16>::max_raw(const uint4& r) {
+    const uint32_t m = bmax2(bmax2(r.x, r.y), bmax2(r.z, r.w));
+    return fmaxf(bf16_lo(m), bf16_hi(m));
+}
+__device__ __forceinline__ float Elem<__nv_bfloat16>::min_raw(const uint4& r) {
+    const uint32_t m = bmin2(bmin2(r.x, r.y), bmin2(r.z, r.w));
+    return fminf(bf16_lo(m), bf16_hi(m));
+}
+__device__ __forceinline__ void Elem<__nv_bfloat16>::clamp_raw(uint4& r) {
+    r.x = bmax2(r.x, kClampBits);
+    r.y = bmax2(r.y, kClampBits);
+    r.z = bmax2(r.z, kClampBits);
+    r.w = bmax2(r.w, kClampBits);
 }
 
 // Online softmax statistics of one set of values: m = max, s = sum 2^((x-m)c).
@@ -87,7 +173,7 @@ struct MaxSum {
 };
 __device__ __forceinline__ MaxSum merge_ms(MaxSum a, MaxSum b, float c_hi, float c_lo) {
     if (b.m > a.m) { MaxSum t = a; a = b; b = t; }
-    if (b.m != kNegInf) a.s += b.s * ex2(mul2(b.m - a.m, c_hi, c_lo));
+    if (b.m != kNegInf) a.s += b.s * ex2(mul_c(b.m - a.m, c_hi, c_lo));
     return a;
 }
 // Argmax with the lowest index on ties.

@@ -25,7 +25,7 @@
 
 namespace osd {
 
-constexpr int kDistThreads = 256;
+constexpr int kDistThreads = 128;
 constexpr int kDistMaxCluster = 8;
 constexpr int kDistSpanBytes = 32768;         // target bytes of both rows per CTA
 constexpr int kDistMaxSmem = 192 * 1024;      // largest staging buffer per CTA
@@ -55,39 +55,18 @@ struct Stats2 {
     float a, b;
 };
 
-template <int kKind>
-__device__ __forceinline__ Stats1 merge1(Stats1 a, Stats1 b) {
-    Stats1 r;
-    r.mz = fmaxf(a.mz, b.mz);
-    r.mt = fmaxf(a.mt, b.mt);
-    const float az = (a.mz == kNegInf) ? 0.f : ex2((a.mz - r.mz) * kLog2e);
-    const float bz = (b.mz == kNegInf) ? 0.f : ex2((b.mz - r.mz) * kLog2e);
-    const float at = (a.mt == kNegInf) ? 0.f : ex2((a.mt - r.mt) * kLog2e);
-    const float bt = (b.mt == kNegInf) ? 0.f : ex2((b.mt - r.mt) * kLog2e);
-    r.Ez = a.Ez * az + b.Ez * bz;
-    r.Et = a.Et * at + b.Et * bt;
-    if (kKind == OSD_FKL) r.X = a.X * at + b.X * bt;       // weighted by target exponentials
-    else if (kKind == OSD_RKL) r.X = a.X * az + b.X * bz;  // weighted by draft exponentials
-    else r.X = 0.f;
-    r.err = a.err | b.err;
-    return r;
-}
-
-// log2 of a probability, (x - m) log2(e) - log2(s), with every operation rounded
-// on its own: the draft and target sides, and passes 2 and 3, must round alike so
-// that sign(q - p) is exactly 0 where the two rows agree.
-__device__ __forceinline__ float log2_prob(float x, float m, float l2s) {
-    return __fsub_rn(__fmul_rn(__fsub_rn(x, m), kLog2e), l2s);
-}
-
 template <typename In>
 __device__ __forceinline__ void copy_raw(In* dst, const In* src) {
     using Raw = std::conditional_t<sizeof(In) == 2, unsigned short, unsigned int>;
     *reinterpret_cast<Raw*>(dst) = __ldg(reinterpret_cast<const Raw*>(src));
 }
 
-// Visit this thread's entries of a staged span: f(z[], t[], count_tag, j0).
-template <typename In, bool kAligned, typename F>
+// Visit this thread's entries of a staged span in chunks of one 16-byte vector
+// (or single entries on the element-wise path).  Clamping (to -1e30, see Elem)
+// happens on the packed words.  f(z[], t[], count_tag, j0, zmax, tmax, ninf)
+// gets the chunk maxima when kMax is set, and ninf = "the chunk holds a -inf"
+// when kMin is set.
+template <typename In, bool kAligned, bool kClampZ, bool kClampT, bool kMax, bool kMin = false, typename F>
 __device__ __forceinline__ void sweep(const In* zs, const In* ts, int n, F&& f) {
     using E = Elem<In>;
     constexpr int kVec = E::kVec;
@@ -95,34 +74,85 @@ __device__ __forceinline__ void sweep(const In* zs, const In* ts, int n, F&& f) 
     if constexpr (kAligned) {
         const int nv = n / kVec;
         for (int v = tid; v < nv; v += kDistThreads) {
+            uint4 zr = lds_v4(zs + v * kVec), tr = lds_v4(ts + v * kVec);
+            if (kClampZ) E::clamp_raw(zr);
+            if (kClampT) E::clamp_raw(tr);
             float z[kVec], t[kVec];
-            E::unpack(lds_v4(zs + v * kVec), z);
-            E::unpack(lds_v4(ts + v * kVec), t);
-            f(z, t, std::integral_constant<int, kVec>{}, v * kVec);
+            E::unpack(zr, z);
+            E::unpack(tr, t);
+            const float cz = kMax ? E::max_raw(zr) : 0.f, ct = kMax ? E::max_raw(tr) : 0.f;
+            const bool ninf = kMin ? (fminf(E::min_raw(zr), E::min_raw(tr)) == kNegInf) : false;
+            f(z, t, std::integral_constant<int, kVec>{}, v * kVec, cz, ct, ninf);
         }
         const int r0 = nv * kVec;
         if (tid < n - r0) {
-            const float z = E::lds(zs + r0 + tid), t = E::lds(ts + r0 + tid);
-            f(&z, &t, std::integral_constant<int, 1>{}, r0 + tid);
+            float z = E::lds(zs + r0 + tid), t = E::lds(ts + r0 + tid);
+            if (kClampZ) z = E::clamp1(z);
+            if (kClampT) t = E::clamp1(t);
+            f(&z, &t, std::integral_constant<int, 1>{}, r0 + tid, z, t, fminf(z, t) == kNegInf);
         }
     } else {
         for (int e = tid; e < n; e += kDistThreads) {
-            const float z = E::lds(zs + e), t = E::lds(ts + e);
-            f(&z, &t, std::integral_constant<int, 1>{}, e);
+            float z = E::lds(zs + e), t = E::lds(ts + e);
+            if (kClampZ) z = E::clamp1(z);
+            if (kClampT) t = E::clamp1(t);
+            f(&z, &t, std::integral_constant<int, 1>{}, e, z, t, fminf(z, t) == kNegInf);
         }
     }
 }
 
+// Block-wide max of two values, then sum of three: the cheap way to merge
+// online softmax partials (every thread rescales its sums once to the block max).
+__device__ __forceinline__ float2 block_max2(float a, float b, float2* scratch) {
+    for (int o = 16; o > 0; o >>= 1) {
+        a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
+        b = fmaxf(b, __shfl_xor_sync(0xffffffffu, b, o));
+    }
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    __syncthreads();
+    if (lane == 0) scratch[warp] = make_float2(a, b);
+    __syncthreads();
+    float2 r = scratch[0];
+#pragma unroll
+    for (int w = 1; w < kDistThreads / 32; ++w) r = make_float2(fmaxf(r.x, scratch[w].x), fmaxf(r.y, scratch[w].y));
+    return r;
+}
+__device__ __forceinline__ float3 block_sum3(float a, float b, float c, float3* scratch) {
+    for (int o = 16; o > 0; o >>= 1) {
+        a += __shfl_xor_sync(0xffffffffu, a, o);
+        b += __shfl_xor_sync(0xffffffffu, b, o);
+        c += __shfl_xor_sync(0xffffffffu, c, o);
+    }
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    __syncthreads();
+    if (lane == 0) scratch[warp] = make_float3(a, b, c);
+    __syncthreads();
+    float3 r = scratch[0];
+#pragma unroll
+    for (int w = 1; w < kDistThreads / 32; ++w) r = make_float3(r.x + scratch[w].x, r.y + scratch[w].y, r.z + scratch[w].z);
+    return r;
+}
+__device__ __forceinline__ float rescale(float m, float mb) {
+    return (m == kNegInf) ? 0.f : ex2((m - mb) * kLog2e);
+}
+
 template <typename In, int kKind, bool kAligned>
 __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
-    using E = Elem<In>;
+    // JSD and TVD clamp both rows to -1e30: a zero probability then stays exactly 0
+    // and every logit difference finite, so no entry needs a guard.  FKL and RKL
+    // keep -inf (their loss is +inf when one row has mass where the other has
+    // none) and guard only the 16-byte chunks that hold a -inf.
+    constexpr bool kClamp = kKind == OSD_JSD || kKind == OSD_TVD;
+    constexpr bool kClampZ = kClamp, kClampT = kClamp;
+    constexpr bool kMoment = kKind == OSD_FKL || kKind == OSD_RKL;
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ __align__(8) uint64_t bar;
     __shared__ Stats1 s1_mine, s1_all;
     __shared__ Stats2 s2_mine, s2_all;
-    __shared__ Stats1 red1[kDistThreads / 32];
-    __shared__ Stats2 red2[kDistThreads / 32];
+    __shared__ float2 red_m[kDistThreads / 32];
+    __shared__ float3 red_s[kDistThreads / 32];
     __shared__ int s_err;
+    __shared__ float s_cu, s_cv, s_loss, s_K;
 
     const int tid = threadIdx.x;
     const int csize = p.csize;
@@ -143,7 +173,6 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
 
     // ---- stage the span of both rows in shared memory
     if (tid == 0) s_err = 0;
-    bool ok = true;
     if constexpr (kAligned) {
         const uint32_t bytes = static_cast<uint32_t>(n * sizeof(In)) & ~15u;
         const int nb = static_cast<int>(bytes / sizeof(In));
@@ -158,12 +187,9 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
             copy_raw(zs + e, zrow + e0 + e);
             copy_raw(ts + e, trow + e0 + e);
         }
-        if (bytes) {
-            ok = mbar_wait_bounded(&bar, 0, kWaitLimitNs);
-            if (!ok) {
-                atomicOr(&s_err, 1);
-                mbar_wait_bounded(&bar, 0, kWaitLimitNs);  // give copies in flight a last chance to land
-            }
+        if (bytes && !mbar_wait_bounded(&bar, 0, kWaitLimitNs)) {
+            atomicOr(&s_err, 1);
+            mbar_wait_bounded(&bar, 0, kWaitLimitNs);  // give copies in flight a last chance to land
         }
     } else {
         __syncthreads();
@@ -175,135 +201,206 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     __syncthreads();
     const int err_local = s_err;
 
-    // ---- pass 1: online max / sum-exp (+ loss moment) of the span
-    Stats1 acc{kNegInf, 0.f, kNegInf, 0.f, 0.f, err_local};
+    // ---- pass 1: online max / sum of 2^((x - m) log2 e) per thread (+ the FKL/RKL moment)
+    float mz = kNegInf, mt = kNegInf;
+    bool row_ninf = false;  // this thread saw a -inf logit (FKL, RKL)
+    float2 Ez2 = f2(0.f), Et2 = f2(0.f), X2 = f2(0.f);
     if (!err_local) {
-        sweep<In, kAligned>(zs, ts, n, [&](const float* z, const float* t, auto tag, int) {
+        sweep<In, kAligned, kClampZ, kClampT, true, kMoment>(zs, ts, n, [&](const float* z, const float* t,
+                                                                            auto tag, int, float cz, float ct,
+                                                                            bool ninf) {
             constexpr int kCnt = decltype(tag)::value;
-            float cz = z[0], ct = t[0];
-#pragma unroll
-            for (int e = 1; e < kCnt; ++e) { cz = fmaxf(cz, z[e]); ct = fmaxf(ct, t[e]); }
-            if (cz > acc.mz) {
-                const float r = (acc.mz == kNegInf) ? 0.f : ex2((acc.mz - cz) * kLog2e);
-                acc.Ez *= r;
-                if (kKind == OSD_RKL) acc.X *= r;
-                acc.mz = cz;
+            if (cz > mz) {
+                const float r = rescale(mz, cz);
+                Ez2 = mul2(Ez2, f2(r));
+                if (kKind == OSD_RKL) X2 = mul2(X2, f2(r));
+                mz = cz;
             }
-            if (ct > acc.mt) {
-                const float r = (acc.mt == kNegInf) ? 0.f : ex2((acc.mt - ct) * kLog2e);
-                acc.Et *= r;
-                if (kKind == OSD_FKL) acc.X *= r;
-                acc.mt = ct;
+            if (ct > mt) {
+                const float r = rescale(mt, ct);
+                Et2 = mul2(Et2, f2(r));
+                if (kKind == OSD_FKL) X2 = mul2(X2, f2(r));
+                mt = ct;
             }
-            if (acc.mz != kNegInf) {
+            row_ninf |= ninf;
+            if (kCnt == 1 || ninf) {  // element-wise, with the guards a -inf needs
 #pragma unroll
                 for (int e = 0; e < kCnt; ++e) {
-                    const float ez = ex2((z[e] - acc.mz) * kLog2e);
-                    acc.Ez += ez;
-                    if (kKind == OSD_RKL) acc.X += (ez > 0.f) ? ez * (z[e] - t[e]) : 0.f;
+                    if (kClampZ || mz != kNegInf) {
+                        const float ez = ex2((z[e] - mz) * kLog2e);
+                        Ez2.x += ez;
+                        if (kKind == OSD_RKL && ez > 0.f) X2.x = fmaf(ez, z[e] - t[e], X2.x);
+                    }
+                    if (kClampT || mt != kNegInf) {
+                        const float et = ex2((t[e] - mt) * kLog2e);
+                        Et2.x += et;
+                        if (kKind == OSD_FKL && et > 0.f) X2.x = fmaf(et, t[e] - z[e], X2.x);
+                    }
                 }
-            }
-            if (acc.mt != kNegInf) {
+            } else {
+                if (kClampZ || mz != kNegInf) {
 #pragma unroll
-                for (int e = 0; e < kCnt; ++e) {
-                    const float et = ex2((t[e] - acc.mt) * kLog2e);
-                    acc.Et += et;
-                    if (kKind == OSD_FKL) acc.X += (et > 0.f) ? et * (t[e] - z[e]) : 0.f;
+                    for (int e = 0; e < kCnt; e += 2) {
+                        const float2 a = mul2(sub2(make_float2(z[e], z[e + 1]), f2(mz)), f2(kLog2e));
+                        const float2 ez = make_float2(ex2(a.x), ex2(a.y));
+                        Ez2 = add2(Ez2, ez);
+                        if (kKind == OSD_RKL)
+                            X2 = fma2(ez, sub2(make_float2(z[e], z[e + 1]), make_float2(t[e], t[e + 1])), X2);
+                    }
+                }
+                if (kClampT || mt != kNegInf) {
+#pragma unroll
+                    for (int e = 0; e < kCnt; e += 2) {
+                        const float2 a = mul2(sub2(make_float2(t[e], t[e + 1]), f2(mt)), f2(kLog2e));
+                        const float2 et = make_float2(ex2(a.x), ex2(a.y));
+                        Et2 = add2(Et2, et);
+                        if (kKind == OSD_FKL)
+                            X2 = fma2(et, sub2(make_float2(t[e], t[e + 1]), make_float2(z[e], z[e + 1])), X2);
+                    }
                 }
             }
         });
     }
-    acc = block_reduce<kDistThreads>(acc, [](Stats1 a, Stats1 b) { return merge1<kKind>(a, b); }, red1);
-    if (tid == 0) s1_mine = acc;
+    // block merge: maxima first, then every thread rescales once and the sums add up
+    {
+        const float2 bm = block_max2(mz, mt, red_m);
+        const float sz = rescale(mz, bm.x), st = rescale(mt, bm.y);
+        const float xs = (kKind == OSD_RKL) ? sz : st;
+        const float3 bs = block_sum3((Ez2.x + Ez2.y) * sz, (Et2.x + Et2.y) * st, (X2.x + X2.y) * xs, red_s);
+        const int any_ninf = __syncthreads_or(row_ninf ? 1 : 0);
+        if (tid == 0) s1_mine = Stats1{bm.x, bs.x, bm.y, bs.y, bs.z, err_local | (any_ninf << 1)};
+    }
+    // cluster merge: warp 0 gathers every CTA's partial (lane r <- CTA r) and reduces
+    // it in a fixed order, so all CTAs of the row hold bit-identical statistics
     if (csize > 1) cluster_sync(); else __syncthreads();
-    if (tid == 0) {
-        Stats1 all = s1_mine;
-        if (csize > 1) {
-            for (int r = 0; r < csize; ++r) {
-                Stats1 o;
-                if (r == rank) {
-                    o = s1_mine;
-                } else {
-                    const uint32_t base = map_rank(&s1_mine, r);
-                    o.mz = ld_dsmem_f32(base + offsetof(Stats1, mz));
-                    o.Ez = ld_dsmem_f32(base + offsetof(Stats1, Ez));
-                    o.mt = ld_dsmem_f32(base + offsetof(Stats1, mt));
-                    o.Et = ld_dsmem_f32(base + offsetof(Stats1, Et));
-                    o.X = ld_dsmem_f32(base + offsetof(Stats1, X));
-                    o.err = ld_dsmem_s32(base + offsetof(Stats1, err));
-                }
-                all = (r == 0) ? o : merge1<kKind>(all, o);
+    if (tid < 32) {
+        Stats1 o{kNegInf, 0.f, kNegInf, 0.f, 0.f, 0};
+        if (tid < csize) {
+            if (tid == rank) {
+                o = s1_mine;
+            } else {
+                const uint32_t base = map_rank(&s1_mine, tid);
+                o.mz = ld_dsmem_f32(base + offsetof(Stats1, mz));
+                o.Ez = ld_dsmem_f32(base + offsetof(Stats1, Ez));
+                o.mt = ld_dsmem_f32(base + offsetof(Stats1, mt));
+                o.Et = ld_dsmem_f32(base + offsetof(Stats1, Et));
+                o.X = ld_dsmem_f32(base + offsetof(Stats1, X));
+                o.err = ld_dsmem_s32(base + offsetof(Stats1, err));
             }
         }
-        s1_all = all;
+        float gz = o.mz, gt = o.mt;
+        int err = o.err;
+        for (int off = 16; off > 0; off >>= 1) {
+            gz = fmaxf(gz, __shfl_xor_sync(0xffffffffu, gz, off));
+            gt = fmaxf(gt, __shfl_xor_sync(0xffffffffu, gt, off));
+            err |= __shfl_xor_sync(0xffffffffu, err, off);
+        }
+        const float sz = rescale(o.mz, gz), st = rescale(o.mt, gt);
+        float Ez = o.Ez * sz, Et = o.Et * st, X = o.X * ((kKind == OSD_RKL) ? sz : st);
+        for (int off = 16; off > 0; off >>= 1) {
+            Ez += __shfl_xor_sync(0xffffffffu, Ez, off);
+            Et += __shfl_xor_sync(0xffffffffu, Et, off);
+            X += __shfl_xor_sync(0xffffffffu, X, off);
+        }
+        if (tid == 0) {
+            s1_all = Stats1{gz, Ez, gt, Et, X, err};
+            // row constants, computed once: log2 p = (t - m_t) log2(e) - log2(E_t); the
+            // difference is exact, so the rounding never scales with the size of the logits
+            s_cu = -log2f(Et);
+            s_cv = -log2f(Ez);
+            const float lr = logf(Ez / Et);
+            float l = 0.f;
+            if (kKind == OSD_FKL) l = X / Et - (gt - gz) + lr;
+            if (kKind == OSD_RKL) l = X / Ez - (gz - gt) - lr;
+            s_loss = l;
+            s_K = (gz - gt) + lr + l;  // RKL: log q - log p - loss = (z - t) - K
+        }
     }
     __syncthreads();
     const Stats1 st = s1_all;
-    const bool row_err = st.err != 0;
-    const float invEz = 1.0f / st.Ez, invEt = 1.0f / st.Et;
-    float loss = 0.f;
-    if (kKind == OSD_FKL) loss = st.X * invEt - (st.mt - st.mz) - logf(st.Et * invEz);
-    if (kKind == OSD_RKL) loss = st.X * invEz - (st.mz - st.mt) - logf(st.Ez * invEt);
+    const bool row_err = (st.err & 1) != 0;
+    const bool has_ninf = (st.err & 2) != 0;  // some logit of the row is -inf
+    const float cu = s_cu, cv = s_cv;
+    const float2 mt2 = f2(st.mt), mz2 = f2(st.mz);
+    float loss = s_loss;
 
     const float beta = p.beta;
     const bool jsd_trivial = (kKind == OSD_JSD) && (beta == 0.f || beta == 1.f);  // m = q or m = p: loss 0
-    const float l2Ez = log2f(st.Ez), l2Et = log2f(st.Et);
     Stats2 s2 = {0.f, 0.f};
     if constexpr (kKind == OSD_JSD || kKind == OSD_TVD) {
         // ---- pass 2: divergence terms with the global normalisers
-        Stats2 a2{0.f, 0.f};
+        float2 A2 = f2(0.f), B2 = f2(0.f);
         if (!row_err && !jsd_trivial) {
-            sweep<In, kAligned>(zs, ts, n, [&](const float* z, const float* t, auto tag, int) {
+            sweep<In, kAligned, kClampZ, kClampT, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
+                                                                        int, float, float, bool) {
                 constexpr int kCnt = decltype(tag)::value;
 #pragma unroll
-                for (int e = 0; e < kCnt; ++e) {
-                    const float u = log2_prob(t[e], st.mt, l2Et);  // log2 p
-                    const float v = log2_prob(z[e], st.mz, l2Ez);  // log2 q
-                    const float d = v - u;
+                for (int e = 0; e < kCnt; e += 2) {
+                    const bool two = (e + 1 < kCnt);
+                    const float2 u = fma2(sub2(make_float2(t[e], two ? t[e + 1] : t[e]), mt2), f2(kLog2e), f2(cu));
+                    const float2 v = fma2(sub2(make_float2(z[e], two ? z[e + 1] : z[e]), mz2), f2(kLog2e), f2(cv));
+                    const float2 d = sub2(v, u);
+                    float2 a, b;
                     if (kKind == OSD_TVD) {
-                        const float pj = ex2(u), qj = ex2(v);
-                        a2.a += fabsf(pj - qj);
-                        a2.b += qj * ((d > 0.f) ? 0.5f : ((d < 0.f) ? -0.5f : 0.f));
+                        const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
+                        const float2 df = sub2(pj, qj);
+                        a = make_float2(fabsf(df.x), fabsf(df.y));
+                        b = make_float2((d.x > 0.f) ? qj.x : ((d.x < 0.f) ? -qj.x : 0.f),
+                                        (d.y > 0.f) ? qj.y : ((d.y < 0.f) ? -qj.y : 0.f));
                     } else {
-                        const float ad = fabsf(d);
-                        const float big = ex2(fmaxf(u, v));
-                        const float rho = ex2(-ad);  // smaller / larger of p, q
-                        const bool pbig = d <= 0.f;
-                        const float pj = pbig ? big : big * rho;
-                        const float qj = pbig ? big * rho : big;
-                        const float wbig = pbig ? beta : 1.f - beta;
-                        const float L = lg2(wbig + (1.f - wbig) * rho);  // log2(m / larger)
-                        const float l2mp = pbig ? L : L + ad;
-                        const float l2mq = pbig ? L + ad : L;
-                        a2.a += (pj > 0.f) ? -pj * l2mp : 0.f;
-                        a2.b += (qj > 0.f) ? -qj * l2mq : 0.f;
+                        float r[2][2];
+                        const float uu[2] = {u.x, u.y}, vv[2] = {v.x, v.y}, dd[2] = {d.x, d.y};
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            const float ad = fabsf(dd[h]);
+                            const float big = ex2(fmaxf(uu[h], vv[h]));
+                            const float rho = ex2(-ad);  // smaller / larger of p, q
+                            const bool pbig = dd[h] <= 0.f;
+                            const float wbig = pbig ? beta : 1.f - beta;
+                            const float L = lg2(fmaf(1.f - wbig, rho, wbig));  // log2(m / larger)
+                            const float pj = pbig ? big : big * rho;
+                            const float qj = pbig ? big * rho : big;
+                            r[h][0] = -pj * (pbig ? L : L + ad);
+                            r[h][1] = -qj * (pbig ? L + ad : L);
+                        }
+                        a = make_float2(r[0][0], r[1][0]);
+                        b = make_float2(r[0][1], r[1][1]);
                     }
+                    if (!two) { a.y = 0.f; b.y = 0.f; }
+                    A2 = add2(A2, a);
+                    B2 = add2(B2, b);
                 }
             });
         }
-        a2 = block_reduce<kDistThreads>(a2, [](Stats2 x, Stats2 y) { return Stats2{x.a + y.a, x.b + y.b}; }, red2);
-        if (tid == 0) s2_mine = a2;
+        const float3 bs = block_sum3(A2.x + A2.y, B2.x + B2.y, 0.f, red_s);
+        if (tid == 0) s2_mine = Stats2{bs.x, bs.y};
         if (csize > 1) cluster_sync(); else __syncthreads();
-        if (tid == 0) {
-            Stats2 all{0.f, 0.f};
-            for (int r = 0; r < csize; ++r) {
-                Stats2 o;
-                if (r == rank) {
-                    o = s2_mine;
+        if (tid < 32) {
+            float a = 0.f, b = 0.f;
+            if (tid < csize) {
+                if (tid == rank) {
+                    a = s2_mine.a;
+                    b = s2_mine.b;
                 } else {
-                    const uint32_t base = map_rank(&s2_mine, r);
-                    o.a = ld_dsmem_f32(base + offsetof(Stats2, a));
-                    o.b = ld_dsmem_f32(base + offsetof(Stats2, b));
+                    const uint32_t base = map_rank(&s2_mine, tid);
+                    a = ld_dsmem_f32(base + offsetof(Stats2, a));
+                    b = ld_dsmem_f32(base + offsetof(Stats2, b));
                 }
-                all.a += o.a;
-                all.b += o.b;
             }
-            s2_all = all;
+            for (int off = 16; off > 0; off >>= 1) {
+                a += __shfl_xor_sync(0xffffffffu, a, off);
+                b += __shfl_xor_sync(0xffffffffu, b, off);
+            }
+            if (tid == 0) s2_all = Stats2{a, b};
         }
         __syncthreads();
         s2 = s2_all;
-        if (kKind == OSD_TVD) loss = 0.5f * s2.a;
-        else loss = jsd_trivial ? 0.f : kLn2 * (beta * s2.a + (1.f - beta) * s2.b);
+        if (kKind == OSD_TVD) {
+            loss = 0.5f * s2.a;
+            s2.b *= 0.5f;  // sum_j q_j g_j with g = sign(q - p) / 2
+        } else {
+            loss = jsd_trivial ? 0.f : kLn2 * (beta * s2.a + (1.f - beta) * s2.b);
+        }
     }
     if (csize > 1) cluster_arrive();  // finished reading the other CTAs' shared memory
 
@@ -315,37 +412,55 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     // ---- pass 3: d loss / d draft logits of the span
     if (!row_err) {
         float* orow = p.dlogits + row * V + e0;
-        const float K_rkl = (st.mz - st.mt) + logf(st.Ez * invEt) + loss;  // RKL: lq - lp - loss = (z - t) - K
+        const float K = s_K;
         const float jsd_scale = (1.f - beta) * kLn2;
-        sweep<In, kAligned>(zs, ts, n, [&](const float* z, const float* t, auto tag, int j0) {
+        sweep<In, kAligned, kClampZ, kClampT, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
+                                                                    int j0, float, float, bool) {
             constexpr int kCnt = decltype(tag)::value;
             float gr[kCnt];
 #pragma unroll
-            for (int e = 0; e < kCnt; ++e) {
-                const float qj = ex2((z[e] - st.mz) * kLog2e) * invEz;
+            for (int e = 0; e < kCnt; e += 2) {
+                const bool two = (e + 1 < kCnt);
+                const float2 zz = make_float2(z[e], two ? z[e + 1] : z[e]);
+                const float2 tt = make_float2(t[e], two ? t[e + 1] : t[e]);
+                const float2 v = fma2(sub2(zz, mz2), f2(kLog2e), f2(cv));
+                const float2 qj = make_float2(ex2(v.x), ex2(v.y));
+                float2 gg;
                 if (kKind == OSD_FKL) {
-                    gr[e] = qj - ex2((t[e] - st.mt) * kLog2e) * invEt;
+                    const float2 u = fma2(sub2(tt, mt2), f2(kLog2e), f2(cu));
+                    gg = sub2(qj, make_float2(ex2(u.x), ex2(u.y)));
                 } else if (kKind == OSD_RKL) {
-                    gr[e] = (qj > 0.f) ? qj * ((z[e] - t[e]) - K_rkl) : 0.f;
+                    gg = mul2(qj, sub2(sub2(zz, tt), f2(K)));
+                    if (has_ninf) {  // q = 0 against an infinite log-ratio contributes 0
+                        if (!(qj.x > 0.f)) gg.x = 0.f;
+                        if (!(qj.y > 0.f)) gg.y = 0.f;
+                    }
                 } else if (kKind == OSD_TVD) {
-                    const float d = log2_prob(z[e], st.mz, l2Ez) - log2_prob(t[e], st.mt, l2Et);
-                    const float sg = (d > 0.f) ? 0.5f : ((d < 0.f) ? -0.5f : 0.f);
-                    gr[e] = qj * (sg - s2.b);
+                    const float2 d = sub2(v, fma2(sub2(tt, mt2), f2(kLog2e), f2(cu)));
+                    const float2 sg = make_float2((d.x > 0.f) ? 0.5f : ((d.x < 0.f) ? -0.5f : 0.f),
+                                                  (d.y > 0.f) ? 0.5f : ((d.y < 0.f) ? -0.5f : 0.f));
+                    gg = mul2(qj, sub2(sg, f2(s2.b)));
                 } else {
                     if (jsd_trivial) {
-                        gr[e] = 0.f;
+                        gg = f2(0.f);
                     } else {
-                        const float u = log2_prob(t[e], st.mt, l2Et);
-                        const float v = log2_prob(z[e], st.mz, l2Ez);
-                        const float d = v - u, ad = fabsf(d);
-                        const float rho = ex2(-ad);
-                        const bool pbig = d <= 0.f;
-                        const float wbig = pbig ? beta : 1.f - beta;
-                        const float L = lg2(wbig + (1.f - wbig) * rho);
-                        const float l2mq = pbig ? L + ad : L;
-                        gr[e] = (qj > 0.f) ? jsd_scale * qj * (-l2mq - s2.b) : 0.f;
+                        const float2 d = sub2(v, fma2(sub2(tt, mt2), f2(kLog2e), f2(cu)));
+                        const float dd[2] = {d.x, d.y};
+                        float l2mq[2];
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            const float ad = fabsf(dd[h]);
+                            const float rho = ex2(-ad);
+                            const bool pbig = dd[h] <= 0.f;
+                            const float wbig = pbig ? beta : 1.f - beta;
+                            const float L = lg2(fmaf(1.f - wbig, rho, wbig));
+                            l2mq[h] = pbig ? L + ad : L;
+                        }
+                        gg = mul2(mul2(qj, f2(jsd_scale)), make_float2(-l2mq[0] - s2.b, -l2mq[1] - s2.b));
                     }
                 }
+                gr[e] = gg.x;
+                if (two) gr[e + 1] = gg.y;
             }
             if constexpr (kAligned && kCnt >= 4) {
 #pragma unroll

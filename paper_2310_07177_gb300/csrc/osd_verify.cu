@@ -40,30 +40,83 @@ struct RowStat {
 };
 
 constexpr int kStatThreads = 256;
-constexpr int kStatUnroll = 4;
-constexpr int kStatSlice = 8192;  // vocabulary entries per row_stats CTA
+constexpr int kStatUnroll = 2;  // 16-byte vectors per thread per group (one group in flight ahead)
 
-constexpr int kFinThreads = 256;
+constexpr int kFinThreads = 128;
 constexpr int kFinMaxCluster = 8;
-constexpr int kFinMaxTiles = 1024;  // tiles of one CTA's vocabulary span
+constexpr int kFinMaxSub = 8192;  // sub-tiles of one CTA's vocabulary span (>= span / 32)
+constexpr int kFinUnroll = 4;     // sub-tiles of loads in flight per warp
+
+// Vocabulary entries per row_stats CTA: long slices amortise the per-CTA merge,
+// short ones keep enough CTAs in flight when there are few rows.
+static int verify_slice_len(int B, int k) {
+    const long long rows = (long long)B * (2 * k + 1);
+    return rows >= 2048 ? 32768 : (rows >= 512 ? 16384 : 8192);
+}
+
+// Sentinel for vector slots past the end of a slice: -inf never raises a
+// maximum and adds 0 to a sum.
+template <typename In> struct NegInfRaw;
+template <> struct NegInfRaw<float> { static constexpr uint32_t bits = 0xFF800000u; };
+template <> struct NegInfRaw<__nv_bfloat16> { static constexpr uint32_t bits = 0xFF80FF80u; };
+
+__device__ __forceinline__ double warp_sum_f64(double v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ double warp_incl_scan_f64(double v) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const double y = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += y;
+    }
+    return v;
+}
+
+template <typename In> __device__ __forceinline__ uint4 ninf_raw() {
+    return make_uint4(NegInfRaw<In>::bits, NegInfRaw<In>::bits, NegInfRaw<In>::bits, NegInfRaw<In>::bits);
+}
+// kW values of type In held in (the low bytes of) a 16-byte register block.
+template <typename In, int kW>
+__device__ __forceinline__ uint4 pack_raw(const float* v) {
+    if constexpr (kW == 1) {
+        return make_uint4(__float_as_uint(v[0]), 0u, 0u, 0u);
+    } else if constexpr (sizeof(In) == 4) {
+        return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]), __float_as_uint(v[3]));
+    } else {  // bf16: the values are exact bf16 numbers, so truncation keeps them
+        uint32_t w[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) w[i] = (__float_as_uint(v[2 * i]) >> 16) | (__float_as_uint(v[2 * i + 1]) & 0xffff0000u);
+        return make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+template <typename In, int kW>
+__device__ __forceinline__ void unpack_raw(const uint4& r, float* v) {
+    if constexpr (kW == 1) v[0] = __uint_as_float(r.x);
+    else Elem<In>::unpack(r, v);
+}
 
 // ------------------------------------------------------------------ pass 1
 template <typename In, bool kGreedy>
 __global__ void __launch_bounds__(kStatThreads)
 row_stats_kernel(const In* __restrict__ draft, const In* __restrict__ target,
-                 long long n_draft_rows, int V, int n_slices, float c_hi, float c_lo,
+                 long long n_draft_rows, int V, int slice_len, int n_slices, float c_hi, float c_lo,
                  RowStat* __restrict__ stats) {
     using E = Elem<In>;
     constexpr int kVec = E::kVec;
-    __shared__ MaxSum red_ms[kStatThreads / 32];
+    constexpr int kGroup = kStatUnroll * kVec;
+    __shared__ float2 red_m[kStatThreads / 32];
+    __shared__ float red_s[kStatThreads / 32];
     __shared__ MaxIdx red_mi[kStatThreads / 32];
 
     const long long item = blockIdx.x;
     const long long row = item / n_slices;
     const int slice = static_cast<int>(item - row * n_slices);
     const In* rowp = (row < n_draft_rows) ? draft + row * V : target + (row - n_draft_rows) * V;
-    const int s0 = slice * kStatSlice;
-    const int n = min(V - s0, kStatSlice);
+    const int s0 = slice * slice_len;
+    const int n = min(V - s0, slice_len);
     const In* p = rowp + s0;
 
     // head (scalar up to the first 16-byte boundary), body (vectors), tail
@@ -74,6 +127,15 @@ row_stats_kernel(const In* __restrict__ draft, const In* __restrict__ target,
     const int tail0 = head + nvec * kVec;
     const In* body = p + head;
     const int tid = threadIdx.x;
+    const uint4 ninf = make_uint4(NegInfRaw<In>::bits, NegInfRaw<In>::bits, NegInfRaw<In>::bits,
+                                  NegInfRaw<In>::bits);
+    auto load_group = [&](int v, uint4* r) {
+#pragma unroll
+        for (int u = 0; u < kStatUnroll; ++u) {
+            const int vv = v + u * kStatThreads;
+            r[u] = (vv < nvec) ? ldg_stream(body + size_t(vv) * kVec) : ninf;
+        }
+    };
 
     if constexpr (kGreedy) {
         MaxIdx acc{kNegInf, INT_MAX};
@@ -81,73 +143,91 @@ row_stats_kernel(const In* __restrict__ draft, const In* __restrict__ target,
             if (x > acc.m) { acc.m = x; acc.i = j; }
         };
         if (tid < head) take(E::load(p + tid), s0 + tid);
+        uint4 cur[kStatUnroll], nxt[kStatUnroll];
         int v = tid;
-        for (; v + (kStatUnroll - 1) * kStatThreads < nvec; v += kStatUnroll * kStatThreads) {
-            uint4 r[kStatUnroll];
+        if (v < nvec) load_group(v, cur);
+        for (; v < nvec; v += kStatUnroll * kStatThreads) {
+            const int vn = v + kStatUnroll * kStatThreads;
+            if (vn < nvec) load_group(vn, nxt);
+            float cm = E::max_raw(cur[0]);
 #pragma unroll
-            for (int u = 0; u < kStatUnroll; ++u) r[u] = ldg_stream(body + size_t(v + u * kStatThreads) * kVec);
+            for (int u = 1; u < kStatUnroll; ++u) cm = fmaxf(cm, E::max_raw(cur[u]));
+            if (cm > acc.m) {  // rare: find the first entry equal to the group maximum
 #pragma unroll
-            for (int u = 0; u < kStatUnroll; ++u) {
-                float x[kVec];
-                E::unpack(r[u], x);
-                const int j0 = s0 + head + (v + u * kStatThreads) * kVec;
+                for (int u = 0; u < kStatUnroll; ++u) {
+                    float x[kVec];
+                    E::unpack(cur[u], x);
+                    const int j0 = s0 + head + (v + u * kStatThreads) * kVec;
 #pragma unroll
-                for (int e = 0; e < kVec; ++e) take(x[e], j0 + e);
+                    for (int e = 0; e < kVec; ++e) take(x[e], j0 + e);
+                }
             }
-        }
-        for (; v < nvec; v += kStatThreads) {
-            float x[kVec];
-            E::unpack(ldg_stream(body + size_t(v) * kVec), x);
-            const int j0 = s0 + head + v * kVec;
 #pragma unroll
-            for (int e = 0; e < kVec; ++e) take(x[e], j0 + e);
+            for (int u = 0; u < kStatUnroll; ++u) cur[u] = nxt[u];
         }
         if (tid < n - tail0) take(E::load(p + tail0 + tid), s0 + tail0 + tid);
-        acc = block_reduce<kStatThreads>(acc, merge_mi, red_mi);
+        acc = block_reduce<kStatThreads>(acc, [](MaxIdx a, MaxIdx b) { return merge_mi(a, b); }, red_mi);
         if (tid == 0) stats[item] = RowStat{acc.m, 0.f, acc.i, 0};
     } else {
-        MaxSum acc{kNegInf, 0.f};
-        // Fold a chunk of values: one max (and at most one rescale) per chunk.
-        auto fold = [&](const float* x, auto cnt_tag) {
-            constexpr int kCnt = decltype(cnt_tag)::value;
-            float cm = x[0];
-#pragma unroll
-            for (int e = 1; e < kCnt; ++e) cm = fmaxf(cm, x[e]);
-            if (cm > acc.m) {
-                acc.s = (acc.m == kNegInf) ? 0.f : acc.s * ex2(mul2(acc.m - cm, c_hi, c_lo));
-                acc.m = cm;
-            }
-            if (acc.m != kNegInf) {
-                float s0v = 0.f, s1v = 0.f;
-#pragma unroll
-                for (int e = 0; e < kCnt; e += 2) {
-                    s0v += ex2(mul2(x[e] - acc.m, c_hi, c_lo));
-                    if (e + 1 < kCnt) s1v += ex2(mul2(x[e + 1] - acc.m, c_hi, c_lo));
-                }
-                acc.s += s0v + s1v;
+        float m = kNegInf;
+        float2 s2 = f2(0.f);
+        // 2^((x - m) c) with x - m exact and c = c_hi + c_lo carried as a float pair
+        auto exp_pair = [&](float a, float b) {
+            const float2 d = sub2(make_float2(a, b), f2(m));
+            const float2 g = fma2(d, f2(c_hi), mul2(d, f2(c_lo)));
+            return make_float2(ex2(g.x), ex2(g.y));
+        };
+        auto raise_max = [&](float cm) {
+            if (cm > m) {
+                s2 = (m == kNegInf) ? f2(0.f) : mul2(s2, f2(ex2(mul_c(m - cm, c_hi, c_lo))));
+                m = cm;
             }
         };
-        using One = std::integral_constant<int, 1>;
-        if (tid < head) { const float x = E::load(p + tid); fold(&x, One{}); }
+        auto one = [&](float x) {
+            raise_max(x);
+            if (m != kNegInf) s2.x += ex2(mul_c(x - m, c_hi, c_lo));
+        };
+        if (tid < head) one(E::load(p + tid));
+        uint4 cur[kStatUnroll], nxt[kStatUnroll];
         int v = tid;
-        for (; v + (kStatUnroll - 1) * kStatThreads < nvec; v += kStatUnroll * kStatThreads) {
-            uint4 r[kStatUnroll];
+        if (v < nvec) load_group(v, cur);
+        for (; v < nvec; v += kStatUnroll * kStatThreads) {
+            const int vn = v + kStatUnroll * kStatThreads;
+            if (vn < nvec) load_group(vn, nxt);
+            float cm = E::max_raw(cur[0]);
 #pragma unroll
-            for (int u = 0; u < kStatUnroll; ++u) r[u] = ldg_stream(body + size_t(v + u * kStatThreads) * kVec);
-            float x[kStatUnroll * kVec];
+            for (int u = 1; u < kStatUnroll; ++u) cm = fmaxf(cm, E::max_raw(cur[u]));
+            raise_max(cm);
+            if (m != kNegInf) {
+                float x[kGroup];
 #pragma unroll
-            for (int u = 0; u < kStatUnroll; ++u) E::unpack(r[u], x + u * kVec);
-            fold(x, std::integral_constant<int, kStatUnroll * kVec>{});
+                for (int u = 0; u < kStatUnroll; ++u) E::unpack(cur[u], x + u * kVec);
+#pragma unroll
+                for (int e = 0; e < kGroup; e += 2) s2 = add2(s2, exp_pair(x[e], x[e + 1]));
+            }
+#pragma unroll
+            for (int u = 0; u < kStatUnroll; ++u) cur[u] = nxt[u];
         }
-        for (; v < nvec; v += kStatThreads) {
-            float x[kVec];
-            E::unpack(ldg_stream(body + size_t(v) * kVec), x);
-            fold(x, std::integral_constant<int, kVec>{});
+        if (tid < n - tail0) one(E::load(p + tail0 + tid));
+        // block merge: maximum first, then one rescale per thread and a plain sum
+        float bm = m;
+        for (int o = 16; o > 0; o >>= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, o));
+        const int lane = tid & 31, warp = tid >> 5;
+        if (lane == 0) red_m[warp].x = bm;
+        __syncthreads();
+        bm = red_m[0].x;
+#pragma unroll
+        for (int w = 1; w < kStatThreads / 32; ++w) bm = fmaxf(bm, red_m[w].x);
+        float s = (m == kNegInf) ? 0.f : (s2.x + s2.y) * ex2(mul_c(m - bm, c_hi, c_lo));
+        for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+        if (lane == 0) red_s[warp] = s;
+        __syncthreads();
+        if (tid == 0) {
+            float tot = red_s[0];
+#pragma unroll
+            for (int w = 1; w < kStatThreads / 32; ++w) tot += red_s[w];
+            stats[item] = RowStat{bm, tot, 0, 0};
         }
-        if (tid < n - tail0) { const float x = E::load(p + tail0 + tid); fold(&x, One{}); }
-        auto merge = [c_hi, c_lo](MaxSum a, MaxSum b) { return merge_ms(a, b, c_hi, c_lo); };
-        acc = block_reduce<kStatThreads>(acc, merge, red_ms);
-        if (tid == 0) stats[item] = RowStat{acc.m, acc.s, 0, 0};
     }
 }
 
@@ -198,21 +278,20 @@ __device__ __forceinline__ double block_exclusive_scan(double v, double* warp_to
 template <typename In, bool kVecPath>
 __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams p) {
     using E = Elem<In>;
-    constexpr int kW = kVecPath ? E::kVec : 1;  // entries per thread per tile
-    constexpr int kTile = kFinThreads * kW;
+    constexpr int kW = kVecPath ? E::kVec : 1;  // entries per lane per sub-tile
+    constexpr int kSub = 32 * kW;
     constexpr int kWarps = kFinThreads / 32;
 
     __shared__ float s_m[2 * OSD_VERIFY_MAX_K + 1];
     __shared__ float s_s[2 * OSD_VERIFY_MAX_K + 1];
     __shared__ int s_idx[OSD_VERIFY_MAX_K + 1];
     __shared__ float s_zy[OSD_VERIFY_MAX_K], s_ty[OSD_VERIFY_MAX_K];
-    __shared__ int s_bad, s_a, s_owner, s_mode, s_tile, s_found;
-    __shared__ double s_tiles[kFinMaxTiles];
+    __shared__ int s_y[OSD_VERIFY_MAX_K];
+    __shared__ float s_u[OSD_VERIFY_MAX_K + 1];
+    __shared__ int s_a, s_owner, s_mode, s_tile;
+    extern __shared__ float s_sub[];  // one residual sum per sub-tile of this CTA's span
     __shared__ double s_span_total;  // read by the other CTAs of the cluster
     __shared__ double s_tau, s_W, s_base;
-    __shared__ double red_d[kWarps];
-    __shared__ MaxIdx red_mi[kWarps];
-    __shared__ int red_i[kWarps];
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int rank = (p.csize > 1) ? static_cast<int>(cluster_rank()) : 0;
@@ -223,43 +302,65 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
     const In* draft = static_cast<const In*>(p.draft);
     const In* target = static_cast<const In*>(p.target);
 
-    if (tid == 0) s_bad = 0;
-    __syncthreads();
-    if (tid < k) {
-        const int t = y[tid];
-        if (t < 0 || t >= V) atomicOr(&s_bad, 1);
+    // Prologue: every independent global load goes out in one round.  The last
+    // warp fetches the draft tokens and gathers the two logits each accept test
+    // needs; the warp before it fetches the uniforms; all warps merge the slice
+    // statistics of the 2k+1 rows (local row r <= k is target row r, r > k is
+    // draft row r-k-1), loading up to four rows per lane before reducing.
+    int bad = 0;
+    if (warp == kWarps - 1) {
+        for (int i = lane; i < k; i += 32) {
+            const int t = y[i];
+            s_y[i] = t;
+            if (t < 0 || t >= V) {
+                bad = 1;
+            } else if (!greedy) {
+                s_zy[i] = E::load(draft + (size_t(b) * k + i) * V + t);
+                s_ty[i] = E::load(target + (size_t(b) * (k + 1) + i) * V + t);
+            }
+        }
     }
-    // Merge slice statistics: local row r <= k is target row r, r > k is draft row r-k-1.
+    if (!greedy && warp == kWarps - 2)
+        for (int i = lane; i <= k; i += 32) s_u[i] = p.uniforms[size_t(b) * (k + 1) + i];
     const int nrows = greedy ? (k + 1) : (2 * k + 1);
-    for (int r = warp; r < nrows; r += kWarps) {
-        const long long srow = (r <= k) ? (p.n_draft_rows + (long long)b * (k + 1) + r)
-                                        : ((long long)b * k + (r - k - 1));
-        const RowStat* st = p.stats + srow * p.n_slices;
-        if (greedy) {
-            MaxIdx acc{kNegInf, INT_MAX};
-            for (int sl = lane; sl < p.n_slices; sl += 32) acc = merge_mi(acc, MaxIdx{st[sl].m, st[sl].idx});
-            acc = warp_reduce(acc, merge_mi);
-            if (lane == 0) { s_m[r] = acc.m; s_idx[r] = (acc.i == INT_MAX) ? 0 : acc.i; }
-        } else {
-            const float ch = p.c_hi, cl = p.c_lo;
-            auto merge = [ch, cl](MaxSum a, MaxSum c) { return merge_ms(a, c, ch, cl); };
-            MaxSum acc{kNegInf, 0.f};
-            for (int sl = lane; sl < p.n_slices; sl += 32) acc = merge(acc, MaxSum{st[sl].m, st[sl].s});
-            acc = warp_reduce(acc, merge);
-            if (lane == 0) { s_m[r] = acc.m; s_s[r] = acc.s; }
+    const float ch0 = p.c_hi, cl0 = p.c_lo;
+    auto srow_of = [&](int r) -> long long {
+        return (r <= k) ? (p.n_draft_rows + (long long)b * (k + 1) + r) : ((long long)b * k + (r - k - 1));
+    };
+    for (int r0 = warp; r0 < nrows; r0 += 4 * kWarps) {
+        RowStat part[4][1];
+        bool have[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int r = r0 + q * kWarps;
+            have[q] = r < nrows && lane < p.n_slices;
+            if (have[q]) part[q][0] = p.stats[srow_of(r) * p.n_slices + lane];
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int r = r0 + q * kWarps;
+            if (r >= nrows) break;  // uniform across the warp
+            const RowStat* st = p.stats + srow_of(r) * p.n_slices;
+            if (greedy) {
+                MaxIdx acc{kNegInf, INT_MAX};
+                if (have[q]) acc = MaxIdx{part[q][0].m, part[q][0].idx};
+                for (int sl = lane + 32; sl < p.n_slices; sl += 32) acc = merge_mi(acc, MaxIdx{st[sl].m, st[sl].idx});
+                acc = warp_reduce(acc, [](MaxIdx x, MaxIdx z) { return merge_mi(x, z); });
+                if (lane == 0) { s_m[r] = acc.m; s_idx[r] = (acc.i == INT_MAX) ? 0 : acc.i; }
+            } else {
+                auto merge = [ch0, cl0](MaxSum x, MaxSum z) { return merge_ms(x, z, ch0, cl0); };
+                MaxSum acc{kNegInf, 0.f};
+                if (have[q]) acc = MaxSum{part[q][0].m, part[q][0].s};
+                for (int sl = lane + 32; sl < p.n_slices; sl += 32) acc = merge(acc, MaxSum{st[sl].m, st[sl].s});
+                acc = warp_reduce(acc, merge);
+                if (lane == 0) { s_m[r] = acc.m; s_s[r] = acc.s; }
+            }
         }
     }
-    if (!greedy && tid < k) {
-        const int t = y[tid];
-        if (t >= 0 && t < V) {
-            s_zy[tid] = E::load(draft + (size_t(b) * k + tid) * V + t);
-            s_ty[tid] = E::load(target + (size_t(b) * (k + 1) + tid) * V + t);
-        }
-    }
-    __syncthreads();
+    bad = __syncthreads_or(bad);
 
     int32_t* out = p.out_tokens + size_t(b) * (k + 1);
-    if (s_bad) {  // uniform over the cluster, before any distributed shared memory access
+    if (bad) {  // uniform over the cluster, before any distributed shared memory access
         if (rank == 0) {
             if (tid == 0) { p.accepted[b] = -1; if (p.diag_gap) p.diag_gap[b] = __int_as_float(0x7fc00000); }
             for (int i = tid; i <= k; i += kFinThreads) out[i] = -1;
@@ -275,14 +376,14 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
     if (tid == 0) {
         int a = 0;
         if (greedy) {
-            while (a < k && y[a] == s_idx[a]) ++a;
+            while (a < k && s_y[a] == s_idx[a]) ++a;
         } else {
             for (; a < k; ++a) {
                 const float mt = s_m[a], st = s_s[a];
                 const float mz = s_m[k + 1 + a], sz = s_s[k + 1 + a];
                 const float D = (s_ty[a] - mt) - (s_zy[a] - mz);
                 const float r = expf(__fdiv_rn(D, p.T)) * __fdiv_rn(sz, st);
-                const float u = p.uniforms[size_t(b) * (k + 1) + a];
+                const float u = s_u[a];
                 if (rank == 0 && p.diag_margin) p.diag_margin[size_t(b) * k + a] = fabsf(u - r);
                 if (!(u < r)) break;
             }
@@ -294,7 +395,7 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
     if (rank == 0) {
         if (tid == 0) p.accepted[b] = a;
         for (int i = tid; i <= k; i += kFinThreads)
-            if (i < a) out[i] = y[i];
+            if (i < a) out[i] = s_y[i];
             else if (i > a) out[i] = -1;
         for (int i = tid; i < k; i += kFinThreads) {
             p.mask[size_t(b) * k + i] = (i == a) ? 1 : 0;
@@ -318,150 +419,206 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
     const float inv_sz = bonus ? 0.f : 1.0f / s_s[k + 1 + a];
     const float ch = p.c_hi, cl = p.c_lo;
     auto weight = [&](float t, float z) -> float {
-        const float pj = ex2(mul2(t - mt, ch, cl)) * inv_st;
+        const float pj = ex2(mul_c(t - mt, ch, cl)) * inv_st;
         if (bonus) return pj;
-        const float qj = ex2(mul2(z - mz, ch, cl)) * inv_sz;
+        const float qj = ex2(mul_c(z - mz, ch, cl)) * inv_sz;
         return fmaxf(pj - qj, 0.f);
     };
     const int e0 = rank * p.span;
     const int n = max(0, min(p.span, V - e0));
-    const int ntiles = (n + kTile - 1) / kTile;
-    // weights of this thread's entries of tile `tile` (entries past the span get 0)
-    auto tile_weights = [&](int tile, float* w) {
-        const int j0 = e0 + tile * kTile + tid * kW;
+    const int nsub = (n + kSub - 1) / kSub;  // sub-tiles: one warp step of 32 x kW entries
+    // raw entries of this lane in sub-tile s (slots past the span read as -inf: weight 0)
+    struct Raw {
+        uint4 t, z;
+    };
+    auto load_sub = [&](int s, Raw& r) {
+        const int j0 = e0 + s * kSub + lane * kW;
         const int cnt = min(kW, e0 + n - j0);
         if (kVecPath && cnt == kW) {
-            float t[kW], z[kW];
-            E::unpack(ldg_stream(trow + j0), t);
-            if (!bonus) E::unpack(ldg_stream(zrow + j0), z);
-#pragma unroll
-            for (int e = 0; e < kW; ++e) w[e] = weight(t[e], bonus ? 0.f : z[e]);
+            r.t = ldg_stream(trow + j0);
+            r.z = bonus ? r.t : ldg_stream(zrow + j0);
         } else {
+            float tv[kW], zv[kW];
 #pragma unroll
-            for (int e = 0; e < kW; ++e)
-                w[e] = (e < cnt) ? weight(E::load(trow + j0 + e), bonus ? 0.f : E::load(zrow + j0 + e)) : 0.f;
+            for (int e = 0; e < kW; ++e) {
+                tv[e] = (e < cnt) ? E::load(trow + j0 + e) : kNegInf;
+                zv[e] = (e < cnt && !bonus) ? E::load(zrow + j0 + e) : kNegInf;
+            }
+            r.t = pack_raw<In, kW>(tv);
+            r.z = pack_raw<In, kW>(zv);
         }
     };
-
-    // pass 1: per-tile sums of this CTA's span
-    double span_total = 0.0;
-    for (int tile = 0; tile < ntiles; ++tile) {
-        float w[kW];
-        tile_weights(tile, w);
-        float sum = 0.f;
+    auto sub_weights = [&](const Raw& r, float* w) {
+        float tv[kW], zv[kW];
+        unpack_raw<In, kW>(r.t, tv);
+        unpack_raw<In, kW>(r.z, zv);
 #pragma unroll
-        for (int e = 0; e < kW; ++e) sum += w[e];
-        const double ts = block_reduce<kFinThreads>(double(sum), [](double x, double z) { return x + z; }, red_d);
-        if (tid == 0) s_tiles[tile] = ts;
-        span_total += ts;
+        for (int e = 0; e < kW; ++e) w[e] = weight(tv[e], zv[e]);
+    };
+
+    // pass 1: one fp32 sum per sub-tile, reduced inside the warp, no block barrier
+    for (int s0 = warp; s0 < nsub; s0 += kWarps * kFinUnroll) {
+        Raw r[kFinUnroll];
+#pragma unroll
+        for (int u = 0; u < kFinUnroll; ++u)
+            if (s0 + u * kWarps < nsub) load_sub(s0 + u * kWarps, r[u]);
+#pragma unroll
+        for (int u = 0; u < kFinUnroll; ++u) {
+            const int s = s0 + u * kWarps;
+            if (s < nsub) {
+                float w[kW];
+                sub_weights(r[u], w);
+                float sum = 0.f;
+#pragma unroll
+                for (int e = 0; e < kW; ++e) sum += w[e];
+                for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+                if (lane == 0) s_sub[s] = sum;
+            }
+        }
     }
-    if (tid == 0) s_span_total = span_total;
+    __syncthreads();
+    // span total in fp64, reduced across warp 0 (no serial chain of fp64 adds)
+    if (warp == 0) {
+        double part = 0.0;
+        for (int s2 = lane; s2 < nsub; s2 += 32) part += double(s_sub[s2]);
+        part = warp_sum_f64(part);
+        if (lane == 0) s_span_total = part;
+    }
     if (p.csize > 1) cluster_sync(); else __syncthreads();
 
-    // every CTA derives W, tau and the owning CTA identically (rank order)
-    if (tid == 0) {
-        const float u = p.uniforms[size_t(b) * (k + 1) + k];
-        double tot[kFinMaxCluster];
-        for (int r = 0; r < p.csize; ++r)
-            tot[r] = (r == rank) ? s_span_total : ld_dsmem_f64(map_rank(&s_span_total, r));
-        double W = 0.0;
-        for (int r = 0; r < p.csize; ++r) W += tot[r];
+    // warp 0 of every CTA derives W, tau and the owning CTA identically: lane r
+    // holds CTA r's total, an fp64 warp scan gives the prefix in rank order
+    if (warp == 0) {
+        const float u = s_u[k];
+        double tot = 0.0;
+        if (lane < p.csize) tot = (lane == rank) ? s_span_total : ld_dsmem_f64(map_rank(&s_span_total, lane));
+        const double incl = warp_incl_scan_f64(tot);
+        const double W = __shfl_sync(0xffffffffu, incl, 31);
         const double tau = double(u) * W;
-        int owner = -1, mode = 0;  // mode 0: inverse CDF, 1: largest positive entry, 2: argmax p
-        double cum = 0.0, base = 0.0;
+        int owner, mode = 0;  // mode 0: inverse CDF, 1: largest positive entry, 2: argmax p
+        double base = 0.0;
         if (W > 0.0) {
-            for (int r = 0; r < p.csize; ++r) {
-                if (cum + tot[r] > tau) { owner = r; base = cum; break; }
-                cum += tot[r];
-            }
-            if (owner < 0) {  // tau >= W (u >= 1 or rounding): largest j with w_j > 0
+            const unsigned hit = __ballot_sync(0xffffffffu, lane < p.csize && incl > tau);
+            if (hit) {
+                owner = __ffs(hit) - 1;
+                base = __shfl_sync(0xffffffffu, incl - tot, owner);
+            } else {  // tau >= W (u >= 1 or rounding): largest j with w_j > 0
                 mode = 1;
-                for (int r = p.csize - 1; r >= 0; --r)
-                    if (tot[r] > 0.0) { owner = r; break; }
+                const unsigned pos = __ballot_sync(0xffffffffu, lane < p.csize && tot > 0.0);
+                owner = 31 - __clz(pos);
             }
         } else {
             mode = 2;
             owner = 0;
         }
-        s_owner = owner; s_mode = mode; s_tau = tau; s_W = W; s_base = base;
+        int tile = -1;
+        if (rank == owner) {
+            // sub-tile holding tau: each lane owns a run of consecutive sub-tiles
+            const int per = (nsub + 31) / 32;
+            const int s_lo = min(nsub, lane * per), s_hi = min(nsub, s_lo + per);
+            double mine = 0.0;
+            for (int s2 = s_lo; s2 < s_hi; ++s2) mine += double(s_sub[s2]);
+            const double excl = base + warp_incl_scan_f64(mine) - mine;
+            if (mode == 0) {
+                const unsigned hit = __ballot_sync(0xffffffffu, excl <= tau && excl + mine > tau);
+                if (hit) {
+                    const int l = __ffs(hit) - 1;
+                    if (lane == l) {
+                        double c = excl;
+                        for (int s2 = s_lo; s2 < s_hi; ++s2) {
+                            if (c + double(s_sub[s2]) > tau) { tile = s2; break; }
+                            c += double(s_sub[s2]);
+                        }
+                        base = c;
+                        if (tile < 0) { tile = s_hi - 1; base = c - double(s_sub[s_hi - 1]); }
+                    }
+                    tile = __shfl_sync(0xffffffffu, tile, l);
+                    base = __shfl_sync(0xffffffffu, base, l);
+                } else {
+                    mode = 1;
+                }
+            }
+            if (mode == 1) {  // the last sub-tile with positive mass
+                int last = -1;
+                for (int s2 = s_lo; s2 < s_hi; ++s2)
+                    if (s_sub[s2] > 0.f) last = s2;
+                for (int o = 16; o > 0; o >>= 1) last = max(last, __shfl_xor_sync(0xffffffffu, last, o));
+                tile = last;
+            }
+        }
+        if (lane == 0) { s_owner = owner; s_mode = mode; s_tau = tau; s_W = W; s_base = base; s_tile = tile; }
     }
     __syncthreads();
     if (p.csize > 1) cluster_arrive();  // done reading the other CTAs' shared memory
 
-    if (rank == s_owner) {
+    if (rank == s_owner && warp == 0) {
         const double tau = s_tau, W = s_W;
-        int mode = s_mode;
-        if (mode == 0 && tid == 0) {  // tile holding tau inside this span
-            double cum = s_base;
-            int tsel = -1;
-            for (int t = 0; t < ntiles; ++t) {
-                if (cum + s_tiles[t] > tau) { tsel = t; break; }
-                cum += s_tiles[t];
-            }
-            s_tile = tsel;
-            s_base = cum;
-            if (tsel < 0) s_mode = 1;
-        }
-        __syncthreads();
-        mode = s_mode;
-        if (mode == 0) {
-            // pass 2: fp64 scan of the selected tile
-            const int tile = s_tile;
+        const int mode = s_mode, s = s_tile;
+        if (mode == 0 || mode == 1) {
             float w[kW];
-            tile_weights(tile, w);
-            double mine = 0.0;
+            {
+                Raw r;
+                if (s >= 0) load_sub(s, r);
+                else { r.t = ninf_raw<In>(); r.z = r.t; }
+                sub_weights(r, w);
+            }
+            const int j0 = e0 + max(s, 0) * kSub + lane * kW;
+            bool done = false;
+            if (mode == 0) {
+                // fp64 scan of the sub-tile across the warp, then within the lane
+                double mine = 0.0;
 #pragma unroll
-            for (int e = 0; e < kW; ++e) mine += double(w[e]);
-            double tile_total;
-            const double excl = s_base + block_exclusive_scan<kFinThreads>(mine, red_d, &tile_total);
-            if (tid == 0) s_found = 0;
-            __syncthreads();
-            if (excl <= tau && excl + mine > tau) {
-                double C = excl;
-                const int j0 = e0 + tile * kTile + tid * kW;
-                for (int e = 0; e < kW; ++e) {
-                    const double Cprev = C;
-                    C += double(w[e]);
-                    if (C > tau) {
-                        out[a] = j0 + e;
-                        if (p.diag_gap) p.diag_gap[b] = float(fmin(C - tau, tau - Cprev) / W);
-                        atomicExch(&s_found, 1);
-                        break;
+                for (int e = 0; e < kW; ++e) mine += double(w[e]);
+                double incl = mine;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const double y = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += y;
+                }
+                const double excl = s_base + incl - mine;
+                const bool hit = excl <= tau && excl + mine > tau;
+                if (hit) {
+                    double C = excl;
+                    for (int e = 0; e < kW; ++e) {
+                        const double Cprev = C;
+                        C += double(w[e]);
+                        if (C > tau) {
+                            out[a] = j0 + e;
+                            if (p.diag_gap) p.diag_gap[b] = float(fmin(C - tau, tau - Cprev) / W);
+                            break;
+                        }
                     }
                 }
+                done = __any_sync(0xffffffffu, hit);
             }
-            __syncthreads();
-            if (!s_found) mode = 1;  // rounding between the two passes: fall through
-        }
-        if (mode == 1) {
-            // largest j of this span with w_j > 0
-            int best = -1;
-            float wbest = 0.f;
-            for (int tile = 0; tile < ntiles; ++tile) {
-                float w[kW];
-                tile_weights(tile, w);
-                const int j0 = e0 + tile * kTile + tid * kW;
+            if (!done) {
+                // largest j of the sub-tile with w_j > 0 (rounding fallback)
+                int best = -1;
+                float wbest = 0.f;
 #pragma unroll
                 for (int e = 0; e < kW; ++e)
-                    if (w[e] > 0.f && j0 + e > best) { best = j0 + e; wbest = w[e]; }
-            }
-            const int jb = block_reduce<kFinThreads>(best, [](int x, int z) { return max(x, z); }, red_i);
-            if (jb >= 0 && best == jb) {
-                out[a] = jb;
-                if (p.diag_gap) {
-                    const double g1 = W - tau, g0 = tau - (W - double(wbest));
-                    p.diag_gap[b] = float(fmin(g1, g0) / W);
+                    if (w[e] > 0.f) { best = j0 + e; wbest = w[e]; }
+                int jb = best;
+                for (int o = 16; o > 0; o >>= 1) jb = max(jb, __shfl_xor_sync(0xffffffffu, jb, o));
+                if (jb >= 0 && best == jb) {
+                    out[a] = jb;
+                    if (p.diag_gap) {
+                        const double g1 = W - tau, g0 = tau - (W - double(wbest));
+                        p.diag_gap[b] = float(fmin(g1, g0) / W);
+                    }
+                } else if (jb < 0 && lane == 0) {
+                    out[a] = e0;  // no positive entry found: cannot happen when W > 0
                 }
             }
-        } else if (mode == 2) {
+        } else {
             // no residual mass at all: argmax of p_a over the whole row
             MaxIdx acc{kNegInf, INT_MAX};
-            for (int j = tid; j < V; j += kFinThreads) {
+            for (int j = lane; j < V; j += 32) {
                 const float t = E::load(trow + j);
                 if (t > acc.m) { acc.m = t; acc.i = j; }
             }
-            acc = block_reduce<kFinThreads>(acc, merge_mi, red_mi);
-            if (tid == 0) {
+            acc = warp_reduce(acc, [](MaxIdx x, MaxIdx y) { return merge_mi(x, y); });
+            if (lane == 0) {
                 out[a] = (acc.i == INT_MAX) ? 0 : acc.i;
                 if (p.diag_gap) p.diag_gap[b] = __int_as_float(0x7fc00000);
             }
@@ -471,7 +628,10 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
 }
 
 // ------------------------------------------------------------------ host
-static int verify_slices(int V) { return (V + kStatSlice - 1) / kStatSlice; }
+static int verify_slices(int B, int k, int V) {
+    const int len = verify_slice_len(B, k);
+    return (V + len - 1) / len;
+}
 
 static void finalize_shape(int V, int* csize, int* span) {
     int c = (V + 4095) / 4096;
@@ -490,7 +650,8 @@ static osd_status launch_verify(const void* draft, const void* target, int B, in
                                 float* diag_margin, float* diag_gap, RowStat* stats,
                                 cudaStream_t stream) {
     const bool greedy = (T == 0.f);
-    const int n_slices = verify_slices(V);
+    const int slice_len = verify_slice_len(B, k);
+    const int n_slices = verify_slices(B, k, V);
     const long long n_draft_rows = greedy ? 0 : (long long)B * k;
     const long long rows = n_draft_rows + (long long)B * (k + 1);
     float c_hi = 0.f, c_lo = 0.f;
@@ -502,11 +663,11 @@ static osd_status launch_verify(const void* draft, const void* target, int B, in
     if (greedy)
         e = launch(row_stats_kernel<In, true>, dim3(unsigned(grid1)), dim3(kStatThreads), 0, stream, 1,
                    static_cast<const In*>(draft), static_cast<const In*>(target), n_draft_rows, V,
-                   n_slices, c_hi, c_lo, stats);
+                   slice_len, n_slices, c_hi, c_lo, stats);
     else
         e = launch(row_stats_kernel<In, false>, dim3(unsigned(grid1)), dim3(kStatThreads), 0, stream, 1,
                    static_cast<const In*>(draft), static_cast<const In*>(target), n_draft_rows, V,
-                   n_slices, c_hi, c_lo, stats);
+                   slice_len, n_slices, c_hi, c_lo, stats);
     if (e != cudaSuccess) return OSD_ERR_CUDA;
 
     FinParams fp;
@@ -522,10 +683,13 @@ static osd_status launch_verify(const void* draft, const void* target, int B, in
     const bool vec = !greedy && aligned_to(draft, 16) && aligned_to(target, 16) &&
                      ((size_t)V * sizeof(In)) % 16 == 0;
     const dim3 grid2(unsigned(B) * unsigned(csize));
+    const int sub = 32 * (vec ? Elem<In>::kVec : 1);
+    const size_t smem2 = greedy ? 0 : size_t((span + sub - 1) / sub) * sizeof(float);
+    if (smem2 > size_t(kFinMaxSub) * sizeof(float)) return OSD_ERR_UNSUPPORTED;
     if (vec)
-        e = launch(verify_finalize_kernel<In, true>, grid2, dim3(kFinThreads), 0, stream, csize, fp);
+        e = launch(verify_finalize_kernel<In, true>, grid2, dim3(kFinThreads), smem2, stream, csize, fp);
     else
-        e = launch(verify_finalize_kernel<In, false>, grid2, dim3(kFinThreads), 0, stream, csize, fp);
+        e = launch(verify_finalize_kernel<In, false>, grid2, dim3(kFinThreads), smem2, stream, csize, fp);
     return from_cuda(e);
 }
 
@@ -537,7 +701,7 @@ extern "C" osd_status osd_verify_workspace_size(int B, int k, int V, size_t* byt
     if (!bytes || B < 0 || k < 1 || V < 1) return OSD_ERR_INVALID_ARG;
     if (k > OSD_VERIFY_MAX_K || V > OSD_VERIFY_MAX_V) return OSD_ERR_UNSUPPORTED;
     const size_t rows = size_t(B) * size_t(2 * k + 1);
-    size_t need = rows * size_t(osd::verify_slices(V)) * sizeof(RowStat);
+    size_t need = rows * size_t(osd::verify_slices(B, k, V)) * sizeof(RowStat);
     need = (need + 255) / 256 * 256;
     *bytes = need < 256 ? 256 : need;
     return OSD_OK;
