@@ -35,6 +35,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "verified positions/s and distilled positions/s at V=32000; % of HBM peak"
+SLEEP_CYCLES = 200_000  # ~0.1 ms of device time ahead of each timed step
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -88,7 +89,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", "20"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.thread = threading.Thread(target=self._read, daemon=True)
             self.thread.start()
         except Exception:
@@ -200,6 +201,9 @@ def run_ours(args):
 
     def step(record):
         l2_flush.zero_()
+        # keep the device busy while the host enqueues the step, so that host-side
+        # launch overhead never shows up inside the timed events
+        torch.cuda._sleep(SLEEP_CYCLES)
         e = [ev() for _ in range(1 + n_ver + len(kinds))]
         e[0].record(stream)
         osd.osd_verify(v["draft"], v["target"], v["tokens"], v["uniforms"], sv.temperature,

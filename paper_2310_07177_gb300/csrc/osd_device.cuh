@@ -279,14 +279,20 @@ __device__ __forceinline__ uint32_t cluster_rank() {
     return r;
 }
 // The .aligned forms need a converged warp, hence the __syncwarp() first.
-__device__ __forceinline__ void cluster_sync() {
+// Arrive without ordering: used once this CTA has consumed every value it read
+// from its peers' shared memory, to tell them they may exit.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
     __syncwarp();
-    asm volatile("barrier.cluster.arrive.release.aligned;\n"
-                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
-__device__ __forceinline__ void cluster_arrive() {
+// Cluster barrier that publishes shared-memory writes made by the calling
+// threads with `writer` set: only they fence, everyone else arrives relaxed,
+// and the wait acquires, so the peers see those writes afterwards.
+__device__ __forceinline__ void cluster_sync_publish(bool writer) {
+    if (writer) asm volatile("fence.acq_rel.cluster;" ::: "memory");
     __syncwarp();
-    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;\n"
+                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 __device__ __forceinline__ void cluster_wait() {
     __syncwarp();

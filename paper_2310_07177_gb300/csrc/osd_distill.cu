@@ -138,11 +138,12 @@ __device__ __forceinline__ float rescale(float m, float mb) {
 
 template <typename In, int kKind, bool kAligned>
 __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
-    // JSD and TVD clamp both rows to -1e30: a zero probability then stays exactly 0
-    // and every logit difference finite, so no entry needs a guard.  FKL and RKL
-    // keep -inf (their loss is +inf when one row has mass where the other has
-    // none) and guard only the 16-byte chunks that hold a -inf.
-    constexpr bool kClamp = kKind == OSD_JSD || kKind == OSD_TVD;
+    // JSD clamps both rows to -1e30: a zero probability then stays exactly 0 and
+    // every logit difference finite, so no entry needs a guard.  TVD needs none
+    // either: a -inf gives p or q = 0, and the sign it picks multiplies q = 0.
+    // FKL and RKL keep -inf (their loss is +inf when one row has mass where the
+    // other has none) and guard only the 16-byte chunks that hold a -inf.
+    constexpr bool kClamp = kKind == OSD_JSD;
     constexpr bool kClampZ = kClamp, kClampT = kClamp;
     constexpr bool kMoment = kKind == OSD_FKL || kKind == OSD_RKL;
     extern __shared__ __align__(128) unsigned char dsm[];
@@ -272,7 +273,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     }
     // cluster merge: warp 0 gathers every CTA's partial (lane r <- CTA r) and reduces
     // it in a fixed order, so all CTAs of the row hold bit-identical statistics
-    if (csize > 1) cluster_sync(); else __syncthreads();
+    if (csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
     if (tid < 32) {
         Stats1 o{kNegInf, 0.f, kNegInf, 0.f, 0.f, 0};
         if (tid < csize) {
@@ -322,6 +323,8 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     const bool has_ninf = (st.err & 2) != 0;  // some logit of the row is -inf
     const float cu = s_cu, cv = s_cv;
     const float2 mt2 = f2(st.mt), mz2 = f2(st.mz);
+    auto log2p = [&](float2 x) { return fma2(sub2(x, mt2), f2(kLog2e), f2(cu)); };
+    auto log2q = [&](float2 x) { return fma2(sub2(x, mz2), f2(kLog2e), f2(cv)); };
     float loss = s_loss;
 
     const float beta = p.beta;
@@ -337,16 +340,15 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
 #pragma unroll
                 for (int e = 0; e < kCnt; e += 2) {
                     const bool two = (e + 1 < kCnt);
-                    const float2 u = fma2(sub2(make_float2(t[e], two ? t[e + 1] : t[e]), mt2), f2(kLog2e), f2(cu));
-                    const float2 v = fma2(sub2(make_float2(z[e], two ? z[e + 1] : z[e]), mz2), f2(kLog2e), f2(cv));
+                    const float2 u = log2p(make_float2(t[e], two ? t[e + 1] : t[e]));  // log2 p
+                    const float2 v = log2q(make_float2(z[e], two ? z[e + 1] : z[e]));  // log2 q
                     const float2 d = sub2(v, u);
                     float2 a, b;
                     if (kKind == OSD_TVD) {
                         const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
                         const float2 df = sub2(pj, qj);
                         a = make_float2(fabsf(df.x), fabsf(df.y));
-                        b = make_float2((d.x > 0.f) ? qj.x : ((d.x < 0.f) ? -qj.x : 0.f),
-                                        (d.y > 0.f) ? qj.y : ((d.y < 0.f) ? -qj.y : 0.f));
+                        b = make_float2(copysignf(qj.x, d.x), copysignf(qj.y, d.y));  // q sign(q - p)
                     } else {
                         float r[2][2];
                         const float uu[2] = {u.x, u.y}, vv[2] = {v.x, v.y}, dd[2] = {d.x, d.y};
@@ -374,7 +376,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         }
         const float3 bs = block_sum3(A2.x + A2.y, B2.x + B2.y, 0.f, red_s);
         if (tid == 0) s2_mine = Stats2{bs.x, bs.y};
-        if (csize > 1) cluster_sync(); else __syncthreads();
+        if (csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
         if (tid < 32) {
             float a = 0.f, b = 0.f;
             if (tid < csize) {
@@ -402,7 +404,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
             loss = jsd_trivial ? 0.f : kLn2 * (beta * s2.a + (1.f - beta) * s2.b);
         }
     }
-    if (csize > 1) cluster_arrive();  // finished reading the other CTAs' shared memory
+    if (csize > 1) cluster_arrive_relaxed();  // finished reading the other CTAs' shared memory
 
     if (rank == 0 && tid == 0) {
         p.loss[row] = row_err ? __int_as_float(0x7fc00000) : loss;
@@ -423,11 +425,11 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                 const bool two = (e + 1 < kCnt);
                 const float2 zz = make_float2(z[e], two ? z[e + 1] : z[e]);
                 const float2 tt = make_float2(t[e], two ? t[e + 1] : t[e]);
-                const float2 v = fma2(sub2(zz, mz2), f2(kLog2e), f2(cv));
+                const float2 v = log2q(zz);
                 const float2 qj = make_float2(ex2(v.x), ex2(v.y));
                 float2 gg;
                 if (kKind == OSD_FKL) {
-                    const float2 u = fma2(sub2(tt, mt2), f2(kLog2e), f2(cu));
+                    const float2 u = log2p(tt);
                     gg = sub2(qj, make_float2(ex2(u.x), ex2(u.y)));
                 } else if (kKind == OSD_RKL) {
                     gg = mul2(qj, sub2(sub2(zz, tt), f2(K)));
@@ -436,15 +438,14 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                         if (!(qj.y > 0.f)) gg.y = 0.f;
                     }
                 } else if (kKind == OSD_TVD) {
-                    const float2 d = sub2(v, fma2(sub2(tt, mt2), f2(kLog2e), f2(cu)));
-                    const float2 sg = make_float2((d.x > 0.f) ? 0.5f : ((d.x < 0.f) ? -0.5f : 0.f),
-                                                  (d.y > 0.f) ? 0.5f : ((d.y < 0.f) ? -0.5f : 0.f));
+                    const float2 d = sub2(v, log2p(tt));
+                    const float2 sg = make_float2(copysignf(0.5f, d.x), copysignf(0.5f, d.y));
                     gg = mul2(qj, sub2(sg, f2(s2.b)));
                 } else {
                     if (jsd_trivial) {
                         gg = f2(0.f);
                     } else {
-                        const float2 d = sub2(v, fma2(sub2(tt, mt2), f2(kLog2e), f2(cu)));
+                        const float2 d = sub2(v, log2p(tt));
                         const float dd[2] = {d.x, d.y};
                         float l2mq[2];
 #pragma unroll

@@ -448,12 +448,33 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
             r.z = pack_raw<In, kW>(zv);
         }
     };
+    // residual weights of one sub-tile slot, two entries per packed f32x2 step
+    // (the same operations as `weight`, so both passes round identically)
     auto sub_weights = [&](const Raw& r, float* w) {
         float tv[kW], zv[kW];
         unpack_raw<In, kW>(r.t, tv);
         unpack_raw<In, kW>(r.z, zv);
+        if constexpr (kW == 1) {
+            w[0] = weight(tv[0], zv[0]);
+        } else {
 #pragma unroll
-        for (int e = 0; e < kW; ++e) w[e] = weight(tv[e], zv[e]);
+            for (int e = 0; e < kW; e += 2) {
+                const float2 dt = sub2(make_float2(tv[e], tv[e + 1]), f2(mt));
+                const float2 at = fma2(dt, f2(ch), mul2(dt, f2(cl)));
+                const float2 pj = mul2(make_float2(ex2(at.x), ex2(at.y)), f2(inv_st));
+                if (bonus) {
+                    w[e] = pj.x;
+                    w[e + 1] = pj.y;
+                } else {
+                    const float2 dz = sub2(make_float2(zv[e], zv[e + 1]), f2(mz));
+                    const float2 az = fma2(dz, f2(ch), mul2(dz, f2(cl)));
+                    const float2 qj = mul2(make_float2(ex2(az.x), ex2(az.y)), f2(inv_sz));
+                    const float2 df = sub2(pj, qj);
+                    w[e] = fmaxf(df.x, 0.f);
+                    w[e + 1] = fmaxf(df.y, 0.f);
+                }
+            }
+        }
     };
 
     // pass 1: one fp32 sum per sub-tile, reduced inside the warp, no block barrier
@@ -484,7 +505,7 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
         part = warp_sum_f64(part);
         if (lane == 0) s_span_total = part;
     }
-    if (p.csize > 1) cluster_sync(); else __syncthreads();
+    if (p.csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
 
     // warp 0 of every CTA derives W, tau and the owning CTA identically: lane r
     // holds CTA r's total, an fp64 warp scan gives the prefix in rank order
@@ -549,7 +570,7 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
         if (lane == 0) { s_owner = owner; s_mode = mode; s_tau = tau; s_W = W; s_base = base; s_tile = tile; }
     }
     __syncthreads();
-    if (p.csize > 1) cluster_arrive();  // done reading the other CTAs' shared memory
+    if (p.csize > 1) cluster_arrive_relaxed();  // done reading the other CTAs' shared memory
 
     if (rank == s_owner && warp == 0) {
         const double tau = s_tau, W = s_W;
