@@ -136,6 +136,83 @@ __device__ __forceinline__ float rescale(float m, float mb) {
     return (m == kNegInf) ? 0.f : ex2((m - mb) * kLog2e);
 }
 
+// TVD keeps q' = q sign(q - p) (fp32) in the two 16-bit (bf16) or the first
+// 32-bit (fp32) staging slots of each entry once pass 2 has read its logits.
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+    uint32_t d;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
+    return d;
+}
+template <typename In, int kCnt>
+__device__ __forceinline__ void store_q(In* zs, In* ts, int j0, const float* q) {
+    if constexpr (sizeof(In) == 4) {
+        if constexpr (kCnt == 4) {
+            *reinterpret_cast<float4*>(zs + j0) = make_float4(q[0], q[1], q[2], q[3]);
+        } else {
+#pragma unroll
+            for (int e = 0; e < kCnt; ++e) reinterpret_cast<float*>(zs)[j0 + e] = q[e];
+        }
+    } else if constexpr (kCnt == 8) {
+        uint32_t hz[4], ht[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const uint32_t a = __float_as_uint(q[2 * i]), b = __float_as_uint(q[2 * i + 1]);
+            hz[i] = prmt(a, b, 0x7632);  // high halves
+            ht[i] = prmt(a, b, 0x5410);  // low halves
+        }
+        *reinterpret_cast<uint4*>(zs + j0) = make_uint4(hz[0], hz[1], hz[2], hz[3]);
+        *reinterpret_cast<uint4*>(ts + j0) = make_uint4(ht[0], ht[1], ht[2], ht[3]);
+    } else {
+#pragma unroll
+        for (int e = 0; e < kCnt; ++e) {
+            const uint32_t a = __float_as_uint(q[e]);
+            reinterpret_cast<unsigned short*>(zs)[j0 + e] = static_cast<unsigned short>(a >> 16);
+            reinterpret_cast<unsigned short*>(ts)[j0 + e] = static_cast<unsigned short>(a & 0xffffu);
+        }
+    }
+}
+template <typename In>
+__device__ __forceinline__ float load_q(const In* zs, const In* ts, int j) {
+    if constexpr (sizeof(In) == 4) {
+        return reinterpret_cast<const float*>(zs)[j];
+    } else {
+        const uint32_t hi = reinterpret_cast<const unsigned short*>(zs)[j];
+        const uint32_t lo = reinterpret_cast<const unsigned short*>(ts)[j];
+        return __uint_as_float((hi << 16) | lo);
+    }
+}
+template <typename In, bool kAligned>
+__device__ __forceinline__ void tvd_gradient(const In* zs, const In* ts, int n, float G, float* orow) {
+    const int tid = threadIdx.x;
+    auto g_of = [G](float q) { return fmaf(-fabsf(q), G, 0.5f * q); };
+    if constexpr (kAligned) {
+        constexpr int kVec = Elem<In>::kVec;
+        const int nv = n / kVec;
+        for (int v = tid; v < nv; v += kDistThreads) {
+            float q[kVec];
+            if constexpr (sizeof(In) == 4) {
+                const float4 f = *reinterpret_cast<const float4*>(zs + v * kVec);
+                q[0] = f.x; q[1] = f.y; q[2] = f.z; q[3] = f.w;
+            } else {
+                const uint4 hz = lds_v4(zs + v * kVec), ht = lds_v4(ts + v * kVec);
+                const uint32_t zw[4] = {hz.x, hz.y, hz.z, hz.w}, tw[4] = {ht.x, ht.y, ht.z, ht.w};
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    q[2 * i] = __uint_as_float(prmt(tw[i], zw[i], 0x5410));
+                    q[2 * i + 1] = __uint_as_float(prmt(tw[i], zw[i], 0x7632));
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < kVec; e += 4)
+                stg_v4(orow + v * kVec + e, g_of(q[e]), g_of(q[e + 1]), g_of(q[e + 2]), g_of(q[e + 3]));
+        }
+        const int r0 = nv * kVec;
+        if (tid < n - r0) orow[r0 + tid] = g_of(load_q(zs, ts, r0 + tid));
+    } else {
+        for (int e = tid; e < n; e += kDistThreads) orow[e] = g_of(load_q(zs, ts, e));
+    }
+}
+
 template <typename In, int kKind, bool kAligned>
 __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     // JSD clamps both rows to -1e30: a zero probability then stays exactly 0 and
@@ -335,8 +412,9 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         float2 A2 = f2(0.f), B2 = f2(0.f);
         if (!row_err && !jsd_trivial) {
             sweep<In, kAligned, kClampZ, kClampT, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
-                                                                        int, float, float, bool) {
+                                                                        int j0, float, float, bool) {
                 constexpr int kCnt = decltype(tag)::value;
+                float qs[kCnt];  // TVD: q sign(q - p), kept for pass 3
 #pragma unroll
                 for (int e = 0; e < kCnt; e += 2) {
                     const bool two = (e + 1 < kCnt);
@@ -349,6 +427,8 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                         const float2 df = sub2(pj, qj);
                         a = make_float2(fabsf(df.x), fabsf(df.y));
                         b = make_float2(copysignf(qj.x, d.x), copysignf(qj.y, d.y));  // q sign(q - p)
+                        qs[e] = b.x;
+                        if (e + 1 < kCnt) qs[e + 1] = b.y;
                     } else {
                         float r[2][2];
                         const float uu[2] = {u.x, u.y}, vv[2] = {v.x, v.y}, dd[2] = {d.x, d.y};
@@ -372,6 +452,8 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                     A2 = add2(A2, a);
                     B2 = add2(B2, b);
                 }
+                // the logits of these entries are not needed again: their slots take q'
+                if constexpr (kKind == OSD_TVD) store_q<In, kCnt>(zs, ts, j0, qs);
             });
         }
         const float3 bs = block_sum3(A2.x + A2.y, B2.x + B2.y, 0.f, red_s);
@@ -412,7 +494,10 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     }
 
     // ---- pass 3: d loss / d draft logits of the span
-    if (!row_err) {
+    if (kKind == OSD_TVD && !row_err) {
+        // g = q (sign(q - p)/2 - G) = q'/2 - |q'| G from the stored q'
+        tvd_gradient<In, kAligned>(zs, ts, n, s2.b, p.dlogits + row * V + e0);
+    } else if (kKind != OSD_TVD && !row_err) {
         float* orow = p.dlogits + row * V + e0;
         const float K = s_K;
         const float jsd_scale = (1.f - beta) * kLn2;
