@@ -129,24 +129,48 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+# ----------------------------------------------------------------------------- ranks
+def job_time_ms(local_ms: float, device=None) -> float:
+    """Whole-job time: the slowest rank's timed total (max over ranks; the
+    identity when torch.distributed is not initialised)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(local_ms)
+    t = torch.tensor([float(local_ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(positions_per_rank: int, world: int, ms_per_step: float) -> float:
+    """Positions per second over all ranks: every rank processes its own shard
+    of the same size in the time of the slowest one (weak scaling)."""
+    return world * positions_per_rank / (ms_per_step / 1e3)
+
+
 # ----------------------------------------------------------------------------- workloads
-def _setup_serving_32k(dev, distill_rows=None):
+def shard_seed(base_seed: int, rank: int) -> int:
+    """Each rank draws its own shard of sequences / rows (weak scaling, no overlap)."""
+    return base_seed + 7919 * rank
+
+
+def _setup_serving_32k(dev, distill_rows=None, rank=0):
     import dataclasses
 
     from paper_2310_07177_gb300 import workloads as W
     spec_v, spec_d = W.VERIFY[2], W.DISTILL[4]
     if distill_rows:
         spec_d = dataclasses.replace(spec_d, N=distill_rows)
-    v = W.verify_inputs(spec_v, seed=W.seed_for(2), device=dev)
-    d = W.distill_inputs(spec_d, seed=W.seed_for(4), device=dev)
+    v = W.verify_inputs(spec_v, seed=shard_seed(W.seed_for(2), rank), device=dev)
+    d = W.distill_inputs(spec_d, seed=shard_seed(W.seed_for(4), rank), device=dev)
     return {"v": v, "d": d, "spec_v": spec_v, "spec_d": spec_d,
             "desc": "serving-32k: verify B=32 k=5 V=32000 bf16 T=1.0 + greedy T=0 pass; "
                     f"distill flush N={spec_d.N} V=32000 bf16 reverse-KL + TVD"}
 
 
-def _setup_large_vocab(dev):
+def _setup_large_vocab(dev, rank=0):
     from paper_2310_07177_gb300 import workloads as W
-    v = W.verify_inputs(W.VERIFY[5], seed=W.seed_for(5), device=dev)
+    v = W.verify_inputs(W.VERIFY[5], seed=shard_seed(W.seed_for(5), rank), device=dev)
     return {"v": v, "spec_v": W.VERIFY[5],
             "desc": "large-vocab: verify B=256 k=8 V=128256 bf16 T=0.7 -> forward-KL distill of "
                     "the mismatch rows against target[:, :k]"}
@@ -173,7 +197,8 @@ def run_ours(args):
     osd.load_library()
 
     wl = args.workload
-    setup = _setup_serving_32k(dev, args.distill_rows) if wl == "serving-32k" else _setup_large_vocab(dev)
+    setup = (_setup_serving_32k(dev, args.distill_rows, rank) if wl == "serving-32k"
+             else _setup_large_vocab(dev, rank))
     stream = torch.cuda.current_stream(dev)
     v = setup["v"]
     sv = setup["spec_v"]
@@ -252,11 +277,7 @@ def run_ours(args):
     else:
         dist_ms = [r[1].elapsed_time(r[2]) for r in recs]
         n_active = int(vout.mismatch_mask.sum().item())
-    total_ms = sum(step_ms)
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = t.item()
+    total_ms = job_time_ms(sum(step_ms), dev if world > 1 else None)
     ms_step = total_ms / args.steps
 
     if wl == "serving-32k":
@@ -271,7 +292,7 @@ def run_ours(args):
         launches = 2 + 1
         bytes_v = _bytes_verify(sv.B, sv.k, sv.V, s_in, False)
         dist_bytes = n_active * sv.V * (2 * s_in + 4)
-    value = world * positions / (ms_step / 1e3)
+    value = job_throughput(positions, world, ms_step)
     peak, peak_src = _peak_hbm()
     avg_dist = statistics.mean(dist_ms)
     avg_ver = statistics.mean(verify_ms)
