@@ -52,12 +52,14 @@ typedef enum osd_status {
 
 typedef enum osd_dtype { OSD_F32 = 0, OSD_BF16 = 1 } osd_dtype;
 
-/* Distances of Eq. 3 (Section 4.1) plus total variation distance. */
+/* Distances of Eq. 3 (Section 4.1), total variation distance, and the
+ * label fine-tuning baseline of Table 1 (FT). */
 typedef enum osd_loss {
     OSD_FKL = 0,  /* KL(p || q)                                               */
     OSD_RKL = 1,  /* KL(q || p)                                               */
     OSD_JSD = 2,  /* beta KL(p || m) + (1 - beta) KL(q || m), m = beta p + (1-beta) q */
-    OSD_TVD = 3   /* 1/2 sum |p - q|                                          */
+    OSD_TVD = 3,  /* 1/2 sum |p - q|                                          */
+    OSD_CE = 4    /* -log q(y*), y* = argmax of the target logits (lowest index on ties) */
 } osd_loss;
 
 /* Largest vocabulary osd_verify accepts. */
@@ -68,7 +70,8 @@ typedef enum osd_loss {
 /* Human-readable name of a status code (static string, never NULL). */
 const char *osd_status_string(osd_status status);
 
-/* ABI version of this library: (major << 16) | minor. */
+/* ABI version of this library: (major << 16) | minor.  2.0 added the
+ * temperature argument of osd_distill and the OSD_CE loss. */
 int osd_abi_version(void);
 
 /*
@@ -153,19 +156,22 @@ osd_status osd_verify_noalloc(const void *draft_logits, const void *target_logit
                               float *diag_margin, float *diag_cdf_gap, void *stream);
 
 /*
- * Per-position distillation loss and gradient (Eq. 2-3, Section 4.1), at
- * temperature 1, over rows laid out as [G, P, V] with element strides
- * (the [N, V] case is G = N, P = 1, d_stride_g = t_stride_g = V).
- * q = softmax(draft row), p = softmax(target row).
+ * Per-position distillation loss and gradient (Eq. 2-3, Section 4.1) over
+ * rows laid out as [G, P, V] with element strides (the [N, V] case is G = N,
+ * P = 1, d_stride_g = t_stride_g = V).  q = softmax(draft row / tau),
+ * p = softmax(target row / tau), tau = `temperature` (Section 4.1's tunable
+ * softmax temperature; 1 is the plain softmax).
  *
  * draft_logits, target_logits  row (g, p) starts at base + g*stride_g +
  *                p*stride_p elements; the V entries of a row are contiguous.
  * mask           [G, P] uint8, nullable (NULL = every row active).
  * kind, beta     the distance; beta in [0, 1] is used by OSD_JSD only.
+ * temperature    tau > 0 and finite, else OSD_ERR_INVALID_ARG.
  * loss           [G, P] fp32 out: the per-position loss (the 1/n_B batch
  *                mean of Eq. 2 is left to the caller); 0 for inactive rows.
- * dlogits        [G, P, V] fp32 contiguous out: d loss / d draft logits,
- *                unscaled; rows of inactive positions are NOT written.
+ * dlogits        [G, P, V] fp32 contiguous out: d loss / d draft logits
+ *                (the raw logits, so including the factor 1/tau), unscaled
+ *                by any batch size; rows of inactive positions are NOT written.
  * status         nullable device int32: set to 0 by this call, then to
  *                OSD_ERR_TIMEOUT if a bounded wait for a bulk copy gave up
  *                (that row's loss is then NaN and its gradient not written).
@@ -177,7 +183,7 @@ osd_status osd_distill(const void *draft_logits, const void *target_logits,
                        osd_dtype dtype, int G, int P, int V,
                        int64_t d_stride_g, int64_t d_stride_p,
                        int64_t t_stride_g, int64_t t_stride_p,
-                       const uint8_t *mask, osd_loss kind, float beta,
+                       const uint8_t *mask, osd_loss kind, float beta, float temperature,
                        float *loss, float *dlogits, int32_t *status, void *stream);
 
 #ifdef __cplusplus

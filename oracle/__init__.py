@@ -22,7 +22,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "osd_oracle.c")
 LIB_PATH = os.path.join(_HERE, "libosd_oracle.so")
 
-LOSS_KINDS = {"fkl": 0, "rkl": 1, "jsd": 2, "tvd": 3}
+LOSS_KINDS = {"fkl": 0, "rkl": 1, "jsd": 2, "tvd": 3, "ce": 4}
 
 _lib = None
 _lock = threading.Lock()
@@ -68,7 +68,7 @@ def _load():
                                           i32p, i32p, u8p, dp, dp, dp]
         lib.osd_oracle_distill.restype = ctypes.c_int
         lib.osd_oracle_distill.argtypes = [dp, dp, L, L, u8p, ctypes.c_int,
-                                           ctypes.c_double, dp, dp]
+                                           ctypes.c_double, ctypes.c_double, dp, dp]
         lib.osd_oracle_log_softmax.restype = None
         lib.osd_oracle_log_softmax.argtypes = [dp, L, ctypes.c_double, dp]
         _lib = lib
@@ -137,8 +137,10 @@ def verify(draft_logits, target_logits, draft_tokens, uniforms, temperature):
 
 
 def distill(draft_logits, target_logits, mask=None, loss_kind="fkl", beta=0.5,
-            dlogits_init=None):
-    """Per-position distillation loss and d loss / d draft_logits (Eq. 2-3).
+            dlogits_init=None, temperature=1.0):
+    """Per-position distillation loss and d loss / d draft_logits (Eq. 2-3),
+    both softmaxes at ``temperature`` (Section 4.1); ``loss_kind`` "ce" is the
+    label fine-tuning cross-entropy to the target argmax.
 
     draft_logits, target_logits [N, V] (any leading shape is flattened to
     rows); mask [N] of 0/1 or None.  Returns (loss [N], dlogits [N, V]) in
@@ -163,7 +165,7 @@ def distill(draft_logits, target_logits, mask=None, loss_kind="fkl", beta=0.5,
     kind = LOSS_KINDS[loss_kind] if isinstance(loss_kind, str) else int(loss_kind)
     rc = lib.osd_oracle_distill(_ptr(z, ctypes.c_double), _ptr(t, ctypes.c_double), N, V,
                                 None if m is None else _ptr(m, ctypes.c_uint8),
-                                kind, float(beta), _ptr(loss, ctypes.c_double),
+                                kind, float(beta), float(temperature), _ptr(loss, ctypes.c_double),
                                 _ptr(g, ctypes.c_double))
     if rc != 0:
         raise ValueError("osd_oracle_distill rejected its arguments")

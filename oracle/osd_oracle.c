@@ -35,9 +35,13 @@
  *   - any draft token outside [0, V) marks the whole sequence bad:
  *     accepted = -1, out_tokens = -1, mask = 0, diagnostics NaN.
  *   - the mismatch mask marks only the first rejected position (a < k).
- *   - distill uses temperature 1, returns the per-position loss and the
- *     unscaled per-position gradient; inactive rows get loss 0 and their
+ *   - distill applies one temperature tau to both rows (Section 4.1: the
+ *     logits are divided by tau before the softmax) and returns the
+ *     per-position loss and its gradient with respect to the raw draft
+ *     logits (hence a factor 1/tau); inactive rows get loss 0 and their
  *     gradient row is left untouched.
+ *   - the label fine-tuning loss (FT of Table 1) is the cross-entropy of q
+ *     to the target's argmax label, lowest index on ties.
  *   - TVD = 1/2 sum |p - q|, subgradient with sign(0) = 0.
  *   - 0 * log 0 = 0: terms with zero probability contribute nothing.
  *
@@ -51,7 +55,7 @@
 #include <stdlib.h>
 
 /* Loss kinds; values are part of the oracle's own interface. */
-enum { ORACLE_FKL = 0, ORACLE_RKL = 1, ORACLE_JSD = 2, ORACLE_TVD = 3 };
+enum { ORACLE_FKL = 0, ORACLE_RKL = 1, ORACLE_JSD = 2, ORACLE_TVD = 3, ORACLE_CE = 4 };
 
 /* log-softmax of x[0..V-1] / T into out (T > 0). Eq. 3 / Section 4.1
  * "softmax with temperature": lp_j = x_j/T - log sum_i exp(x_i/T).      */
@@ -196,32 +200,34 @@ int osd_oracle_verify(const double *draft, const double *target,
 }
 
 /*
- * Per-position distillation loss and gradient, Eq. 2-3 (Section 4.1) at
- * temperature 1, for every row n with mask[n] != 0 (mask may be NULL).
+ * Per-position distillation loss and gradient, Eq. 2-3 (Section 4.1), with
+ * softmax temperature tau, for every row n with mask[n] != 0 (mask may be NULL).
  *
- * draft, target [N, V]   logits z, t;  q = softmax(z), p = softmax(t)
+ * draft, target [N, V]   logits z, t;  q = softmax(z/tau), p = softmax(t/tau)
  * kind                   0 FKL = KL(p||q), 1 RKL = KL(q||p),
  *                        2 JSD[beta] = beta KL(p||m) + (1-beta) KL(q||m),
  *                          m = beta p + (1-beta) q,
- *                        3 TVD = 1/2 sum |p - q|
+ *                        3 TVD = 1/2 sum |p - q|,
+ *                        4 CE = -log q(y*), y* = argmax t (label fine-tuning)
  * loss [N]               per-position loss; 0 for inactive rows
- * dlogits [N, V]         d loss / d z; inactive rows are not written
+ * dlogits [N, V]         d loss / d z (raw logits); inactive rows are not written
  * Returns 0, or -1 on bad arguments / allocation failure.
  */
 int osd_oracle_distill(const double *draft, const double *target, long N, long V,
-                       const uint8_t *mask, int kind, double beta,
+                       const uint8_t *mask, int kind, double beta, double tau,
                        double *loss, double *dlogits)
 {
-    if (N < 0 || V < 1 || kind < 0 || kind > 3) return -1;
+    if (N < 0 || V < 1 || kind < 0 || kind > 4) return -1;
     if (kind == ORACLE_JSD && !(beta >= 0.0 && beta <= 1.0)) return -1;
+    if (!(tau > 0.0) || !isfinite(tau)) return -1;
     double *lq = (double *)malloc(sizeof(double) * (size_t)V);
     double *lp = (double *)malloc(sizeof(double) * (size_t)V);
     if (!lq || !lp) { free(lq); free(lp); return -1; }
 
     for (long n = 0; n < N; ++n) {
         if (mask && !mask[n]) { loss[n] = 0.0; continue; }
-        log_softmax(draft + n * V, V, 1.0, lq);
-        log_softmax(target + n * V, V, 1.0, lp);
+        log_softmax(draft + n * V, V, tau, lq);
+        log_softmax(target + n * V, V, tau, lp);
         double *g = dlogits + n * V;
         double l = 0.0;
         if (kind == ORACLE_FKL) {
@@ -255,6 +261,10 @@ int osd_oracle_distill(const double *draft, const double *target, long N, long V
                 g[j] = (q > 0.0 && beta < 1.0)
                            ? (1.0 - beta) * q * (log(q / m) - klq) : 0.0;
             }
+        } else if (kind == ORACLE_CE) {
+            long ystar = argmax_first(target + n * V, V);
+            l = -lq[ystar];
+            for (long j = 0; j < V; ++j) g[j] = exp(lq[j]) - (j == ystar ? 1.0 : 0.0);
         } else { /* ORACLE_TVD */
             double G = 0.0;
             for (long j = 0; j < V; ++j) {
@@ -269,6 +279,8 @@ int osd_oracle_distill(const double *draft, const double *target, long N, long V
                 g[j] = q * (s - G);
             }
         }
+        /* the softmax sees z / tau, so d/dz carries a factor 1 / tau */
+        for (long j = 0; j < V; ++j) g[j] /= tau;
         loss[n] = l;
     }
     free(lq); free(lp);

@@ -23,7 +23,7 @@ from ._build import LIB_PATH, build as build_library  # noqa: F401
 
 OSD_OK, OSD_ERR_INVALID_ARG, OSD_ERR_UNSUPPORTED, OSD_ERR_CUDA, OSD_ERR_TIMEOUT = range(5)
 OSD_F32, OSD_BF16 = 0, 1
-LOSS_KINDS = {"fkl": 0, "rkl": 1, "jsd": 2, "tvd": 3}
+LOSS_KINDS = {"fkl": 0, "rkl": 1, "jsd": 2, "tvd": 3, "ce": 4}
 VERIFY_MAX_K = 64
 VERIFY_MAX_V = 1 << 21
 
@@ -39,6 +39,7 @@ class OsdError(RuntimeError):
 
 
 _lib = None
+ABI_MAJOR = 2  # osd_distill gained its temperature argument in 2.0
 
 
 def load_library():
@@ -54,6 +55,9 @@ def load_library():
     lib.osd_status_string.argtypes = [i32]
     lib.osd_abi_version.restype = i32
     lib.osd_abi_version.argtypes = []
+    if lib.osd_abi_version() >> 16 != ABI_MAJOR:
+        raise RuntimeError(f"{LIB_PATH} has ABI {lib.osd_abi_version() >> 16}.x, this binding needs "
+                           f"{ABI_MAJOR}.x: rebuild it with paper_2310_07177_gb300.build_library()")
     lib.osd_verify_workspace_size.restype = i32
     lib.osd_verify_workspace_size.argtypes = [i32, i32, i32, ctypes.POINTER(sz)]
     lib.osd_verify.restype = i32
@@ -61,7 +65,7 @@ def load_library():
     lib.osd_verify_noalloc.restype = i32
     lib.osd_verify_noalloc.argtypes = [vp, vp, i32, i32, i32, i32, vp, vp, f32, vp, vp, vp, vp, vp, vp]
     lib.osd_distill.restype = i32
-    lib.osd_distill.argtypes = [vp, vp, i32, i32, i32, i32, i64, i64, i64, i64, vp, i32, f32, vp, vp, vp, vp]
+    lib.osd_distill.argtypes = [vp, vp, i32, i32, i32, i32, i64, i64, i64, i64, vp, i32, f32, f32, vp, vp, vp, vp]
     _lib = lib
     return lib
 
@@ -196,10 +200,13 @@ def _rows_view(t: torch.Tensor):
 
 
 def osd_distill(draft_logits: torch.Tensor, target_logits: torch.Tensor, mask: Optional[torch.Tensor] = None,
-                loss_kind: str = "fkl", beta: float = 0.5, *, loss: Optional[torch.Tensor] = None,
+                loss_kind: str = "fkl", beta: float = 0.5, *, temperature: float = 1.0,
+                loss: Optional[torch.Tensor] = None,
                 dlogits: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
                 stream: Optional[torch.cuda.Stream] = None):
-    """Per-position distillation loss and d loss / d draft_logits (Eq. 2-3).
+    """Per-position distillation loss and d loss / d draft_logits (Eq. 2-3) at
+    softmax temperature ``temperature`` (Section 4.1); ``loss_kind`` is one of
+    fkl, rkl, jsd, tvd, ce (label fine-tuning to the target argmax).
 
     Logits are [N,V] or [G,P,V] views whose rows are contiguous (e.g.
     ``target[:, :k, :]`` of a [B,k+1,V] tensor).  Returns ``(loss, dlogits)``:
@@ -225,7 +232,8 @@ def osd_distill(draft_logits: torch.Tensor, target_logits: torch.Tensor, mask: O
         raise ValueError("loss / dlogits must be contiguous float32 of the logits' shape")
     kind = LOSS_KINDS[loss_kind] if isinstance(loss_kind, str) else int(loss_kind)
     st = lib.osd_distill(_ptr(draft_logits), _ptr(target_logits), _dtype_code(draft_logits), G, P, V,
-                         dsg, dsp, tsg, tsp, _ptr(mask), kind, float(beta), _ptr(loss), _ptr(dlogits),
+                         dsg, dsp, tsg, tsp, _ptr(mask), kind, float(beta), float(temperature), _ptr(loss),
+                         _ptr(dlogits),
                          _ptr(status), _stream(dev, stream))
     if st != OSD_OK:
         raise OsdError(st, "osd_distill")

@@ -1,5 +1,7 @@
 // osd_distill.cu -- per-position distillation loss and gradient (Eq. 2-3 of
-// the paper, Section 4.1; the analytic draft update of Algorithm 1) on sm_103a.
+// the paper, Section 4.1, with its softmax temperature; the analytic draft
+// update of Algorithm 1; and the label fine-tuning cross-entropy of Table 1)
+// on sm_103a.
 //
 // One thread-block cluster per active row.  Each CTA owns a contiguous span of
 // the vocabulary: it stages its span of the draft and target rows into shared
@@ -16,6 +18,7 @@
 // see bit-identical statistics.  Logs and exponentials use the hardware
 // lg2/ex2 units in base 2; loss terms are converted to nats at the end.
 #include <climits>
+#include <cmath>
 #include <cstdint>
 #include <type_traits>
 
@@ -38,6 +41,10 @@ struct DistParams {
     long long dsg, dsp, tsg, tsp;
     const uint8_t* mask;
     float beta;
+    float c;        // log2(e) / temperature: exp(x / tau) = 2^(x c)
+    float inv_tau;  // the gradient w.r.t. raw logits carries 1 / tau
+    float lg_scale; // log2 of the gradient's constant factor (1/tau; JSD (1-beta) ln2 / tau),
+                    // folded into the exponents of pass 3
     float* loss;
     float* dlogits;
     int32_t* status;
@@ -49,10 +56,13 @@ struct DistParams {
 struct Stats1 {
     float mz, Ez, mt, Et, X;
     int err;
+    int idx;   // CE: first index of the target maximum
+    float zy;  // CE: draft logit at that index; RKL: the pivot target logit
 };
-// Pass-2 partial: JSD (KL(p||m), KL(q||m)) in bits, or TVD (sum |p-q|, sum q g).
+// Pass-2 partial: JSD (KL(p||m), KL(q||m) in bits), or TVD (sum |p - q|,
+// Q+ = sum of q over entries with q >= p, Q- = sum of q over q < p).
 struct Stats2 {
-    float a, b;
+    float a, b, c;
 };
 
 template <typename In>
@@ -132,8 +142,41 @@ __device__ __forceinline__ float3 block_sum3(float a, float b, float c, float3* 
     for (int w = 1; w < kDistThreads / 32; ++w) r = make_float3(r.x + scratch[w].x, r.y + scratch[w].y, r.z + scratch[w].z);
     return r;
 }
-__device__ __forceinline__ float rescale(float m, float mb) {
-    return (m == kNegInf) ? 0.f : ex2((m - mb) * kLog2e);
+// RKL: the draft maximum with the target logit at it (the larger one on ties),
+// merged in the same round as the target maximum.
+__device__ __forceinline__ bool pivot_wins(float m, float t, float m0, float t0) {
+    return m > m0 || (m == m0 && t > t0);
+}
+__device__ __forceinline__ float3 block_max_pivot(float mz, float tp, float mt, float3* scratch) {
+    for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, mz, o), t2 = __shfl_xor_sync(0xffffffffu, tp, o);
+        if (pivot_wins(m2, t2, mz, tp)) { mz = m2; tp = t2; }
+        mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
+    }
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    __syncthreads();
+    if (lane == 0) scratch[warp] = make_float3(mz, tp, mt);
+    __syncthreads();
+    float3 r = scratch[0];
+#pragma unroll
+    for (int w = 1; w < kDistThreads / 32; ++w) {
+        const float3 x = scratch[w];
+        if (pivot_wins(x.x, x.y, r.x, r.y)) { r.x = x.x; r.y = x.y; }
+        r.z = fmaxf(r.z, x.z);
+    }
+    return r;
+}
+__device__ __forceinline__ float rescale(float m, float mb, float c) {
+    return (m == kNegInf) ? 0.f : ex2((m - mb) * c);
+}
+// CE label: the target maximum with the lowest index, and the draft logit there.
+struct Label {
+    float m;
+    int i;
+    float z;
+};
+__device__ __forceinline__ Label merge_label(Label a, Label b) {
+    return (b.m > a.m || (b.m == a.m && b.i < a.i)) ? b : a;
 }
 
 // TVD keeps q' = q sign(q - p) (fp32) in the two 16-bit (bf16) or the first
@@ -181,10 +224,15 @@ __device__ __forceinline__ float load_q(const In* zs, const In* ts, int j) {
         return __uint_as_float((hi << 16) | lo);
     }
 }
+// With s = sign(q - p), G = sum_k q_k s_k / 2 and Q+ + Q- = sum q = 1, the TVD
+// gradient q (s/2 - G) / tau is q Q- / tau where q >= p and -q Q+ / tau where
+// q < p: both products of positive sums, so nothing cancels when one side
+// holds almost all the mass.
 template <typename In, bool kAligned>
-__device__ __forceinline__ void tvd_gradient(const In* zs, const In* ts, int n, float G, float* orow) {
+__device__ __forceinline__ void tvd_gradient(const In* zs, const In* ts, int n, float gpos, float gneg,
+                                             float* orow) {
     const int tid = threadIdx.x;
-    auto g_of = [G](float q) { return fmaf(-fabsf(q), G, 0.5f * q); };
+    auto g_of = [gpos, gneg](float q) { return q * (__float_as_int(q) < 0 ? gneg : gpos); };
     if constexpr (kAligned) {
         constexpr int kVec = Elem<In>::kVec;
         const int nv = n / kVec;
@@ -223,6 +271,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     constexpr bool kClamp = kKind == OSD_JSD;
     constexpr bool kClampZ = kClamp, kClampT = kClamp;
     constexpr bool kMoment = kKind == OSD_FKL || kKind == OSD_RKL;
+    constexpr bool kNeedEt = kKind != OSD_CE;  // CE needs only the draft normaliser and the label
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ __align__(8) uint64_t bar;
     __shared__ Stats1 s1_mine, s1_all;
@@ -230,10 +279,12 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     __shared__ float2 red_m[kDistThreads / 32];
     __shared__ float3 red_s[kDistThreads / 32];
     __shared__ int s_err;
-    __shared__ float s_cu, s_cv, s_loss, s_K;
+    __shared__ float s_cu, s_cv, s_loss, s_K, s_tp;
+    __shared__ Label red_l[kDistThreads / 32];
 
     const int tid = threadIdx.x;
     const int csize = p.csize;
+    const float c = p.c, inv_tau = p.inv_tau;
     const int rank = (csize > 1) ? static_cast<int>(cluster_rank()) : 0;
     const long long row = blockIdx.x / csize;
     if (p.mask && !p.mask[row]) {  // uniform over the cluster; no shared memory is exchanged
@@ -279,57 +330,105 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     __syncthreads();
     const int err_local = s_err;
 
-    // ---- pass 1: online max / sum of 2^((x - m) log2 e) per thread (+ the FKL/RKL moment)
+    // ---- pass 0: this thread's maxima, and the chunk where each first appears
     float mz = kNegInf, mt = kNegInf;
-    bool row_ninf = false;  // this thread saw a -inf logit (FKL, RKL)
-    float2 Ez2 = f2(0.f), Et2 = f2(0.f), X2 = f2(0.f);
+    int jz = -1, jt = -1;
     if (!err_local) {
-        sweep<In, kAligned, kClampZ, kClampT, true, kMoment>(zs, ts, n, [&](const float* z, const float* t,
-                                                                            auto tag, int, float cz, float ct,
-                                                                            bool ninf) {
+        sweep<In, kAligned, kClampZ, kClampT, true>(zs, ts, n, [&](const float*, const float*, auto, int j0,
+                                                                   float cz, float ct, bool) {
+            if (cz > mz) { mz = cz; jz = j0; }
+            if (ct > mt) { mt = ct; jt = j0; }
+        });
+    }
+    // the entry that holds a maximum: RKL's pivot target logit, CE's label
+    auto chunk_len = [n](int j0) {
+        constexpr int kVec = Elem<In>::kVec;
+        return (kAligned && j0 < (n / kVec) * kVec) ? kVec : 1;
+    };
+    float tp = 0.f;                      // RKL: target logit at this thread's draft maximum
+    Label lab{kNegInf, INT_MAX, 0.f};    // CE: this thread's first target maximum
+    if (kKind == OSD_RKL && jz >= 0) {
+        const int cnt = chunk_len(jz);
+#pragma unroll 1
+        for (int e = cnt - 1; e >= 0; --e)
+            if (Elem<In>::lds(zs + jz + e) == mz) tp = Elem<In>::lds(ts + jz + e);
+        if (tp == kNegInf) tp = 0.f;  // any finite pivot works; the loss is +inf then anyway
+    }
+    if (kKind == OSD_CE && jt >= 0) {
+        const int cnt = chunk_len(jt);
+        int ei = 0;
+#pragma unroll 1
+        for (int e = cnt - 1; e >= 0; --e)
+            if (Elem<In>::lds(ts + jt + e) == mt) ei = e;
+        lab = Label{mt, e0 + jt + ei, Elem<In>::lds(zs + jt + ei)};
+    }
+    // block maxima: every thread's sums of pass 1 then share one reference
+    float gzb, gtb, tpv = 0.f;
+    Label bl{kNegInf, INT_MAX, 0.f};
+    if constexpr (kKind == OSD_RKL) {
+        const float3 r = block_max_pivot(mz, tp, mt, red_s);
+        gzb = r.x;
+        tpv = r.y;
+        gtb = r.z;
+    } else {
+        const float2 bm = block_max2(mz, mt, red_m);
+        gzb = bm.x;
+        gtb = bm.y;
+        if constexpr (kKind == OSD_CE)
+            bl = block_reduce<kDistThreads>(lab, [](Label a, Label b) { return merge_label(a, b); }, red_l);
+    }
+
+    // ---- pass 1: sums of 2^((x - m) c) against the block maxima (+ the FKL/RKL moment)
+    // The RKL moment is taken about a pivot, the draft maximum m_z and the target
+    // logit t_pv found there: X = sum_j e_j ((z_j - m_z) - (t_j - t_pv)).  The
+    // pivot's own term is exactly 0, so when q is nearly one-hot the gradient
+    // q_j (log q_j - log p_j - loss) at the peak comes out as a sum of small
+    // terms instead of the difference of two large ones.
+    bool row_ninf = false;  // this thread saw a -inf logit (FKL, RKL)
+    bool rkl_inf = false;   // RKL: a finite draft logit meets a -inf target logit
+    float2 Ez2 = f2(0.f), Et2 = f2(0.f), X2 = f2(0.f);
+    const bool zok = kClampZ || gzb != kNegInf;
+    const bool tok = kNeedEt && (kClampT || gtb != kNegInf);
+    if (!err_local) {
+        const float2 gz2 = f2(gzb), gt2 = f2(gtb), tp2 = f2(tpv);
+        sweep<In, kAligned, kClampZ, kClampT, false, kMoment>(zs, ts, n, [&](const float* z, const float* t,
+                                                                             auto tag, int, float, float,
+                                                                             bool ninf) {
             constexpr int kCnt = decltype(tag)::value;
-            if (cz > mz) {
-                const float r = rescale(mz, cz);
-                Ez2 = mul2(Ez2, f2(r));
-                if (kKind == OSD_RKL) X2 = mul2(X2, f2(r));
-                mz = cz;
-            }
-            if (ct > mt) {
-                const float r = rescale(mt, ct);
-                Et2 = mul2(Et2, f2(r));
-                if (kKind == OSD_FKL) X2 = mul2(X2, f2(r));
-                mt = ct;
-            }
             row_ninf |= ninf;
             if (kCnt == 1 || ninf) {  // element-wise, with the guards a -inf needs
 #pragma unroll
                 for (int e = 0; e < kCnt; ++e) {
-                    if (kClampZ || mz != kNegInf) {
-                        const float ez = ex2((z[e] - mz) * kLog2e);
+                    if (zok) {
+                        const float ez = ex2((z[e] - gzb) * c);
                         Ez2.x += ez;
-                        if (kKind == OSD_RKL && ez > 0.f) X2.x = fmaf(ez, z[e] - t[e], X2.x);
+                        if (kKind == OSD_RKL && z[e] != kNegInf) {
+                            if (t[e] == kNegInf) rkl_inf = true;  // q > 0 = p: the loss is +inf
+                            else X2.x = fmaf(ez, (z[e] - gzb) - (t[e] - tpv), X2.x);
+                        }
                     }
-                    if (kClampT || mt != kNegInf) {
-                        const float et = ex2((t[e] - mt) * kLog2e);
+                    if (tok) {
+                        const float et = ex2((t[e] - gtb) * c);
                         Et2.x += et;
                         if (kKind == OSD_FKL && et > 0.f) X2.x = fmaf(et, t[e] - z[e], X2.x);
                     }
                 }
             } else {
-                if (kClampZ || mz != kNegInf) {
+                if (zok) {
 #pragma unroll
                     for (int e = 0; e < kCnt; e += 2) {
-                        const float2 a = mul2(sub2(make_float2(z[e], z[e + 1]), f2(mz)), f2(kLog2e));
+                        const float2 zd = sub2(make_float2(z[e], z[e + 1]), gz2);
+                        const float2 a = mul2(zd, f2(c));
                         const float2 ez = make_float2(ex2(a.x), ex2(a.y));
                         Ez2 = add2(Ez2, ez);
                         if (kKind == OSD_RKL)
-                            X2 = fma2(ez, sub2(make_float2(z[e], z[e + 1]), make_float2(t[e], t[e + 1])), X2);
+                            X2 = fma2(ez, sub2(zd, sub2(make_float2(t[e], t[e + 1]), tp2)), X2);
                     }
                 }
-                if (kClampT || mt != kNegInf) {
+                if (tok) {
 #pragma unroll
                     for (int e = 0; e < kCnt; e += 2) {
-                        const float2 a = mul2(sub2(make_float2(t[e], t[e + 1]), f2(mt)), f2(kLog2e));
+                        const float2 a = mul2(sub2(make_float2(t[e], t[e + 1]), gt2), f2(c));
                         const float2 et = make_float2(ex2(a.x), ex2(a.y));
                         Et2 = add2(Et2, et);
                         if (kKind == OSD_FKL)
@@ -339,20 +438,20 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
             }
         });
     }
-    // block merge: maxima first, then every thread rescales once and the sums add up
     {
-        const float2 bm = block_max2(mz, mt, red_m);
-        const float sz = rescale(mz, bm.x), st = rescale(mt, bm.y);
-        const float xs = (kKind == OSD_RKL) ? sz : st;
-        const float3 bs = block_sum3((Ez2.x + Ez2.y) * sz, (Et2.x + Et2.y) * st, (X2.x + X2.y) * xs, red_s);
+        const float3 bs = block_sum3(Ez2.x + Ez2.y, Et2.x + Et2.y, X2.x + X2.y, red_s);
         const int any_ninf = __syncthreads_or(row_ninf ? 1 : 0);
-        if (tid == 0) s1_mine = Stats1{bm.x, bs.x, bm.y, bs.y, bs.z, err_local | (any_ninf << 1)};
+        const int any_inf = (kKind == OSD_RKL) ? __syncthreads_or(rkl_inf ? 1 : 0) : 0;
+        if (tid == 0)
+            s1_mine = Stats1{gzb, bs.x, (kKind == OSD_CE) ? bl.m : gtb, bs.y, bs.z,
+                             err_local | (any_ninf << 1) | (any_inf << 2), bl.i,
+                             (kKind == OSD_RKL) ? tpv : bl.z};
     }
     // cluster merge: warp 0 gathers every CTA's partial (lane r <- CTA r) and reduces
     // it in a fixed order, so all CTAs of the row hold bit-identical statistics
     if (csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
     if (tid < 32) {
-        Stats1 o{kNegInf, 0.f, kNegInf, 0.f, 0.f, 0};
+        Stats1 o{kNegInf, 0.f, kNegInf, 0.f, 0.f, 0, INT_MAX, 0.f};
         if (tid < csize) {
             if (tid == rank) {
                 o = s1_mine;
@@ -364,6 +463,16 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                 o.Et = ld_dsmem_f32(base + offsetof(Stats1, Et));
                 o.X = ld_dsmem_f32(base + offsetof(Stats1, X));
                 o.err = ld_dsmem_s32(base + offsetof(Stats1, err));
+                if (kKind == OSD_CE) o.idx = ld_dsmem_s32(base + offsetof(Stats1, idx));
+                if (kKind == OSD_CE || kKind == OSD_RKL) o.zy = ld_dsmem_f32(base + offsetof(Stats1, zy));
+            }
+        }
+        Label L{o.mt, o.idx, o.zy};  // CE label: the CTA labels merge like an argmax
+        if constexpr (kKind == OSD_CE) {
+            for (int off = 16; off > 0; off >>= 1) {
+                const Label w{__shfl_xor_sync(0xffffffffu, L.m, off), __shfl_xor_sync(0xffffffffu, L.i, off),
+                              __shfl_xor_sync(0xffffffffu, L.z, off)};
+                L = merge_label(L, w);
             }
         }
         float gz = o.mz, gt = o.mt;
@@ -373,25 +482,40 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
             gt = fmaxf(gt, __shfl_xor_sync(0xffffffffu, gt, off));
             err |= __shfl_xor_sync(0xffffffffu, err, off);
         }
-        const float sz = rescale(o.mz, gz), st = rescale(o.mt, gt);
-        float Ez = o.Ez * sz, Et = o.Et * st, X = o.X * ((kKind == OSD_RKL) ? sz : st);
+        const float sz = rescale(o.mz, gz, c), st = rescale(o.mt, gt, c);
+        float tg = 0.f;  // RKL: the row's pivot target logit
+        if constexpr (kKind == OSD_RKL) {
+            tg = (o.mz == gz && o.mz != kNegInf) ? o.zy : kNegInf;
+            for (int off = 16; off > 0; off >>= 1) tg = fmaxf(tg, __shfl_xor_sync(0xffffffffu, tg, off));
+            if (tg == kNegInf) tg = 0.f;
+        }
+        float Ez = o.Ez * sz, Et = o.Et * st, X;
+        if constexpr (kKind == OSD_RKL)
+            X = (o.mz == kNegInf) ? 0.f : fmaf(o.Ez, (o.mz - gz) - (o.zy - tg), o.X) * sz;
+        else
+            X = o.X * st;
         for (int off = 16; off > 0; off >>= 1) {
             Ez += __shfl_xor_sync(0xffffffffu, Ez, off);
             Et += __shfl_xor_sync(0xffffffffu, Et, off);
             X += __shfl_xor_sync(0xffffffffu, X, off);
         }
         if (tid == 0) {
-            s1_all = Stats1{gz, Ez, gt, Et, X, err};
-            // row constants, computed once: log2 p = (t - m_t) log2(e) - log2(E_t); the
-            // difference is exact, so the rounding never scales with the size of the logits
+            s1_all = Stats1{gz, Ez, gt, Et, X, err, L.i, L.z};
+            // row constants, computed once: log2 p = (t - m_t) c - log2(E_t) with
+            // c = log2(e)/tau; the difference is exact, so the rounding never scales
+            // with the size of the logits
             s_cu = -log2f(Et);
             s_cv = -log2f(Ez);
             const float lr = logf(Ez / Et);
             float l = 0.f;
-            if (kKind == OSD_FKL) l = X / Et - (gt - gz) + lr;
-            if (kKind == OSD_RKL) l = X / Ez - (gz - gt) - lr;
+            if (kKind == OSD_FKL) l = (X / Et - (gt - gz)) * inv_tau + lr;
+            // RKL about the pivot: loss = log q - log p at the pivot + sum_j q_j D_j, with
+            // D_j = ((z_j - m_z) - (t_j - t_pv)) / tau; s_K keeps the sum for pass 3
+            if (kKind == OSD_RKL) l = (err & 4) ? __builtin_huge_valf() : (X / Ez + (gt - tg)) * inv_tau - lr;
+            if (kKind == OSD_CE) l = (gz - L.z) * inv_tau + logf(Ez);  // -log q(y*)
             s_loss = l;
-            s_K = (gz - gt) + lr + l;  // RKL: log q - log p - loss = (z - t) - K
+            s_K = X / Ez * inv_tau;
+            s_tp = tg;
         }
     }
     __syncthreads();
@@ -400,16 +524,16 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     const bool has_ninf = (st.err & 2) != 0;  // some logit of the row is -inf
     const float cu = s_cu, cv = s_cv;
     const float2 mt2 = f2(st.mt), mz2 = f2(st.mz);
-    auto log2p = [&](float2 x) { return fma2(sub2(x, mt2), f2(kLog2e), f2(cu)); };
-    auto log2q = [&](float2 x) { return fma2(sub2(x, mz2), f2(kLog2e), f2(cv)); };
+    auto log2p = [&](float2 x) { return fma2(sub2(x, mt2), f2(c), f2(cu)); };
+    auto log2q = [&](float2 x) { return fma2(sub2(x, mz2), f2(c), f2(cv)); };
     float loss = s_loss;
 
     const float beta = p.beta;
     const bool jsd_trivial = (kKind == OSD_JSD) && (beta == 0.f || beta == 1.f);  // m = q or m = p: loss 0
-    Stats2 s2 = {0.f, 0.f};
+    Stats2 s2 = {0.f, 0.f, 0.f};
     if constexpr (kKind == OSD_JSD || kKind == OSD_TVD) {
         // ---- pass 2: divergence terms with the global normalisers
-        float2 A2 = f2(0.f), B2 = f2(0.f);
+        float2 A2 = f2(0.f), B2 = f2(0.f), C2 = f2(0.f);
         if (!row_err && !jsd_trivial) {
             sweep<In, kAligned, kClampZ, kClampT, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
                                                                         int j0, float, float, bool) {
@@ -421,14 +545,16 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                     const float2 u = log2p(make_float2(t[e], two ? t[e + 1] : t[e]));  // log2 p
                     const float2 v = log2q(make_float2(z[e], two ? z[e + 1] : z[e]));  // log2 q
                     const float2 d = sub2(v, u);
-                    float2 a, b;
+                    float2 a, b, c2 = f2(0.f);
                     if (kKind == OSD_TVD) {
                         const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
                         const float2 df = sub2(pj, qj);
                         a = make_float2(fabsf(df.x), fabsf(df.y));
-                        b = make_float2(copysignf(qj.x, d.x), copysignf(qj.y, d.y));  // q sign(q - p)
-                        qs[e] = b.x;
-                        if (e + 1 < kCnt) qs[e + 1] = b.y;
+                        const float2 qq = make_float2(copysignf(qj.x, d.x), copysignf(qj.y, d.y));  // q sign(q - p)
+                        qs[e] = qq.x;
+                        if (e + 1 < kCnt) qs[e + 1] = qq.y;
+                        b = add2(qj, qq);   // 2q where q >= p, else 0 (exact): into 2 Q+
+                        c2 = sub2(qj, qq);  // 2q where q < p, else 0: into 2 Q-
                     } else {
                         float r[2][2];
                         const float uu[2] = {u.x, u.y}, vv[2] = {v.x, v.y}, dd[2] = {d.x, d.y};
@@ -448,40 +574,45 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                         a = make_float2(r[0][0], r[1][0]);
                         b = make_float2(r[0][1], r[1][1]);
                     }
-                    if (!two) { a.y = 0.f; b.y = 0.f; }
+                    if (!two) { a.y = 0.f; b.y = 0.f; c2.y = 0.f; }
                     A2 = add2(A2, a);
                     B2 = add2(B2, b);
+                    C2 = add2(C2, c2);
                 }
                 // the logits of these entries are not needed again: their slots take q'
                 if constexpr (kKind == OSD_TVD) store_q<In, kCnt>(zs, ts, j0, qs);
             });
         }
-        const float3 bs = block_sum3(A2.x + A2.y, B2.x + B2.y, 0.f, red_s);
-        if (tid == 0) s2_mine = Stats2{bs.x, bs.y};
+        const float3 bs = block_sum3(A2.x + A2.y, B2.x + B2.y, C2.x + C2.y, red_s);
+        if (tid == 0) s2_mine = Stats2{bs.x, bs.y, bs.z};
         if (csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
         if (tid < 32) {
-            float a = 0.f, b = 0.f;
+            float a = 0.f, b = 0.f, cc = 0.f;
             if (tid < csize) {
                 if (tid == rank) {
                     a = s2_mine.a;
                     b = s2_mine.b;
+                    cc = s2_mine.c;
                 } else {
                     const uint32_t base = map_rank(&s2_mine, tid);
                     a = ld_dsmem_f32(base + offsetof(Stats2, a));
                     b = ld_dsmem_f32(base + offsetof(Stats2, b));
+                    if (kKind == OSD_TVD) cc = ld_dsmem_f32(base + offsetof(Stats2, c));
                 }
             }
             for (int off = 16; off > 0; off >>= 1) {
                 a += __shfl_xor_sync(0xffffffffu, a, off);
                 b += __shfl_xor_sync(0xffffffffu, b, off);
+                if (kKind == OSD_TVD) cc += __shfl_xor_sync(0xffffffffu, cc, off);
             }
-            if (tid == 0) s2_all = Stats2{a, b};
+            if (tid == 0) s2_all = Stats2{a, b, cc};
         }
         __syncthreads();
         s2 = s2_all;
         if (kKind == OSD_TVD) {
             loss = 0.5f * s2.a;
-            s2.b *= 0.5f;  // sum_j q_j g_j with g = sign(q - p) / 2
+            s2.b *= 0.5f;
+            s2.c *= 0.5f;
         } else {
             loss = jsd_trivial ? 0.f : kLn2 * (beta * s2.a + (1.f - beta) * s2.b);
         }
@@ -495,12 +626,14 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
 
     // ---- pass 3: d loss / d draft logits of the span
     if (kKind == OSD_TVD && !row_err) {
-        // g = q (sign(q - p)/2 - G) = q'/2 - |q'| G from the stored q'
-        tvd_gradient<In, kAligned>(zs, ts, n, s2.b, p.dlogits + row * V + e0);
+        // from the stored q' = q sign(q - p): q' Q- / tau, or q' Q+ / tau where q' < 0
+        tvd_gradient<In, kAligned>(zs, ts, n, s2.c * inv_tau, s2.b * inv_tau, p.dlogits + row * V + e0);
     } else if (kKind != OSD_TVD && !row_err) {
         float* orow = p.dlogits + row * V + e0;
-        const float K = s_K;
-        const float jsd_scale = (1.f - beta) * kLn2;
+        const float K = s_K, tpg = s_tp;
+        // q and p of this pass come out multiplied by the gradient's constant factor
+        const float2 cvs = f2(cv + p.lg_scale), cus = f2(cu + p.lg_scale);
+        const int label = st.idx;
         sweep<In, kAligned, kClampZ, kClampT, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
                                                                     int j0, float, float, bool) {
             constexpr int kCnt = decltype(tag)::value;
@@ -510,27 +643,28 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                 const bool two = (e + 1 < kCnt);
                 const float2 zz = make_float2(z[e], two ? z[e + 1] : z[e]);
                 const float2 tt = make_float2(t[e], two ? t[e + 1] : t[e]);
-                const float2 v = log2q(zz);
+                const float2 zd = sub2(zz, mz2);
+                const float2 v = fma2(zd, f2(c), cvs);  // log2 q + lg_scale
                 const float2 qj = make_float2(ex2(v.x), ex2(v.y));
                 float2 gg;
-                if (kKind == OSD_FKL) {
-                    const float2 u = log2p(tt);
+                if (kKind == OSD_FKL) {  // (q - p) / tau
+                    const float2 u = fma2(sub2(tt, mt2), f2(c), cus);
                     gg = sub2(qj, make_float2(ex2(u.x), ex2(u.y)));
-                } else if (kKind == OSD_RKL) {
-                    gg = mul2(qj, sub2(sub2(zz, tt), f2(K)));
+                } else if (kKind == OSD_CE) {  // (q - onehot(y*)) / tau
+                    const int j = e0 + j0 + e;
+                    gg = sub2(qj, make_float2(j == label ? inv_tau : 0.f, j + 1 == label ? inv_tau : 0.f));
+                } else if (kKind == OSD_RKL) {  // q_j (D_j - sum_k q_k D_k) / tau
+                    const float2 dd = sub2(zd, sub2(tt, f2(tpg)));
+                    gg = mul2(qj, fma2(dd, f2(inv_tau), f2(-K)));
                     if (has_ninf) {  // q = 0 against an infinite log-ratio contributes 0
                         if (!(qj.x > 0.f)) gg.x = 0.f;
                         if (!(qj.y > 0.f)) gg.y = 0.f;
                     }
-                } else if (kKind == OSD_TVD) {
-                    const float2 d = sub2(v, log2p(tt));
-                    const float2 sg = make_float2(copysignf(0.5f, d.x), copysignf(0.5f, d.y));
-                    gg = mul2(qj, sub2(sg, f2(s2.b)));
                 } else {
                     if (jsd_trivial) {
                         gg = f2(0.f);
                     } else {
-                        const float2 d = sub2(v, log2p(tt));
+                        const float2 d = sub2(v, fma2(sub2(tt, mt2), f2(c), cus));  // log2 q - log2 p
                         const float dd[2] = {d.x, d.y};
                         float l2mq[2];
 #pragma unroll
@@ -542,7 +676,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                             const float L = lg2(fmaf(1.f - wbig, rho, wbig));
                             l2mq[h] = pbig ? L + ad : L;
                         }
-                        gg = mul2(mul2(qj, f2(jsd_scale)), make_float2(-l2mq[0] - s2.b, -l2mq[1] - s2.b));
+                        gg = mul2(qj, make_float2(-l2mq[0] - s2.b, -l2mq[1] - s2.b));
                     }
                 }
                 gr[e] = gg.x;
@@ -580,6 +714,7 @@ static cudaError_t launch_distill_dtype(osd_loss kind, const DistParams& dp, lon
         case OSD_FKL: return launch_distill_kind<In, OSD_FKL, kAligned>(dp, rows, smem, s);
         case OSD_RKL: return launch_distill_kind<In, OSD_RKL, kAligned>(dp, rows, smem, s);
         case OSD_JSD: return launch_distill_kind<In, OSD_JSD, kAligned>(dp, rows, smem, s);
+        case OSD_CE: return launch_distill_kind<In, OSD_CE, kAligned>(dp, rows, smem, s);
         default: return launch_distill_kind<In, OSD_TVD, kAligned>(dp, rows, smem, s);
     }
 }
@@ -605,10 +740,12 @@ static bool distill_shape(int V, size_t es, int* csize, int* span) {
 extern "C" osd_status osd_distill(const void* draft_logits, const void* target_logits, osd_dtype dtype,
                                   int G, int P, int V, int64_t d_stride_g, int64_t d_stride_p,
                                   int64_t t_stride_g, int64_t t_stride_p, const uint8_t* mask, osd_loss kind,
-                                  float beta, float* loss, float* dlogits, int32_t* status, void* stream) {
+                                  float beta, float temperature, float* loss, float* dlogits, int32_t* status,
+                                  void* stream) {
     using namespace osd;
     if (dtype != OSD_F32 && dtype != OSD_BF16) return OSD_ERR_INVALID_ARG;
-    if (kind < OSD_FKL || kind > OSD_TVD) return OSD_ERR_INVALID_ARG;
+    if (kind < OSD_FKL || kind > OSD_CE) return OSD_ERR_INVALID_ARG;
+    if (!(temperature > 0.f) || !std::isfinite(temperature)) return OSD_ERR_INVALID_ARG;
     if (G < 0 || P < 0 || V < 1) return OSD_ERR_INVALID_ARG;
     if (d_stride_g < 0 || d_stride_p < 0 || t_stride_g < 0 || t_stride_p < 0) return OSD_ERR_INVALID_ARG;
     if (kind == OSD_JSD && !(beta >= 0.f && beta <= 1.f)) return OSD_ERR_INVALID_ARG;
@@ -642,6 +779,13 @@ extern "C" osd_status osd_distill(const void* draft_logits, const void* target_l
     dp.G = G; dp.P = P; dp.V = V;
     dp.dsg = d_stride_g; dp.dsp = d_stride_p; dp.tsg = t_stride_g; dp.tsp = t_stride_p;
     dp.mask = mask; dp.beta = beta; dp.loss = loss; dp.dlogits = dlogits; dp.status = status;
+    dp.c = static_cast<float>(1.4426950408889634074 / static_cast<double>(temperature));
+    dp.inv_tau = static_cast<float>(1.0 / static_cast<double>(temperature));
+    {
+        double scale = 1.0 / static_cast<double>(temperature);
+        if (kind == OSD_JSD) scale *= (1.0 - static_cast<double>(beta)) * 0.69314718055994530942;
+        dp.lg_scale = scale > 0.0 ? static_cast<float>(std::log2(scale)) : 0.f;  // beta = 1: gradient is 0
+    }
     dp.csize = csize; dp.span = span;
     const size_t smem = 2 * size_t(span) * es;
     cudaError_t e;

@@ -33,7 +33,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 def test_status_strings_and_version(lib):
     import paper_2310_07177_gb300 as osd
-    assert osd.osd_abi_version() >> 16 == 1
+    assert osd.osd_abi_version() >> 16 == osd.ABI_MAJOR == 2
     for code in range(5):
         assert osd.osd_status_string(code).startswith("OSD_")
     assert osd.osd_status_string(99) == "OSD_ERR_UNKNOWN"
@@ -65,16 +65,19 @@ def test_argument_errors_return_before_any_launch(lib):
     # empty batch is a no-op
     assert lib.osd_verify(None, None, 0, 0, 2, 16, None, None, 1.0, None, None, None, None, None,
                           None, 0, None) == osd.OSD_OK
-    # distill: bad beta, bad kind, vocabulary beyond the limit, negative stride
-    assert lib.osd_distill(fake, fake, 1, 2, 1, 16, 16, 0, 16, 0, None, 2, 1.5, fake, fake, None,
+    # distill: bad beta, bad kind, bad temperature, vocabulary beyond the limit, negative stride
+    assert lib.osd_distill(fake, fake, 1, 2, 1, 16, 16, 0, 16, 0, None, 2, 1.5, 1.0, fake, fake, None,
                            None) == osd.OSD_ERR_INVALID_ARG
-    assert lib.osd_distill(fake, fake, 1, 2, 1, 16, 16, 0, 16, 0, None, 9, 0.5, fake, fake, None,
+    assert lib.osd_distill(fake, fake, 1, 2, 1, 16, 16, 0, 16, 0, None, 9, 0.5, 1.0, fake, fake, None,
                            None) == osd.OSD_ERR_INVALID_ARG
-    assert lib.osd_distill(fake, fake, 1, 1, 1, 500000, 0, 0, 0, 0, None, 0, 0.5, fake, fake, None,
+    for tau in (0.0, -1.0, float("nan"), float("inf")):
+        assert lib.osd_distill(fake, fake, 1, 2, 1, 16, 16, 0, 16, 0, None, 0, 0.5, tau, fake, fake, None,
+                               None) == osd.OSD_ERR_INVALID_ARG
+    assert lib.osd_distill(fake, fake, 1, 1, 1, 500000, 0, 0, 0, 0, None, 0, 0.5, 1.0, fake, fake, None,
                            None) == osd.OSD_ERR_UNSUPPORTED
-    assert lib.osd_distill(fake, fake, 1, 2, 1, 16, -16, 0, 16, 0, None, 0, 0.5, fake, fake, None,
+    assert lib.osd_distill(fake, fake, 1, 2, 1, 16, -16, 0, 16, 0, None, 0, 0.5, 1.0, fake, fake, None,
                            None) == osd.OSD_ERR_INVALID_ARG
-    assert lib.osd_distill(None, None, 1, 0, 4, 16, 16, 0, 16, 0, None, 0, 0.5, None, None, None,
+    assert lib.osd_distill(None, None, 1, 0, 4, 16, 16, 0, 16, 0, None, 0, 0.5, 1.0, None, None, None,
                            None) == osd.OSD_OK
 
 

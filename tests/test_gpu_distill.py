@@ -10,7 +10,7 @@ from paper_2310_07177_gb300 import workloads as W
 from tests.parity import check_distill
 
 pytestmark = pytest.mark.gpu
-KINDS = ["fkl", "rkl", "jsd", "tvd"]
+KINDS = ["fkl", "rkl", "jsd", "tvd", "ce"]
 
 
 @pytest.fixture(scope="module")
@@ -23,30 +23,30 @@ def osd():
     return pkg
 
 
-def _tvd_ambiguous(z, t):
+def _tvd_ambiguous(z, t, tau=1.0):
     """Entries where sign(q - p) is not decided by fp32: |ln q - ln p| < 1e-5."""
-    lq = oracle.log_softmax(z.reshape(-1, z.shape[-1]))
-    lp = oracle.log_softmax(t.reshape(-1, t.shape[-1]))
+    lq = oracle.log_softmax(z.reshape(-1, z.shape[-1]), tau)
+    lp = oracle.log_softmax(t.reshape(-1, t.shape[-1]), tau)
     return np.abs(lq - lp) < 1e-5
 
 
-def _run(osd, z, t, mask, kind, beta, dev="cuda"):
+def _run(osd, z, t, mask, kind, beta, dev="cuda", tau=1.0):
     zd, td = z.to(dev), t.to(dev)
     md = None if mask is None else mask.to(dev)
     V = z.shape[-1]
     lead = tuple(z.shape[:-1])
     dl = torch.full(lead + (V,), float("nan"), dtype=torch.float32, device=dev)
-    loss, g = osd.osd_distill(zd, td, md, kind, beta, dlogits=dl)
+    loss, g = osd.osd_distill(zd, td, md, kind, beta, dlogits=dl, temperature=tau)
     torch.cuda.synchronize()
     return loss.cpu().numpy().reshape(-1), g.cpu().numpy().reshape(-1, V)
 
 
-def _oracle(z, t, mask, kind, beta):
+def _oracle(z, t, mask, kind, beta, tau=1.0):
     V = z.shape[-1]
     zc = z.reshape(-1, V)
     tc = t.reshape(-1, V)
     m = None if mask is None else mask.reshape(-1)
-    return oracle.distill(zc, tc, m, kind, beta)
+    return oracle.distill(zc, tc, m, kind, beta, temperature=float(np.float32(tau)))
 
 
 SHAPES = [  # (N, V, dtype)
@@ -72,11 +72,12 @@ def test_distill_matches_oracle(osd, kind, N, V, dtype):
     if N >= 3:
         mask[1] = 0
     beta = 0.3 if kind == "jsd" else 0.5
-    lg, gg = _run(osd, z, t, mask, kind, beta)
-    lr, gr = _oracle(z, t, mask, kind, beta)
-    skip = _tvd_ambiguous(z, t) if kind == "tvd" else None
-    rep = check_distill(lg, gg, lr, gr, mask.numpy() == 1, skip)
-    print(f"{kind} N={N} V={V} {dtype}: {rep}")
+    for tau in (1.0, 0.7) if V in (100, 33001, 128256) else (1.0,):
+        lg, gg = _run(osd, z, t, mask, kind, beta, tau=tau)
+        lr, gr = _oracle(z, t, mask, kind, beta, tau=tau)
+        skip = _tvd_ambiguous(z, t, tau) if kind == "tvd" else None
+        rep = check_distill(lg, gg, lr, gr, mask.numpy() == 1, skip)
+        print(f"{kind} N={N} V={V} {dtype} tau={tau}: {rep}")
 
 
 @pytest.mark.parametrize("kind", KINDS)
@@ -99,6 +100,19 @@ def test_strided_target_view(osd, kind):
                   mask.numpy().reshape(-1) == 1, skip)
 
 
+def test_ce_label_ties_take_the_lowest_index(osd):
+    """FT (Table 1): the label is the first target maximum, also across CTAs of a cluster."""
+    z = torch.randn(3, 40000, generator=torch.Generator().manual_seed(4)).to(torch.bfloat16)
+    t = torch.randn(3, 40000, generator=torch.Generator().manual_seed(5)).to(torch.bfloat16)
+    t[0, 30000] = t[0, 9000] = t[0, 35000] = 20.0   # tie spanning several CTAs of the row
+    t[1, 5] = t[1, 6] = 20.0                        # tie inside one chunk
+    t[2, 39999] = 20.0                              # label in the last entry
+    lg, gg = _run(osd, z, t, None, "ce", 0.5)
+    lr, gr = _oracle(z, t, None, "ce", 0.5)
+    check_distill(lg, gg, lr, gr, np.ones(3, bool))
+    assert np.argmin(gg[0]) == 9000 and np.argmin(gg[1]) == 5 and np.argmin(gg[2]) == 39999
+
+
 def test_unaligned_rows(osd):
     """Rows starting off a 16-byte boundary take the element-wise path."""
     base = torch.randn(4 * 1001 + 3, generator=torch.Generator().manual_seed(1)) * 2
@@ -118,7 +132,7 @@ def test_unaligned_rows(osd):
 def test_identical_rows_and_jsd_endpoints(osd):
     dev = torch.device("cuda")
     z = (torch.randn(4, 3000) * 3).to(torch.bfloat16).to(dev)
-    for kind in KINDS:
+    for kind in ("fkl", "rkl", "jsd", "tvd"):
         loss, g = osd.osd_distill(z, z, None, kind, 0.5)
         assert loss.abs().max().item() < 1e-6
         assert g.abs().max().item() < 1e-7
@@ -138,9 +152,9 @@ def test_extreme_and_neg_inf_logits(osd):
     t[2, :100] = float("-inf")
     t[3, 7] = 60.0
     for kind in KINDS:
-        lg, gg = _run(osd, z, t, None, kind, 0.4)
-        lr, gr = _oracle(z, t, None, kind, 0.4)
-        skip = _tvd_ambiguous(z, t) if kind == "tvd" else None
+        lg, gg = _run(osd, z, t, None, kind, 0.4, tau=1.3)
+        lr, gr = _oracle(z, t, None, kind, 0.4, tau=1.3)
+        skip = _tvd_ambiguous(z, t, 1.3) if kind == "tvd" else None
         check_distill(lg, gg, lr, gr, np.ones(5, bool), skip)
 
 
@@ -152,6 +166,9 @@ def test_invalid_arguments_are_rejected(osd):
     assert ei.value.status == osd.OSD_ERR_INVALID_ARG
     with pytest.raises(osd.OsdError) as ei:
         osd.osd_distill(z, z, None, 7, 0.5)
+    assert ei.value.status == osd.OSD_ERR_INVALID_ARG
+    with pytest.raises(osd.OsdError) as ei:
+        osd.osd_distill(z, z, None, "fkl", 0.5, temperature=0.0)
     assert ei.value.status == osd.OSD_ERR_INVALID_ARG
     big = torch.zeros(1, 500000, dtype=torch.bfloat16, device=dev)
     with pytest.raises(osd.OsdError) as ei:

@@ -8,13 +8,13 @@ import os
 import numpy as np
 import pytest
 from scipy.spatial.distance import cityblock, jensenshannon
-from scipy.special import rel_entr, softmax
+from scipy.special import log_softmax, rel_entr, softmax
 from scipy.stats import entropy
 
 import oracle
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "distill_v2_worked.txt")
-KINDS = ["fkl", "rkl", "jsd", "tvd"]
+KINDS = ["fkl", "rkl", "jsd", "tvd", "ce"]
 
 
 def _golden():
@@ -40,7 +40,8 @@ def test_worked_example_v2():
                                      ("jsd", 0.5, "loss_jsd_0.5", "grad_jsd_0.5"),
                                      ("jsd", 0.1, "loss_jsd_0.1", None),
                                      ("jsd", 0.9, "loss_jsd_0.9", None),
-                                     ("tvd", 0.5, "loss_tvd", "grad_tvd")]:
+                                     ("tvd", 0.5, "loss_tvd", "grad_tvd"),
+                                     ("ce", 0.5, "loss_ce", "grad_ce")]:
         loss, grad = oracle.distill(z, t, loss_kind=kind, beta=beta)
         assert abs(loss[0] - g[lname]) < 1e-14, (kind, beta, loss[0], g[lname])
         if gname:
@@ -90,32 +91,62 @@ def test_tvd_matches_scipy_cityblock():
         assert loss[n] == pytest.approx(0.5 * cityblock(softmax(t[n]), softmax(z[n])), rel=1e-12)
 
 
-def _fd_grad(z, t, kind, beta, h=1e-6):
+def _fd_grad(z, t, kind, beta, tau=1.0, h=1e-6):
     g = np.empty_like(z)
     for j in range(z.shape[-1]):
         zp, zm = z.copy(), z.copy()
         zp[0, j] += h
         zm[0, j] -= h
-        lp, _ = oracle.distill(zp, t, loss_kind=kind, beta=beta)
-        lm, _ = oracle.distill(zm, t, loss_kind=kind, beta=beta)
+        lp, _ = oracle.distill(zp, t, loss_kind=kind, beta=beta, temperature=tau)
+        lm, _ = oracle.distill(zm, t, loss_kind=kind, beta=beta, temperature=tau)
         g[0, j] = (lp[0] - lm[0]) / (2 * h)
     return g
 
 
 @pytest.mark.parametrize("kind", KINDS)
 @pytest.mark.parametrize("V", [2, 7, 64])
-def test_gradient_matches_central_differences(kind, V):
-    """The analytic gradient w.r.t. draft logits (Algorithm 1, update step)
-    against central finite differences of the oracle's loss."""
-    rng = np.random.default_rng(100 + V + 7 * KINDS.index(kind))
+@pytest.mark.parametrize("tau", [1.0, 0.5, 2.0])
+def test_gradient_matches_central_differences(kind, V, tau):
+    """The analytic gradient w.r.t. the raw draft logits (Algorithm 1, update
+    step; temperature of Section 4.1) against central finite differences of
+    the oracle's loss."""
+    rng = np.random.default_rng(100 + V + 7 * KINDS.index(kind) + int(10 * tau))
     for beta in ([0.5, 0.3] if kind == "jsd" else [0.5]):
         z, t = _rows(rng, 1, V, scale=1.5)
-        if kind == "tvd":
-            p, q = softmax(t[0]), softmax(z[0])
-            assert np.min(np.abs(p - q)) > 1e-5  # FD is only valid off the kinks
-        _, g = oracle.distill(z, t, loss_kind=kind, beta=beta)
-        fd = _fd_grad(z, t, kind, beta)
-        np.testing.assert_allclose(g, fd, atol=2e-8, rtol=1e-6)
+        while kind == "tvd" and np.min(np.abs(softmax(t[0] / tau) - softmax(z[0] / tau))) < 1e-5:
+            z, t = _rows(rng, 1, V, scale=1.5)  # FD is only valid off the kinks of |p - q|
+        _, g = oracle.distill(z, t, loss_kind=kind, beta=beta, temperature=tau)
+        fd = _fd_grad(z, t, kind, beta, tau)
+        np.testing.assert_allclose(g, fd, atol=4e-8, rtol=1e-6)
+
+
+def test_ce_matches_scipy_log_softmax():
+    """FT (Table 1): cross-entropy of q to the target's argmax label."""
+    rng = np.random.default_rng(21)
+    z, t = _rows(rng, 6, 300)
+    t[2, 7] = t[2, 9] = t[2].max() + 1.0  # tie: the lowest index is the label
+    for tau in (1.0, 0.7):
+        loss, _ = oracle.distill(z, t, loss_kind="ce", temperature=tau)
+        for n in range(6):
+            y = int(np.argmax(t[n]))
+            assert loss[n] == pytest.approx(-log_softmax(z[n] / tau)[y], rel=1e-12)
+    assert int(np.argmax(t[2])) == 7
+
+
+@pytest.mark.parametrize("kind", ["fkl", "rkl", "jsd", "tvd"])
+def test_temperature_against_library(kind):
+    """Section 4.1: temperature divides both rows' logits before the softmax."""
+    rng = np.random.default_rng(22)
+    z, t = _rows(rng, 4, 120)
+    tau = 0.6
+    loss, _ = oracle.distill(z, t, loss_kind=kind, beta=0.5, temperature=tau)
+    for n in range(4):
+        p, q = softmax(t[n] / tau), softmax(z[n] / tau)
+        m = 0.5 * (p + q)
+        want = {"fkl": entropy(p, q), "rkl": entropy(q, p),
+                "jsd": 0.5 * entropy(p, m) + 0.5 * entropy(q, m),
+                "tvd": 0.5 * cityblock(p, q)}[kind]
+        assert loss[n] == pytest.approx(want, rel=1e-10, abs=1e-14)
 
 
 @pytest.mark.parametrize("kind", KINDS)
@@ -127,7 +158,7 @@ def test_gradient_sums_to_zero(kind):
     assert np.max(np.abs(g.sum(axis=1))) < 1e-12
 
 
-@pytest.mark.parametrize("kind", KINDS)
+@pytest.mark.parametrize("kind", ["fkl", "rkl", "jsd", "tvd"])
 def test_identical_inputs_give_zero(kind):
     rng = np.random.default_rng(4)
     z = rng.normal(0, 3, (3, 400))

@@ -40,6 +40,11 @@ MUTANTS = [
     ("tvd_sign_flipped", "double s = (q > p) ? 0.5 : (q < p ? -0.5 : 0.0);",
      "double s = (q < p) ? 0.5 : (q > p ? -0.5 : 0.0);", 2),
     ("tvd_half_dropped", "l += 0.5 * fabs(p - q);", "l += fabs(p - q);", 1),
+    ("temperature_factor_dropped", "for (long j = 0; j < V; ++j) g[j] /= tau;", "", 1),
+    ("ce_label_from_draft", "long ystar = argmax_first(target + n * V, V);",
+     "long ystar = argmax_first(draft + n * V, V);", 1),
+    ("distill_temperature_ignored", "log_softmax(target + n * V, V, tau, lp);",
+     "log_softmax(target + n * V, V, 1.0, lp);", 1),
 ]
 
 
