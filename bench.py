@@ -5,6 +5,8 @@ distillation loss/gradient, at vocabulary 32000 (bf16 logits).
 One step is one pass of the whole hot path over synthetic inputs:
   verify   B=32 sequences, k=5 draft tokens, V=32000, T=1.0, then the greedy
            (T=0) pass over the same logits            -> 2 x 160 verified positions
+  distill  reverse KL on the rows the T=1 pass rejected, picked on the device
+           from its accepted counts                   -> one row per rejecting sequence
   distill  a buffer flush of N=65536 positions x V=32000, reverse KL then TVD,
            loss and d loss / d draft logits           -> 2 x 65536 distilled positions
 The value is positions (verified + distilled) per second for the whole job.
@@ -13,7 +15,7 @@ The value is positions (verified + distilled) per second for the whole job.
                     [--workload serving-32k|large-vocab]
 
 `--workload large-vocab` times verify at B=256, k=8, V=128256, T=0.7 followed
-by forward-KL distill of its mismatch rows (the 128k-vocabulary serving step).
+by forward-KL distill of its rejected rows (the 128k-vocabulary serving step).
 `--impl reference` times the CPU oracle (the correctness reference) on a
 bounded sample of the same workload, on the host cores.
 Prints one JSON line (rank 0).
@@ -164,7 +166,8 @@ def _setup_serving_32k(dev, distill_rows=None, rank=0):
     v = W.verify_inputs(spec_v, seed=shard_seed(W.seed_for(2), rank), device=dev)
     d = W.distill_inputs(spec_d, seed=shard_seed(W.seed_for(4), rank), device=dev)
     return {"v": v, "d": d, "spec_v": spec_v, "spec_d": spec_d,
-            "desc": "serving-32k: verify B=32 k=5 V=32000 bf16 T=1.0 + greedy T=0 pass; "
+            "desc": "serving-32k: verify B=32 k=5 V=32000 bf16 T=1.0 -> reverse-KL distill of its "
+                    "rejected rows (selected on the device) + greedy T=0 pass; "
                     f"distill flush N={spec_d.N} V=32000 bf16 reverse-KL + TVD"}
 
 
@@ -173,7 +176,7 @@ def _setup_large_vocab(dev, rank=0):
     v = W.verify_inputs(W.VERIFY[5], seed=shard_seed(W.seed_for(5), rank), device=dev)
     return {"v": v, "spec_v": W.VERIFY[5],
             "desc": "large-vocab: verify B=256 k=8 V=128256 bf16 T=0.7 -> forward-KL distill of "
-                    "the mismatch rows against target[:, :k]"}
+                    "its rejected rows (selected and compacted on the device)"}
 
 
 def _bytes_verify(B, k, V, s_in, greedy):
@@ -217,10 +220,12 @@ def run_ours(args):
         dist_pos = 2 * sd.N
         dist_bytes = sd.N * sd.V * (2 * 2 + 4)  # per launch
     else:
-        dl = torch.empty(sv.B, sv.k, sv.V, dtype=torch.float32, device=dev)
-        loss = torch.empty(sv.B, sv.k, dtype=torch.float32, device=dev)
-        kinds = ["fkl"]
+        kinds = []
 
+    rej_kind = "rkl" if wl == "serving-32k" else "fkl"
+    rej = osd.osd_distill_accepted(v["draft"], v["target"], vout.accepted, rej_kind)
+    torch.cuda.synchronize()
+    n_rej = int(rej.count.item())  # the inputs are the same every step, so is the count
     ev = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
     n_ver = 2 if wl == "serving-32k" else 1
 
@@ -229,21 +234,20 @@ def run_ours(args):
         # keep the device busy while the host enqueues the step, so that host-side
         # launch overhead never shows up inside the timed events
         torch.cuda._sleep(SLEEP_CYCLES)
-        e = [ev() for _ in range(1 + n_ver + len(kinds))]
+        e = [ev() for _ in range(2 + n_ver + (len(kinds) if wl == "serving-32k" else 0))]
         e[0].record(stream)
         osd.osd_verify(v["draft"], v["target"], v["tokens"], v["uniforms"], sv.temperature,
                        workspace=ws, out=vout)
         e[1].record(stream)
+        # the rows this pass rejected, straight from its accepted counts
+        osd.osd_distill_accepted(v["draft"], v["target"], vout.accepted, rej_kind, 0.5, out=rej)
+        e[2].record(stream)
         if wl == "serving-32k":
             osd.osd_verify(None, v["target"], v["greedy_tokens"], None, 0.0, workspace=ws, out=vout0)
-            e[2].record(stream)
+            e[3].record(stream)
             for i, kind in enumerate(kinds):
                 osd.osd_distill(d["draft"], d["target"], d["mask"], kind, 0.5, loss=loss, dlogits=dl)
-                e[3 + i].record(stream)
-        else:
-            osd.osd_distill(v["draft"], v["target"][:, :sv.k], vout.mismatch_mask, "fkl", 0.5,
-                            loss=loss, dlogits=dl)
-            e[2].record(stream)
+                e[4 + i].record(stream)
         record.append(e)
 
     warm = []
@@ -270,51 +274,57 @@ def run_ours(args):
 
     step_ms = [r[0].elapsed_time(r[-1]) for r in recs]
     verify_ms = [r[0].elapsed_time(r[1]) for r in recs]
+    rej_ms = [r[1].elapsed_time(r[2]) for r in recs]
     if wl == "serving-32k":
-        greedy_ms = [r[1].elapsed_time(r[2]) for r in recs]
-        dist_ms = [r[2 + i].elapsed_time(r[3 + i]) for r in recs for i in range(len(kinds))]
-        n_active = sd.N
-    else:
-        dist_ms = [r[1].elapsed_time(r[2]) for r in recs]
-        n_active = int(vout.mismatch_mask.sum().item())
+        greedy_ms = [r[2].elapsed_time(r[3]) for r in recs]
+        dist_ms = [r[3 + i].elapsed_time(r[4 + i]) for r in recs for i in range(len(kinds))]
     total_ms = job_time_ms(sum(step_ms), dev if world > 1 else None)
     ms_step = total_ms / args.steps
 
+    bytes_rej = n_rej * sv.V * (2 * s_in + 4) + sv.B * 4  # the rejected rows, plus the counts
     if wl == "serving-32k":
         ver_pos = 2 * sv.B * sv.k
-        positions = ver_pos + dist_pos
-        launches = 2 * 2 + len(kinds)
+        positions = ver_pos + dist_pos + n_rej
+        launches = 2 * 2 + 1 + len(kinds)
         bytes_v = _bytes_verify(sv.B, sv.k, sv.V, s_in, False)
         bytes_g = _bytes_verify(sv.B, sv.k, sv.V, s_in, True)
     else:
         ver_pos = sv.B * sv.k
-        positions = ver_pos + n_active
+        positions = ver_pos + n_rej
         launches = 2 + 1
         bytes_v = _bytes_verify(sv.B, sv.k, sv.V, s_in, False)
-        dist_bytes = n_active * sv.V * (2 * s_in + 4)
     value = job_throughput(positions, world, ms_step)
     peak, peak_src = _peak_hbm()
-    avg_dist = statistics.mean(dist_ms)
     avg_ver = statistics.mean(verify_ms)
+    avg_rej = statistics.mean(rej_ms)
     kernels = {
         "verify": {"us_per_call": avg_ver * 1e3, "alg_bytes": bytes_v,
                    "gbs": bytes_v / (avg_ver / 1e3) / 1e9,
                    "positions_per_s": sv.B * sv.k / (avg_ver / 1e3)},
-        "distill": {"us_per_call": avg_dist * 1e3, "alg_bytes": dist_bytes,
-                    "gbs": dist_bytes / (avg_dist / 1e3) / 1e9,
-                    "positions_per_s": (sd.N if wl == "serving-32k" else n_active) / (avg_dist / 1e3)},
+        "distill_rejected": {"us_per_call": avg_rej * 1e3, "alg_bytes": bytes_rej, "rows": n_rej,
+                             "gbs": bytes_rej / (avg_rej / 1e3) / 1e9,
+                             "positions_per_s": n_rej / (avg_rej / 1e3)},
     }
     if wl == "serving-32k":
+        avg_dist = statistics.mean(dist_ms)
+        kernels["distill"] = {"us_per_call": avg_dist * 1e3, "alg_bytes": dist_bytes,
+                              "gbs": dist_bytes / (avg_dist / 1e3) / 1e9,
+                              "positions_per_s": sd.N / (avg_dist / 1e3)}
         avg_g = statistics.mean(greedy_ms)
         kernels["verify_greedy"] = {"us_per_call": avg_g * 1e3, "alg_bytes": bytes_g,
                                     "gbs": bytes_g / (avg_g / 1e3) / 1e9,
                                     "positions_per_s": sv.B * sv.k / (avg_g / 1e3)}
     for kv in kernels.values():
         kv["frac_of_peak"] = kv["gbs"] / peak
-    achieved = kernels["distill"]["gbs"]
+    # the dominant kernel: distill on the default step, verify's row statistics at 128k
+    top = "distill" if wl == "serving-32k" else "verify"
+    achieved = kernels[top]["gbs"]
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                "frac": round(achieved / peak, 4), "traffic": _traffic("distill", DISTILL_SOURCES),
-                "kernel": "distill_kernel", "peak_source": peak_src}
+                "frac": round(achieved / peak, 4),
+                "traffic": (_traffic("distill", DISTILL_SOURCES) if top == "distill"
+                            else _traffic("verify", VERIFY_SOURCES)),
+                "kernel": "distill_kernel" if top == "distill" else "row_stats_kernel + verify_finalize_kernel",
+                "peak_source": peak_src}
 
     e2e = None
     if not args.no_e2e and (world == 1 or rank == 0):
@@ -357,6 +367,16 @@ def run_e2e(args, osd, setup, dev, stream, positions, wl):
     ws = torch.empty(osd.osd_verify_workspace_size(sv.B, sv.k, sv.V), dtype=torch.uint8, device=dev)
     h2d = sum(t.numel() * t.element_size() for k, t in host.items()
               if wl == "serving-32k" or k != "greedy_tokens")
+    rej_kind = "rkl" if wl == "serving-32k" else "fkl"
+    rej = osd.DistillAcceptedResult(torch.empty(sv.B, dtype=torch.float32, device=dev),
+                                    torch.empty(sv.B, sv.V, dtype=torch.float32, device=dev),
+                                    torch.empty(sv.B, dtype=torch.int32, device=dev),
+                                    torch.empty(1, dtype=torch.int32, device=dev))
+    h_rej = {"loss": torch.empty(sv.B, dtype=torch.float32).pin_memory(),
+             "seq": torch.empty(sv.B, dtype=torch.int32).pin_memory(),
+             "count": torch.empty(1, dtype=torch.int32).pin_memory()}
+    d2h = (h_out["acc"].numel() * 4 + h_out["tok"].numel() * 4 + h_out["mask"].numel()
+           + sum(t.numel() * 4 for t in h_rej.values()))
     if wl == "serving-32k":
         d = setup["d"]
         sd = setup["spec_d"]
@@ -366,12 +386,7 @@ def run_e2e(args, osd, setup, dev, stream, positions, wl):
         dl = torch.empty(sd.N, sd.V, dtype=torch.float32, device=dev)
         h_loss = torch.empty(2, sd.N, dtype=torch.float32).pin_memory()
         h2d += sum(t.numel() * t.element_size() for t in hd.values())
-        d2h = 2 * (h_out["acc"].numel() * 4 + h_out["tok"].numel() * 4 + h_out["mask"].numel()) + h_loss.numel() * 4
-    else:
-        loss = torch.empty(sv.B, sv.k, dtype=torch.float32, device=dev)
-        dl = torch.empty(sv.B, sv.k, sv.V, dtype=torch.float32, device=dev)
-        h_loss = torch.empty(1, sv.B * sv.k, dtype=torch.float32).pin_memory()
-        d2h = h_out["acc"].numel() * 4 + h_out["tok"].numel() * 4 + h_out["mask"].numel() + h_loss.numel() * 4
+        d2h += h_out["acc"].numel() * 4 + h_out["tok"].numel() * 4 + h_out["mask"].numel() + h_loss.numel() * 4
 
     def step():
         for k in host:
@@ -380,6 +395,10 @@ def run_e2e(args, osd, setup, dev, stream, positions, wl):
         h_out["acc"].copy_(r.accepted, non_blocking=True)
         h_out["tok"].copy_(r.out_tokens, non_blocking=True)
         h_out["mask"].copy_(r.mismatch_mask, non_blocking=True)
+        osd.osd_distill_accepted(dv["draft"], dv["target"], r.accepted, rej_kind, 0.5, out=rej)
+        h_rej["loss"].copy_(rej.loss, non_blocking=True)
+        h_rej["seq"].copy_(rej.seq_of_row, non_blocking=True)
+        h_rej["count"].copy_(rej.count, non_blocking=True)
         if wl == "serving-32k":
             r0 = osd.osd_verify(None, dv["target"], dv["greedy_tokens"], None, 0.0, workspace=ws)
             h_out["acc"].copy_(r0.accepted, non_blocking=True)
@@ -390,9 +409,6 @@ def run_e2e(args, osd, setup, dev, stream, positions, wl):
             for i, kind in enumerate(("rkl", "tvd")):
                 osd.osd_distill(dd["draft"], dd["target"], None, kind, 0.5, loss=loss, dlogits=dl)
                 h_loss[i].copy_(loss, non_blocking=True)
-        else:
-            osd.osd_distill(dv["draft"], dv["target"][:, :sv.k], r.mismatch_mask, "fkl", 0.5, loss=loss, dlogits=dl)
-            h_loss[0].copy_(loss.reshape(-1), non_blocking=True)
 
     for _ in range(max(1, args.warmup)):
         step()
@@ -405,8 +421,6 @@ def run_e2e(args, osd, setup, dev, stream, positions, wl):
     e1.record(stream)
     e1.synchronize()
     ms = e0.elapsed_time(e1) / n
-    if wl != "serving-32k":
-        positions = sv.B * sv.k + int(h_out["mask"].sum())
     return {"value": round(positions / (ms / 1e3), 1), "unit": "positions/s", "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "ms_per_step": round(ms, 3), "steps": n,
             "note": "dlogits stays on the device, where the draft model's backward pass consumes it"}
@@ -414,8 +428,9 @@ def run_e2e(args, osd, setup, dev, stream, positions, wl):
 
 # ----------------------------------------------------------------------------- CPU oracle
 def _oracle_step_time(setup, n_rows, threads):
-    """Time the oracle on the verify batch (whole) and on n_rows distill rows per
-    loss kind; returns (seconds, positions) of that bounded sample."""
+    """Time the oracle on the verify batch (whole, with the distillation of the
+    rows it rejects) and on n_rows distill rows per loss kind; returns
+    (seconds, positions) of that bounded sample."""
     import concurrent.futures as cf
 
     import numpy as np
@@ -434,23 +449,29 @@ def _oracle_step_time(setup, n_rows, threads):
         step = max(1, (n + parts - 1) // parts)
         return [(i, min(n, i + step)) for i in range(0, n, step)]
 
+    rej_kind = "rkl" if "d" in setup else "fkl"
+
+    def verify_and_distill(a, b):
+        r = oracle.verify(z[a:b], t[a:b], y[a:b], u[a:b], T)
+        n_rej = oracle.distill_rejected(z[a:b], t[a:b], r["accepted"], rej_kind, 0.5)[3]
+        return (b - a) * sv.k + n_rej
+
     jobs = []
     for (a, b) in chunks(sv.B, threads):
-        jobs.append(lambda a=a, b=b: oracle.verify(z[a:b], t[a:b], y[a:b], u[a:b], T))
+        jobs.append(lambda a=a, b=b: verify_and_distill(a, b))
         if "d" in setup:
-            jobs.append(lambda a=a, b=b: oracle.verify(z[a:b], t[a:b], yg[a:b], u[a:b], 0.0))
-    positions = sv.B * sv.k * (2 if "d" in setup else 1)
+            jobs.append(lambda a=a, b=b: (oracle.verify(z[a:b], t[a:b], yg[a:b], u[a:b], 0.0), (b - a) * sv.k)[1])
     if "d" in setup:
         d = setup["d"]
         zd = d["draft"][:n_rows].cpu()
         td = d["target"][:n_rows].cpu()
         for kind in ("rkl", "tvd"):
             for (a, b) in chunks(n_rows, threads):
-                jobs.append(lambda a=a, b=b, kind=kind: oracle.distill(zd[a:b], td[a:b], None, kind, 0.5))
-        positions += 2 * n_rows
+                jobs.append(lambda a=a, b=b, kind=kind: (oracle.distill(zd[a:b], td[a:b], None, kind, 0.5),
+                                                         b - a)[1])
     t0 = time.perf_counter()
     with cf.ThreadPoolExecutor(max_workers=threads) as ex:
-        list(ex.map(lambda f: f(), jobs))
+        positions = sum(ex.map(lambda f: f(), jobs))
     return time.perf_counter() - t0, positions
 
 
@@ -459,7 +480,8 @@ def cpu_baseline(args, setup):
     n_rows = args.cpu_rows
     secs, pos = _oracle_step_time(setup, n_rows, threads)
     return {"value": round(pos / secs, 2), "unit": "positions/s", "cores": threads, "kind": "oracle",
-            "sample": f"whole verify batch (both passes) + {n_rows} distill rows per loss kind, "
+            "sample": f"whole verify batch (both passes, with its rejected rows distilled) + {n_rows} "
+                      f"distill rows per loss kind, "
                       f"{secs:.1f} s on {threads} host threads (double-precision C oracle)"}
 
 
@@ -482,7 +504,8 @@ def run_reference(args):
         times.append(s)
     ms = 1e3 * sum(times) / len(times)
     value = pos / (ms / 1e3)
-    sample = (f"per step: whole verify batch (both passes) + {args.cpu_rows} distill rows per loss kind "
+    sample = (f"per step: whole verify batch (both passes, with its rejected rows distilled) + "
+              f"{args.cpu_rows} distill rows per loss kind "
               f"of the same workload, {threads} host threads")
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 2), "unit": "positions/s",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3),

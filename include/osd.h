@@ -2,7 +2,7 @@
  * osd.h -- C ABI of the GB300 (sm_103a) hot path of Online Speculative
  * Decoding (Liu et al., "Online Speculative Decoding", ICML 2024).
  *
- * Two operations run every serving step of the paper's Algorithm 1:
+ * The operations of every serving step of the paper's Algorithm 1:
  *
  *   osd_verify   speculative-sampling verification of k draft tokens against
  *                k+1 target distributions (Section 3 and Appendix A.1; the
@@ -11,9 +11,11 @@
  *                mask that feeds the temporary buffer R of Algorithm 1.
  *   osd_distill  the per-position distillation loss D(p || q_theta) of Eq. 2
  *                with D one of the distances of Eq. 3 (forward KL, reverse
- *                KL, JSD[beta]) or total variation distance, and its gradient
- *                with respect to the draft logits (the analytic update step
- *                of Algorithm 1).
+ *                KL, JSD[beta]), total variation distance or the label
+ *                cross-entropy, and its gradient with respect to the draft
+ *                logits (the analytic update step of Algorithm 1).
+ *   osd_distill_accepted  the same on the rows osd_verify rejected, selected
+ *                and compacted on the device from its accepted counts.
  *
  * Conventions shared by every entry point:
  *   - All array arguments are DEVICE pointers to caller-owned memory on the
@@ -71,7 +73,8 @@ typedef enum osd_loss {
 const char *osd_status_string(osd_status status);
 
 /* ABI version of this library: (major << 16) | minor.  2.0 added the
- * temperature argument of osd_distill and the OSD_CE loss. */
+ * temperature argument of osd_distill and the OSD_CE loss; 2.1 added
+ * osd_distill_accepted. */
 int osd_abi_version(void);
 
 /*
@@ -185,6 +188,40 @@ osd_status osd_distill(const void *draft_logits, const void *target_logits,
                        int64_t t_stride_g, int64_t t_stride_p,
                        const uint8_t *mask, osd_loss kind, float beta, float temperature,
                        float *loss, float *dlogits, int32_t *status, void *stream);
+
+/*
+ * Distillation of the rows that verification rejected, chosen on the device
+ * (Algorithm 1: the first rejected position of each step and the target's
+ * distribution there go into the buffer R; Eq. 2-3 give the loss on them).
+ *
+ * Sequence b contributes the row at position a = accepted[b] when 0 <= a < k,
+ * the first draft token osd_verify rejected (where its mismatch_mask is 1):
+ * draft row (b, a) of draft_logits [B, k, V] and target row (b, a) of
+ * target_logits [B, k+1, V], both contiguous, the layouts osd_verify reads.
+ * Sequences with a == k (all accepted) or a == -1 (bad tokens) contribute
+ * nothing.  Loss, gradient and temperature are those of osd_distill.
+ *
+ * Results go to a stable partition of the sequences: the n active ones
+ * first, in increasing b, then the inactive ones, in increasing b.
+ *
+ * accepted      [B] int32 device, as osd_verify writes it; read on the device,
+ *               so the call can follow osd_verify on the same stream with no
+ *               host synchronisation (and be captured in the same graph).
+ * loss          [B] fp32 out: slot r < n holds the loss of sequence
+ *               seq_of_row[r]; slots r >= n are set to 0.
+ * dlogits       [B, V] fp32 out: rows r < n hold the gradients; rows r >= n
+ *               are not written.
+ * seq_of_row    [B] int32 out, nullable: the sequence b behind slot r.
+ * count         device int32 out, nullable: n.
+ * status        as in osd_distill.
+ * Returns OSD_ERR_INVALID_ARG for k < 1, B < 0, a null `accepted` with
+ * B > 0, and the osd_distill argument errors.  B = 0 only sets *count = 0.
+ */
+osd_status osd_distill_accepted(const void *draft_logits, const void *target_logits,
+                                osd_dtype dtype, int B, int k, int V, const int32_t *accepted,
+                                osd_loss kind, float beta, float temperature,
+                                float *loss, float *dlogits, int32_t *seq_of_row, int32_t *count,
+                                int32_t *status, void *stream);
 
 #ifdef __cplusplus
 }

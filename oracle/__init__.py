@@ -170,3 +170,37 @@ def distill(draft_logits, target_logits, mask=None, loss_kind="fkl", beta=0.5,
     if rc != 0:
         raise ValueError("osd_oracle_distill rejected its arguments")
     return loss.reshape(lead), g.reshape(*lead, V)
+
+
+def distill_rejected(draft_logits, target_logits, accepted, loss_kind="rkl", beta=0.5, temperature=1.0):
+    """Distillation on the positions verification rejected (Algorithm 1).
+
+    Each serving step of Algorithm 1 stores, for every sequence whose draft
+    proposal was cut short, the first rejected position and the target's
+    distribution there in the buffer R; the loss of Eq. 2 is then taken over R.
+    Sequence b has a = accepted[b] accepted tokens: it contributes draft row
+    (b, a) of draft_logits [B, k, V] and target row (b, a) of target_logits
+    [B, k+1, V] when 0 <= a < k, and nothing when a == k (every token
+    accepted) or a == -1 (a bad draft token).
+
+    Returns (loss [B], dlogits [B, V], seq_of_row [B], count) in the order of a
+    stable partition: the count active sequences first in increasing b, then
+    the inactive ones; loss is 0 and dlogits NaN in the inactive slots.
+    """
+    z = _np(draft_logits, np.float64)
+    t = _np(target_logits, np.float64)
+    acc = _np(accepted, np.int64).reshape(-1)
+    B, k, V = z.shape
+    assert t.shape == (B, k + 1, V) and acc.shape == (B,)
+    active = [b for b in range(B) if 0 <= acc[b] < k]
+    inactive = [b for b in range(B) if not 0 <= acc[b] < k]
+    loss = np.zeros(B, np.float64)
+    g = np.full((B, V), np.nan, np.float64)
+    if active:
+        rows_z = np.stack([z[b, acc[b]] for b in active])
+        rows_t = np.stack([t[b, acc[b]] for b in active])
+        l, gr = distill(rows_z, rows_t, None, loss_kind, beta, temperature=temperature)
+        loss[:len(active)] = l
+        g[:len(active)] = gr
+    seq = np.array(active + inactive, np.int64)
+    return loss, g, seq, len(active)

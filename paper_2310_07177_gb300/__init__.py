@@ -29,7 +29,7 @@ VERIFY_MAX_V = 1 << 21
 
 # every symbol include/osd.h declares
 EXPORTS = ("osd_status_string", "osd_abi_version", "osd_verify_workspace_size",
-           "osd_verify", "osd_verify_noalloc", "osd_distill")
+           "osd_verify", "osd_verify_noalloc", "osd_distill", "osd_distill_accepted")
 
 
 class OsdError(RuntimeError):
@@ -66,6 +66,8 @@ def load_library():
     lib.osd_verify_noalloc.argtypes = [vp, vp, i32, i32, i32, i32, vp, vp, f32, vp, vp, vp, vp, vp, vp]
     lib.osd_distill.restype = i32
     lib.osd_distill.argtypes = [vp, vp, i32, i32, i32, i32, i64, i64, i64, i64, vp, i32, f32, f32, vp, vp, vp, vp]
+    lib.osd_distill_accepted.restype = i32
+    lib.osd_distill_accepted.argtypes = [vp, vp, i32, i32, i32, i32, vp, i32, f32, f32, vp, vp, vp, vp, vp, vp]
     _lib = lib
     return lib
 
@@ -238,3 +240,47 @@ def osd_distill(draft_logits: torch.Tensor, target_logits: torch.Tensor, mask: O
     if st != OSD_OK:
         raise OsdError(st, "osd_distill")
     return loss, dlogits
+
+
+class DistillAcceptedResult(NamedTuple):
+    """Outputs of osd_distill_accepted: slot r < count holds sequence seq_of_row[r]."""
+    loss: torch.Tensor        # [B] fp32 (0 beyond count)
+    dlogits: torch.Tensor     # [B, V] fp32 (rows beyond count untouched)
+    seq_of_row: torch.Tensor  # [B] int32
+    count: torch.Tensor       # [1] int32 on the device
+
+
+def osd_distill_accepted(draft_logits: torch.Tensor, target_logits: torch.Tensor, accepted: torch.Tensor,
+                         loss_kind: str = "rkl", beta: float = 0.5, *, temperature: float = 1.0,
+                         out: Optional[DistillAcceptedResult] = None, status: Optional[torch.Tensor] = None,
+                         stream: Optional[torch.cuda.Stream] = None) -> DistillAcceptedResult:
+    """Distil the rows verification rejected (Algorithm 1's buffer R, Eq. 2-3).
+
+    ``draft_logits`` [B,k,V] and ``target_logits`` [B,k+1,V] are the contiguous
+    tensors osd_verify read; ``accepted`` [B] int32 is its output.  Sequence b
+    contributes row (b, accepted[b]) when that is < k; results are compacted on
+    the device, active sequences first (see ``DistillAcceptedResult``).
+    """
+    lib = load_library()
+    dev = _need_cuda(draft_logits, target_logits, accepted, status, *(out or ()))
+    if draft_logits.dim() != 3 or target_logits.dim() != 3:
+        raise ValueError("draft_logits must be [B,k,V] and target_logits [B,k+1,V]")
+    B, k, V = draft_logits.shape
+    if (tuple(target_logits.shape) != (B, k + 1, V) or draft_logits.dtype != target_logits.dtype
+            or not draft_logits.is_contiguous() or not target_logits.is_contiguous()):
+        raise ValueError("draft_logits [B,k,V] and target_logits [B,k+1,V] must be contiguous, same dtype")
+    if accepted.dtype != torch.int32 or tuple(accepted.shape) != (B,) or not accepted.is_contiguous():
+        raise ValueError("accepted must be contiguous int32 [B]")
+    if out is None:
+        out = DistillAcceptedResult(torch.empty(B, dtype=torch.float32, device=dev),
+                                    torch.empty(B, V, dtype=torch.float32, device=dev),
+                                    torch.empty(B, dtype=torch.int32, device=dev),
+                                    torch.empty(1, dtype=torch.int32, device=dev))
+    kind = LOSS_KINDS[loss_kind] if isinstance(loss_kind, str) else int(loss_kind)
+    st = lib.osd_distill_accepted(_ptr(draft_logits), _ptr(target_logits), _dtype_code(draft_logits), B, k, V,
+                                  _ptr(accepted), kind, float(beta), float(temperature), _ptr(out.loss),
+                                  _ptr(out.dlogits), _ptr(out.seq_of_row), _ptr(out.count), _ptr(status),
+                                  _stream(dev, stream))
+    if st != OSD_OK:
+        raise OsdError(st, "osd_distill_accepted")
+    return out

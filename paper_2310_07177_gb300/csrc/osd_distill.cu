@@ -17,6 +17,7 @@
 // Every CTA merges the cluster's partials in rank order, so all CTAs of a row
 // see bit-identical statistics.  Logs and exponentials use the hardware
 // lg2/ex2 units in base 2; loss terms are converted to nats at the end.
+#include <atomic>
 #include <climits>
 #include <cmath>
 #include <cstdint>
@@ -48,6 +49,13 @@ struct DistParams {
     float* loss;
     float* dlogits;
     int32_t* status;
+    // Rows chosen by verification (accepted != null): row b of the launch is
+    // position accepted[b] of sequence b when 0 <= accepted[b] < k (G = B, P = 1)
+    // and its results go to slot r of a stable partition, active sequences first.
+    const int32_t* accepted;
+    int k;
+    int32_t* seq_of_row;  // nullable: seq_of_row[r] = b
+    int32_t* count;       // nullable: number of active sequences
     int csize;  // CTAs per row (cluster size)
     int span;   // vocabulary entries per CTA (multiple of 64)
 };
@@ -281,17 +289,48 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     __shared__ int s_err;
     __shared__ float s_cu, s_cv, s_loss, s_K, s_tp;
     __shared__ Label red_l[kDistThreads / 32];
+    __shared__ int2 red_i[kDistThreads / 32];
 
     const int tid = threadIdx.x;
     const int csize = p.csize;
     const float c = p.c, inv_tau = p.inv_tau;
     const int rank = (csize > 1) ? static_cast<int>(cluster_rank()) : 0;
-    const long long row = blockIdx.x / csize;
-    if (p.mask && !p.mask[row]) {  // uniform over the cluster; no shared memory is exchanged
-        if (rank == 0 && tid == 0) p.loss[row] = 0.f;
-        return;
+    long long row = blockIdx.x / csize;  // the launch row; from here on, the output row
+    long long g, pp;
+    if (p.accepted) {
+        // sequence b = row keeps position a = accepted[b] when a < k (the first rejected
+        // draft token); the output slot counts the active sequences before it
+        const int b = static_cast<int>(row), a = p.accepted[b];
+        const bool active = a >= 0 && a < p.k;
+        int2 cnt = make_int2(0, 0);  // (active before b, active in total)
+        for (int i = tid; i < p.G; i += kDistThreads) {
+            const int ai = p.accepted[i];
+            const int act = (ai >= 0 && ai < p.k) ? 1 : 0;
+            cnt.x += (i < b) ? act : 0;
+            cnt.y += act;
+        }
+        cnt = block_reduce<kDistThreads>(cnt, [](int2 u, int2 v) { return make_int2(u.x + v.x, u.y + v.y); },
+                                         red_i);
+        const long long slot = active ? cnt.x : cnt.y + (b - cnt.x);
+        if (rank == 0 && tid == 0) {
+            if (p.seq_of_row) p.seq_of_row[slot] = b;
+            if (p.count && b == 0) *p.count = cnt.y;
+        }
+        row = slot;
+        if (!active) {  // uniform over the cluster
+            if (rank == 0 && tid == 0) p.loss[row] = 0.f;
+            return;
+        }
+        g = b;
+        pp = a;
+    } else {
+        if (p.mask && !p.mask[row]) {  // uniform over the cluster; no shared memory is exchanged
+            if (rank == 0 && tid == 0) p.loss[row] = 0.f;
+            return;
+        }
+        g = row / p.P;
+        pp = row - g * p.P;
     }
-    const long long g = row / p.P, pp = row - g * p.P;
     const In* zrow = static_cast<const In*>(p.draft) + g * p.dsg + pp * p.dsp;
     const In* trow = static_cast<const In*>(p.target) + g * p.tsg + pp * p.tsp;
     const int V = p.V;
@@ -699,9 +738,22 @@ template <typename In, int kKind, bool kAligned>
 static cudaError_t launch_distill_kind(const DistParams& dp, long long rows, size_t smem, cudaStream_t s) {
     auto kern = distill_kernel<In, kKind, kAligned>;
     if (smem > 48 * 1024) {
-        const cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                   static_cast<int>(smem));
+        // the opt-in is per device and kernel; set it once, so that later calls
+        // (including ones under stream capture) make no attribute call
+        static std::atomic<int> allowed[64];
+        int dev = 0;
+        cudaError_t e = cudaGetDevice(&dev);
         if (e != cudaSuccess) return e;
+        if (dev < 0 || dev >= 64 || allowed[dev].load(std::memory_order_relaxed) < static_cast<int>(smem)) {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+            if (e != cudaSuccess) return e;
+            if (dev >= 0 && dev < 64) {
+                int cur = allowed[dev].load(std::memory_order_relaxed);
+                while (cur < static_cast<int>(smem) &&
+                       !allowed[dev].compare_exchange_weak(cur, static_cast<int>(smem))) {
+                }
+            }
+        }
     }
     return launch(kern, dim3(static_cast<unsigned>(rows * dp.csize)), dim3(kDistThreads), smem, s,
                   dp.csize, dp);
@@ -735,14 +787,12 @@ static bool distill_shape(int V, size_t es, int* csize, int* span) {
     return true;
 }
 
-}  // namespace osd
-
-extern "C" osd_status osd_distill(const void* draft_logits, const void* target_logits, osd_dtype dtype,
-                                  int G, int P, int V, int64_t d_stride_g, int64_t d_stride_p,
-                                  int64_t t_stride_g, int64_t t_stride_p, const uint8_t* mask, osd_loss kind,
-                                  float beta, float temperature, float* loss, float* dlogits, int32_t* status,
-                                  void* stream) {
-    using namespace osd;
+// Shared by both entry points: argument checks, shape, and the launch.
+static osd_status distill_run(const void* draft_logits, const void* target_logits, osd_dtype dtype, int G,
+                              int P, int V, int64_t d_stride_g, int64_t d_stride_p, int64_t t_stride_g,
+                              int64_t t_stride_p, const uint8_t* mask, const int32_t* accepted, int k,
+                              int32_t* seq_of_row, int32_t* count, osd_loss kind, float beta,
+                              float temperature, float* loss, float* dlogits, int32_t* status, void* stream) {
     if (dtype != OSD_F32 && dtype != OSD_BF16) return OSD_ERR_INVALID_ARG;
     if (kind < OSD_FKL || kind > OSD_CE) return OSD_ERR_INVALID_ARG;
     if (!(temperature > 0.f) || !std::isfinite(temperature)) return OSD_ERR_INVALID_ARG;
@@ -755,11 +805,14 @@ extern "C" osd_status osd_distill(const void* draft_logits, const void* target_l
     const long long rows = static_cast<long long>(G) * P;
     if (rows * csize > INT_MAX) return OSD_ERR_UNSUPPORTED;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (status) {
-        if (!aligned_to(status, 4)) return OSD_ERR_INVALID_ARG;
-    }
+    if (status && !aligned_to(status, 4)) return OSD_ERR_INVALID_ARG;
+    if ((seq_of_row && !aligned_to(seq_of_row, 4)) || (count && !aligned_to(count, 4))) return OSD_ERR_INVALID_ARG;
     if (rows == 0) {
-        return status ? from_cuda(cudaMemsetAsync(status, 0, sizeof(int32_t), s)) : OSD_OK;
+        if (status) {
+            const cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int32_t), s);
+            if (e != cudaSuccess) return OSD_ERR_CUDA;
+        }
+        return count ? from_cuda(cudaMemsetAsync(count, 0, sizeof(int32_t), s)) : OSD_OK;
     }
     if (!draft_logits || !target_logits || !loss || !dlogits) return OSD_ERR_INVALID_ARG;
     if (!aligned_to(draft_logits, es) || !aligned_to(target_logits, es) || !aligned_to(loss, 4) ||
@@ -769,16 +822,18 @@ extern "C" osd_status osd_distill(const void* draft_logits, const void* target_l
         const cudaError_t e = cudaMemsetAsync(status, 0, sizeof(int32_t), s);
         if (e != cudaSuccess) return OSD_ERR_CUDA;
     }
-    auto row_ok = [&](int64_t stride, int count) { return count <= 1 || (stride * int64_t(es)) % 16 == 0; };
+    auto row_ok = [&](int64_t stride, int n) { return n <= 1 || (stride * int64_t(es)) % 16 == 0; };
+    const int p_rows = accepted ? k : P;  // the position index runs over k rows in accepted mode
     const bool aligned = aligned_to(draft_logits, 16) && aligned_to(target_logits, 16) &&
                          aligned_to(dlogits, 16) && (size_t(V) * 4) % 16 == 0 &&
-                         row_ok(d_stride_g, G) && row_ok(d_stride_p, P) && row_ok(t_stride_g, G) &&
-                         row_ok(t_stride_p, P);
+                         row_ok(d_stride_g, G) && row_ok(d_stride_p, p_rows) && row_ok(t_stride_g, G) &&
+                         row_ok(t_stride_p, p_rows);
     DistParams dp;
     dp.draft = draft_logits; dp.target = target_logits;
     dp.G = G; dp.P = P; dp.V = V;
     dp.dsg = d_stride_g; dp.dsp = d_stride_p; dp.tsg = t_stride_g; dp.tsp = t_stride_p;
     dp.mask = mask; dp.beta = beta; dp.loss = loss; dp.dlogits = dlogits; dp.status = status;
+    dp.accepted = accepted; dp.k = k; dp.seq_of_row = seq_of_row; dp.count = count;
     dp.c = static_cast<float>(1.4426950408889634074 / static_cast<double>(temperature));
     dp.inv_tau = static_cast<float>(1.0 / static_cast<double>(temperature));
     {
@@ -796,4 +851,29 @@ extern "C" osd_status osd_distill(const void* draft_logits, const void* target_l
         e = aligned ? launch_distill_dtype<float, true>(kind, dp, rows, smem, s)
                     : launch_distill_dtype<float, false>(kind, dp, rows, smem, s);
     return from_cuda(e);
+}
+
+}  // namespace osd
+
+extern "C" osd_status osd_distill(const void* draft_logits, const void* target_logits, osd_dtype dtype,
+                                  int G, int P, int V, int64_t d_stride_g, int64_t d_stride_p,
+                                  int64_t t_stride_g, int64_t t_stride_p, const uint8_t* mask, osd_loss kind,
+                                  float beta, float temperature, float* loss, float* dlogits, int32_t* status,
+                                  void* stream) {
+    return osd::distill_run(draft_logits, target_logits, dtype, G, P, V, d_stride_g, d_stride_p, t_stride_g,
+                            t_stride_p, mask, nullptr, 0, nullptr, nullptr, kind, beta, temperature, loss,
+                            dlogits, status, stream);
+}
+
+extern "C" osd_status osd_distill_accepted(const void* draft_logits, const void* target_logits,
+                                           osd_dtype dtype, int B, int k, int V, const int32_t* accepted,
+                                           osd_loss kind, float beta, float temperature, float* loss,
+                                           float* dlogits, int32_t* seq_of_row, int32_t* count,
+                                           int32_t* status, void* stream) {
+    if (k < 1 || B < 0 || V < 1) return OSD_ERR_INVALID_ARG;
+    if (B > 0 && (!accepted || !osd::aligned_to(accepted, 4))) return OSD_ERR_INVALID_ARG;
+    const int64_t kv = int64_t(k) * V;
+    return osd::distill_run(draft_logits, target_logits, dtype, B, 1, V, kv, V, kv + V, V, nullptr,
+                            B > 0 ? accepted : nullptr, k, seq_of_row, count, kind, beta, temperature, loss,
+                            dlogits, status, stream);
 }

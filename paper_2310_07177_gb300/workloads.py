@@ -139,3 +139,15 @@ def distill_inputs(spec: DistillSpec, seed: int, device="cpu", N: Optional[int] 
 
 def seed_for(config_id: int) -> int:
     return SEED_BASE + config_id
+
+
+def accepted_inputs(B: int, k: int, seed: int, p_bad: float = 0.05, p_all: float = 0.25) -> torch.Tensor:
+    """Accepted counts [B] int32 on the CPU as verification reports them: -1
+    (a bad draft token) with probability p_bad, k (every token accepted) with
+    probability p_all, otherwise uniform over 0..k-1."""
+    g = _gen(seed, "cpu")
+    u = torch.rand(B, generator=g)
+    a = torch.randint(0, k, (B,), generator=g, dtype=torch.int32)
+    a[u < p_all + p_bad] = k
+    a[u < p_bad] = -1
+    return a

@@ -79,6 +79,22 @@ def test_argument_errors_return_before_any_launch(lib):
                            None) == osd.OSD_ERR_INVALID_ARG
     assert lib.osd_distill(None, None, 1, 0, 4, 16, 16, 0, 16, 0, None, 0, 0.5, 1.0, None, None, None,
                            None) == osd.OSD_OK
+    # distill_accepted: k < 1, negative B, missing accepted, bad kind / temperature; B = 0 with no count
+    fa = lib.osd_distill_accepted
+    assert fa(fake, fake, 1, 2, 0, 16, fake, 0, 0.5, 1.0, fake, fake, None, None, None,
+              None) == osd.OSD_ERR_INVALID_ARG
+    assert fa(fake, fake, 1, -1, 2, 16, fake, 0, 0.5, 1.0, fake, fake, None, None, None,
+              None) == osd.OSD_ERR_INVALID_ARG
+    assert fa(fake, fake, 1, 2, 2, 16, None, 0, 0.5, 1.0, fake, fake, None, None, None,
+              None) == osd.OSD_ERR_INVALID_ARG
+    assert fa(fake, fake, 1, 2, 2, 16, fake, 9, 0.5, 1.0, fake, fake, None, None, None,
+              None) == osd.OSD_ERR_INVALID_ARG
+    assert fa(fake, fake, 1, 2, 2, 16, fake, 0, 0.5, 0.0, fake, fake, None, None, None,
+              None) == osd.OSD_ERR_INVALID_ARG
+    assert fa(fake, fake, 1, 2, 2, 500000, fake, 0, 0.5, 1.0, fake, fake, None, None, None,
+              None) == osd.OSD_ERR_UNSUPPORTED
+    assert fa(None, None, 1, 0, 2, 16, None, 0, 0.5, 1.0, None, None, None, None, None,
+              None) == osd.OSD_OK
 
 
 def test_product_path_fails_loudly_without_library(tmp_path, monkeypatch):
