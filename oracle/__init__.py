@@ -71,6 +71,9 @@ def _load():
                                            ctypes.c_double, ctypes.c_double, dp, dp]
         lib.osd_oracle_log_softmax.restype = None
         lib.osd_oracle_log_softmax.argtypes = [dp, L, ctypes.c_double, dp]
+        lib.osd_oracle_mixed_sample.restype = ctypes.c_int
+        lib.osd_oracle_mixed_sample.argtypes = [dp, dp, L, L, L, L, dp, ctypes.c_double, ctypes.c_double,
+                                                i32p, dp]
         _lib = lib
         return lib
 
@@ -204,3 +207,28 @@ def distill_rejected(draft_logits, target_logits, accepted, loss_kind="rkl", bet
         g[:len(active)] = gr
     seq = np.array(active + inactive, np.int64)
     return loss, g, seq, len(active)
+
+
+def mixed_sample(draft_logits, target_logits, uniforms, beta, temperature=1.0):
+    """One token per row from beta p + (1 - beta) q (Section 4.1, mixed
+    sampling), p = softmax(target / T), q = softmax(draft / T), by inverse CDF
+    in ascending vocabulary order with uniforms [N].  Rows are [N, V] (any
+    leading shape is flattened).  Returns (tokens [N] int32, cdf_gap [N])."""
+    lib = _load()
+    z = _np(draft_logits, np.float64)
+    t = _np(target_logits, np.float64)
+    V = z.shape[-1]
+    z = z.reshape(-1, V)
+    t = t.reshape(-1, V)
+    N = z.shape[0]
+    assert t.shape == (N, V)
+    u = _np(uniforms, np.float64).reshape(-1)
+    assert u.shape == (N,)
+    tok = np.empty(N, np.int32)
+    gap = np.empty(N, np.float64)
+    rc = lib.osd_oracle_mixed_sample(_ptr(z, ctypes.c_double), _ptr(t, ctypes.c_double), N, V, V, V,
+                                     _ptr(u, ctypes.c_double), float(beta), float(temperature),
+                                     _ptr(tok, ctypes.c_int32), _ptr(gap, ctypes.c_double))
+    if rc != 0:
+        raise ValueError("osd_oracle_mixed_sample rejected its arguments")
+    return tok, gap

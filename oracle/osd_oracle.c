@@ -11,6 +11,9 @@
  *                       variation distance, and the analytic gradient with
  *                       respect to the draft logits (Algorithm 1, "Update
  *                       q_theta ... analytically").
+ *   osd_oracle_mixed_sample  one draw per position from the mixture
+ *                       beta p + (1 - beta) q_theta (Section 4.1, mixed
+ *                       sampling of the tokens the distillation is run on).
  *
  * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and the
  * cpu_baseline leg of bench.py may load this library.  It shares no code,
@@ -284,5 +287,59 @@ int osd_oracle_distill(const double *draft, const double *target, long N, long V
         loss[n] = l;
     }
     free(lq); free(lp);
+    return 0;
+}
+
+/*
+ * Mixed-token sampling, Section 4.1: y ~ beta p + (1 - beta) q, with
+ * p = softmax(t / tau) and q = softmax(z / tau) of one position, for each of
+ * N rows (row n of the draft starts at draft + n*d_stride, of the target at
+ * target + n*t_stride).  The draw is one inverse-CDF step over the mixture
+ * weights w_j = beta p_j + (1 - beta) q_j in ascending vocabulary order, with
+ * the conventions of the verify oracle's extra token: j* = min{ j : C_j > u W },
+ * W = sum_j w_j; if rounding leaves no such j, the largest j with w_j > 0.
+ *
+ * uniforms [N]  u in [0, 1);  tokens [N] out;  cdf_gap [N] out (nullable):
+ * distance of u W to the nearest edge of the chosen CDF step, divided by W.
+ * Returns 0, or -1 on bad arguments / allocation failure.
+ */
+int osd_oracle_mixed_sample(const double *draft, const double *target, long N, long V,
+                            long d_stride, long t_stride, const double *uniforms,
+                            double beta, double tau, int32_t *tokens, double *cdf_gap)
+{
+    if (N < 0 || V < 1 || !(tau > 0.0) || !(beta >= 0.0 && beta <= 1.0)) return -1;
+    double *lq = (double *)malloc(sizeof(double) * (size_t)V);
+    double *lp = (double *)malloc(sizeof(double) * (size_t)V);
+    double *w  = (double *)malloc(sizeof(double) * (size_t)V);
+    if (!lq || !lp || !w) { free(lq); free(lp); free(w); return -1; }
+    for (long n = 0; n < N; ++n) {
+        log_softmax(draft + n * d_stride, V, tau, lq);
+        log_softmax(target + n * t_stride, V, tau, lp);
+        double W = 0.0;
+        for (long j = 0; j < V; ++j) {
+            w[j] = beta * exp(lp[j]) + (1.0 - beta) * exp(lq[j]);
+            W += w[j];
+        }
+        const double target_mass = uniforms[n] * W;
+        double C = 0.0, Cprev = 0.0;
+        long pick = -1;
+        for (long j = 0; j < V; ++j) {
+            Cprev = C;
+            C += w[j];
+            if (C > target_mass) { pick = j; break; }
+        }
+        if (pick < 0) {                              /* rounding left none */
+            for (long j = V - 1; j >= 0; --j)
+                if (w[j] > 0.0) { pick = j; break; }
+            Cprev = W - w[pick];
+            C = W;
+        }
+        tokens[n] = (int32_t)pick;
+        if (cdf_gap) {
+            double g1 = C - target_mass, g0 = target_mass - Cprev;
+            cdf_gap[n] = (g1 < g0 ? g1 : g0) / W;
+        }
+    }
+    free(lq); free(lp); free(w);
     return 0;
 }

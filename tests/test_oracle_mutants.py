@@ -45,6 +45,14 @@ MUTANTS = [
      "long ystar = argmax_first(draft + n * V, V);", 1),
     ("distill_temperature_ignored", "log_softmax(target + n * V, V, tau, lp);",
      "log_softmax(target + n * V, V, 1.0, lp);", 1),
+    ("mixture_weights_swapped", "w[j] = beta * exp(lp[j]) + (1.0 - beta) * exp(lq[j]);",
+     "w[j] = (1.0 - beta) * exp(lp[j]) + beta * exp(lq[j]);", 1),
+    ("mixture_temperature_ignored", "log_softmax(draft + n * d_stride, V, tau, lq);",
+     "log_softmax(draft + n * d_stride, V, 1.0, lq);", 1),
+    ("mixture_cdf_not_strict", "if (C > target_mass) { pick = j; break; }",
+     "if (C >= target_mass) { pick = j; break; }", 1),
+    ("mixture_target_only", "w[j] = beta * exp(lp[j]) + (1.0 - beta) * exp(lq[j]);",
+     "w[j] = exp(lp[j]);", 1),
 ]
 
 
@@ -58,6 +66,7 @@ def test_mutant_is_caught(tmp_path, name, old, new, count):
     env = dict(os.environ, OSD_ORACLE_LIB=lib)
     r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
                         os.path.join(HERE, "test_oracle_distill.py"),
-                        os.path.join(HERE, "test_oracle_verify.py")],
+                        os.path.join(HERE, "test_oracle_verify.py"),
+                        os.path.join(HERE, "test_oracle_mixed.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode == 1, f"mutant {name} survived every pin:\n{r.stdout[-2000:]}"
