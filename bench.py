@@ -58,7 +58,8 @@ def _source_hash(files):
     return h.hexdigest()[:16]
 
 
-DISTILL_SOURCES = ["paper_2310_07177_gb300/csrc/osd_distill.cu", "paper_2310_07177_gb300/csrc/osd_device.cuh"]
+DISTILL_SOURCES = ["paper_2310_07177_gb300/csrc/osd_distill.cu", "paper_2310_07177_gb300/csrc/osd_device.cuh",
+                   "paper_2310_07177_gb300/csrc/osd_rowspan.cuh"]
 VERIFY_SOURCES = ["paper_2310_07177_gb300/csrc/osd_verify.cu", "paper_2310_07177_gb300/csrc/osd_device.cuh"]
 
 
@@ -314,6 +315,8 @@ def run_ours(args):
         kernels["verify_greedy"] = {"us_per_call": avg_g * 1e3, "alg_bytes": bytes_g,
                                     "gbs": bytes_g / (avg_g / 1e3) / 1e9,
                                     "positions_per_s": sv.B * sv.k / (avg_g / 1e3)}
+    if wl == "serving-32k" and not args.no_extras:
+        kernels["mixed_sample"] = _time_mixed_sample(osd, d, sd, l2_flush, stream, reps=max(3, args.steps // 2))
     for kv in kernels.values():
         kv["frac_of_peak"] = kv["gbs"] / peak
     # the dominant kernel: distill on the default step, verify's row statistics at 128k
@@ -351,6 +354,32 @@ def run_ours(args):
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
+
+
+def _time_mixed_sample(osd, d, sd, l2_flush, stream, reps):
+    """Mixed sampling (y ~ beta p + (1 - beta) q) over the distill workload's rows,
+    timed on its own after the step loop (it is not part of the serving step)."""
+    import torch
+    g = torch.Generator(device=d["draft"].device)
+    g.manual_seed(2310071779)
+    u = torch.rand(sd.N, generator=g, device=d["draft"].device)
+    tok = torch.empty(sd.N, dtype=torch.int32, device=d["draft"].device)
+    for _ in range(2):
+        osd.osd_mixed_sample(d["draft"], d["target"], u, 0.5, tokens=tok)
+    ms = []
+    for _ in range(reps):
+        l2_flush.zero_()
+        torch.cuda._sleep(SLEEP_CYCLES)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        osd.osd_mixed_sample(d["draft"], d["target"], u, 0.5, tokens=tok)
+        b.record(stream)
+        b.synchronize()
+        ms.append(a.elapsed_time(b))
+    avg = statistics.mean(ms)
+    alg = sd.N * sd.V * 2 * 2 + sd.N * 8  # both bf16 rows, the uniform and the token
+    return {"us_per_call": avg * 1e3, "alg_bytes": alg, "gbs": alg / (avg / 1e3) / 1e9,
+            "positions_per_s": sd.N / (avg / 1e3), "in_step": False, "beta": 0.5}
 
 
 def run_e2e(args, osd, setup, dev, stream, positions, wl):
@@ -529,6 +558,8 @@ def main():
     ap.add_argument("--cpu-rows", type=int, default=4096, help="distill rows per loss kind in the oracle sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
+    ap.add_argument("--no-extras", action="store_true",
+                    help="skip the kernels timed outside the step (mixed sampling)")
     ap.add_argument("--distill-rows", type=int, default=None,
                     help="override the distill buffer size N (small cases for profiling)")
     args = ap.parse_args()

@@ -16,6 +16,8 @@
  *                logits (the analytic update step of Algorithm 1).
  *   osd_distill_accepted  the same on the rows osd_verify rejected, selected
  *                and compacted on the device from its accepted counts.
+ *   osd_mixed_sample  one token per position from beta p + (1 - beta) q
+ *                (Section 4.1, mixed sampling).
  *
  * Conventions shared by every entry point:
  *   - All array arguments are DEVICE pointers to caller-owned memory on the
@@ -74,7 +76,7 @@ const char *osd_status_string(osd_status status);
 
 /* ABI version of this library: (major << 16) | minor.  2.0 added the
  * temperature argument of osd_distill and the OSD_CE loss; 2.1 added
- * osd_distill_accepted. */
+ * osd_distill_accepted; 2.2 added osd_mixed_sample. */
 int osd_abi_version(void);
 
 /*
@@ -222,6 +224,36 @@ osd_status osd_distill_accepted(const void *draft_logits, const void *target_log
                                 osd_loss kind, float beta, float temperature,
                                 float *loss, float *dlogits, int32_t *seq_of_row, int32_t *count,
                                 int32_t *status, void *stream);
+
+/*
+ * Mixed-token sampling (Section 4.1): one token per position from the mixture
+ * beta p + (1 - beta) q, p = softmax(target row / tau), q = softmax(draft row
+ * / tau), the sampling the paper borrows to pick the tokens y the distillation
+ * loss is evaluated on.  The draw is one inverse-CDF step over the mixture
+ * weights w_j = beta p_j + (1 - beta) q_j in ascending vocabulary order:
+ * j* = min{ j : C_j > u W }, W = sum_j w_j, with the largest j with w_j > 0
+ * if rounding leaves none (the convention of osd_verify's extra token).
+ *
+ * draft_logits, target_logits  row n starts at base + n * stride elements
+ *                (stride 0 repeats one row); the V entries of a row are
+ *                contiguous; dtype as in osd_distill.
+ * uniforms       [N] fp32 in [0, 1), one per row.
+ * beta           in [0, 1]: 1 samples the target, 0 the draft.
+ * temperature    tau > 0 and finite.
+ * tokens         [N] int32 out.
+ * cdf_gap        [N] fp32 out, nullable: distance of u W to the nearest edge of
+ *                the chosen CDF step, divided by W (<= 0 when rounding left
+ *                no step above u W).
+ * status         nullable device int32: 0, or OSD_ERR_TIMEOUT if a bounded
+ *                wait for a bulk copy gave up (that row's token is then -1).
+ * Limits as osd_distill's: V <= 393216 (bf16) or 196608 (fp32).
+ * Argument errors: OSD_ERR_INVALID_ARG (null pointers with N > 0, negative
+ * sizes or strides, beta outside [0, 1], bad temperature, misalignment).
+ */
+osd_status osd_mixed_sample(const void *draft_logits, const void *target_logits, osd_dtype dtype,
+                            int N, int V, int64_t d_stride, int64_t t_stride,
+                            const float *uniforms, float beta, float temperature,
+                            int32_t *tokens, float *cdf_gap, int32_t *status, void *stream);
 
 #ifdef __cplusplus
 }

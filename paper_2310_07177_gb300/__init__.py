@@ -29,7 +29,8 @@ VERIFY_MAX_V = 1 << 21
 
 # every symbol include/osd.h declares
 EXPORTS = ("osd_status_string", "osd_abi_version", "osd_verify_workspace_size",
-           "osd_verify", "osd_verify_noalloc", "osd_distill", "osd_distill_accepted")
+           "osd_verify", "osd_verify_noalloc", "osd_distill", "osd_distill_accepted",
+           "osd_mixed_sample")
 
 
 class OsdError(RuntimeError):
@@ -68,6 +69,8 @@ def load_library():
     lib.osd_distill.argtypes = [vp, vp, i32, i32, i32, i32, i64, i64, i64, i64, vp, i32, f32, f32, vp, vp, vp, vp]
     lib.osd_distill_accepted.restype = i32
     lib.osd_distill_accepted.argtypes = [vp, vp, i32, i32, i32, i32, vp, i32, f32, f32, vp, vp, vp, vp, vp, vp]
+    lib.osd_mixed_sample.restype = i32
+    lib.osd_mixed_sample.argtypes = [vp, vp, i32, i32, i32, i64, i64, vp, f32, f32, vp, vp, vp, vp]
     _lib = lib
     return lib
 
@@ -284,3 +287,38 @@ def osd_distill_accepted(draft_logits: torch.Tensor, target_logits: torch.Tensor
     if st != OSD_OK:
         raise OsdError(st, "osd_distill_accepted")
     return out
+
+
+def _rows_2d(t: torch.Tensor):
+    """(N, V, row stride) of a 2-D view whose rows are contiguous (stride 0 repeats a row)."""
+    if t.dim() != 2 or (t.shape[1] > 1 and t.stride(1) != 1):
+        raise ValueError("logits must be a 2-D [N, V] view with contiguous rows")
+    return t.shape[0], t.shape[1], t.stride(0)
+
+
+def osd_mixed_sample(draft_logits: torch.Tensor, target_logits: torch.Tensor, uniforms: torch.Tensor,
+                     beta: float, *, temperature: float = 1.0, tokens: Optional[torch.Tensor] = None,
+                     cdf_gap: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
+                     stream: Optional[torch.cuda.Stream] = None):
+    """One token per row from beta p + (1 - beta) q (Section 4.1, mixed sampling).
+
+    ``draft_logits`` and ``target_logits`` are [N, V] views with contiguous rows
+    (``expand`` of one row is fine); ``uniforms`` [N] fp32 in [0, 1).  Returns
+    ``(tokens [N] int32, cdf_gap [N] fp32 or None)``.
+    """
+    lib = load_library()
+    dev = _need_cuda(draft_logits, target_logits, uniforms, tokens, cdf_gap, status)
+    N, V, ds = _rows_2d(draft_logits)
+    N2, V2, tsd = _rows_2d(target_logits)
+    if (N, V) != (N2, V2) or draft_logits.dtype != target_logits.dtype:
+        raise ValueError("draft and target logits must have the same shape and dtype")
+    if uniforms.dtype != torch.float32 or tuple(uniforms.shape) != (N,) or not uniforms.is_contiguous():
+        raise ValueError("uniforms must be contiguous float32 [N]")
+    if tokens is None:
+        tokens = torch.empty(N, dtype=torch.int32, device=dev)
+    st = lib.osd_mixed_sample(_ptr(draft_logits), _ptr(target_logits), _dtype_code(draft_logits), N, V, ds, tsd,
+                              _ptr(uniforms), float(beta), float(temperature), _ptr(tokens), _ptr(cdf_gap),
+                              _ptr(status), _stream(dev, stream))
+    if st != OSD_OK:
+        raise OsdError(st, "osd_mixed_sample")
+    return tokens, cdf_gap

@@ -228,6 +228,23 @@ __device__ __forceinline__ T block_reduce(T v, F f, T* scratch) {
     return r;
 }
 
+// fp64 sum and inclusive prefix sum across a warp (used where a sum decides a
+// sample position)
+__device__ __forceinline__ double warp_sum_f64(double v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ double warp_incl_scan_f64(double v) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const double y = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += y;
+    }
+    return v;
+}
+
 // ---------------------------------------------------------------- timers / errors
 __device__ __forceinline__ uint64_t global_ns() {
     uint64_t t;

@@ -26,14 +26,14 @@
 #include "osd.h"
 #include "osd_device.cuh"
 #include "osd_host.hpp"
+#include "osd_rowspan.cuh"
 
 namespace osd {
 
-constexpr int kDistThreads = 128;
+constexpr int kDistThreads = kRowThreads;
 constexpr int kDistMaxCluster = 8;
 constexpr int kDistSpanBytes = 32768;         // target bytes of both rows per CTA
 constexpr int kDistMaxSmem = 192 * 1024;      // largest staging buffer per CTA
-constexpr uint64_t kWaitLimitNs = 1000000000ull;
 
 struct DistParams {
     const void* draft;
@@ -73,83 +73,6 @@ struct Stats2 {
     float a, b, c;
 };
 
-template <typename In>
-__device__ __forceinline__ void copy_raw(In* dst, const In* src) {
-    using Raw = std::conditional_t<sizeof(In) == 2, unsigned short, unsigned int>;
-    *reinterpret_cast<Raw*>(dst) = __ldg(reinterpret_cast<const Raw*>(src));
-}
-
-// Visit this thread's entries of a staged span in chunks of one 16-byte vector
-// (or single entries on the element-wise path).  Clamping (to -1e30, see Elem)
-// happens on the packed words.  f(z[], t[], count_tag, j0, zmax, tmax, ninf)
-// gets the chunk maxima when kMax is set, and ninf = "the chunk holds a -inf"
-// when kMin is set.
-template <typename In, bool kAligned, bool kClampZ, bool kClampT, bool kMax, bool kMin = false, typename F>
-__device__ __forceinline__ void sweep(const In* zs, const In* ts, int n, F&& f) {
-    using E = Elem<In>;
-    constexpr int kVec = E::kVec;
-    const int tid = threadIdx.x;
-    if constexpr (kAligned) {
-        const int nv = n / kVec;
-        for (int v = tid; v < nv; v += kDistThreads) {
-            uint4 zr = lds_v4(zs + v * kVec), tr = lds_v4(ts + v * kVec);
-            if (kClampZ) E::clamp_raw(zr);
-            if (kClampT) E::clamp_raw(tr);
-            float z[kVec], t[kVec];
-            E::unpack(zr, z);
-            E::unpack(tr, t);
-            const float cz = kMax ? E::max_raw(zr) : 0.f, ct = kMax ? E::max_raw(tr) : 0.f;
-            const bool ninf = kMin ? (fminf(E::min_raw(zr), E::min_raw(tr)) == kNegInf) : false;
-            f(z, t, std::integral_constant<int, kVec>{}, v * kVec, cz, ct, ninf);
-        }
-        const int r0 = nv * kVec;
-        if (tid < n - r0) {
-            float z = E::lds(zs + r0 + tid), t = E::lds(ts + r0 + tid);
-            if (kClampZ) z = E::clamp1(z);
-            if (kClampT) t = E::clamp1(t);
-            f(&z, &t, std::integral_constant<int, 1>{}, r0 + tid, z, t, fminf(z, t) == kNegInf);
-        }
-    } else {
-        for (int e = tid; e < n; e += kDistThreads) {
-            float z = E::lds(zs + e), t = E::lds(ts + e);
-            if (kClampZ) z = E::clamp1(z);
-            if (kClampT) t = E::clamp1(t);
-            f(&z, &t, std::integral_constant<int, 1>{}, e, z, t, fminf(z, t) == kNegInf);
-        }
-    }
-}
-
-// Block-wide max of two values, then sum of three: the cheap way to merge
-// online softmax partials (every thread rescales its sums once to the block max).
-__device__ __forceinline__ float2 block_max2(float a, float b, float2* scratch) {
-    for (int o = 16; o > 0; o >>= 1) {
-        a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
-        b = fmaxf(b, __shfl_xor_sync(0xffffffffu, b, o));
-    }
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    __syncthreads();
-    if (lane == 0) scratch[warp] = make_float2(a, b);
-    __syncthreads();
-    float2 r = scratch[0];
-#pragma unroll
-    for (int w = 1; w < kDistThreads / 32; ++w) r = make_float2(fmaxf(r.x, scratch[w].x), fmaxf(r.y, scratch[w].y));
-    return r;
-}
-__device__ __forceinline__ float3 block_sum3(float a, float b, float c, float3* scratch) {
-    for (int o = 16; o > 0; o >>= 1) {
-        a += __shfl_xor_sync(0xffffffffu, a, o);
-        b += __shfl_xor_sync(0xffffffffu, b, o);
-        c += __shfl_xor_sync(0xffffffffu, c, o);
-    }
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    __syncthreads();
-    if (lane == 0) scratch[warp] = make_float3(a, b, c);
-    __syncthreads();
-    float3 r = scratch[0];
-#pragma unroll
-    for (int w = 1; w < kDistThreads / 32; ++w) r = make_float3(r.x + scratch[w].x, r.y + scratch[w].y, r.z + scratch[w].z);
-    return r;
-}
 // RKL: the draft maximum with the target logit at it (the larger one on ties),
 // merged in the same round as the target maximum.
 __device__ __forceinline__ bool pivot_wins(float m, float t, float m0, float t0) {
@@ -340,34 +263,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     In* ts = zs + p.span;
 
     // ---- stage the span of both rows in shared memory
-    if (tid == 0) s_err = 0;
-    if constexpr (kAligned) {
-        const uint32_t bytes = static_cast<uint32_t>(n * sizeof(In)) & ~15u;
-        const int nb = static_cast<int>(bytes / sizeof(In));
-        if (tid == 0 && bytes) mbar_init(&bar, 1);
-        __syncthreads();
-        if (tid == 0 && bytes) {
-            mbar_arrive_expect_tx(&bar, 2 * bytes);
-            bulk_g2s(zs, zrow + e0, bytes, &bar);
-            bulk_g2s(ts, trow + e0, bytes, &bar);
-        }
-        for (int e = nb + tid; e < n; e += kDistThreads) {
-            copy_raw(zs + e, zrow + e0 + e);
-            copy_raw(ts + e, trow + e0 + e);
-        }
-        if (bytes && !mbar_wait_bounded(&bar, 0, kWaitLimitNs)) {
-            atomicOr(&s_err, 1);
-            mbar_wait_bounded(&bar, 0, kWaitLimitNs);  // give copies in flight a last chance to land
-        }
-    } else {
-        __syncthreads();
-        for (int e = tid; e < n; e += kDistThreads) {
-            copy_raw(zs + e, zrow + e0 + e);
-            copy_raw(ts + e, trow + e0 + e);
-        }
-    }
-    __syncthreads();
-    const int err_local = s_err;
+    const int err_local = stage_span<In, kAligned>(zs, ts, zrow + e0, trow + e0, n, &bar, &s_err);
 
     // ---- pass 0: this thread's maxima, and the chunk where each first appears
     float mz = kNegInf, mt = kNegInf;
@@ -771,22 +667,6 @@ static cudaError_t launch_distill_dtype(osd_loss kind, const DistParams& dp, lon
     }
 }
 
-// Split V over a cluster: about kDistSpanBytes of staged logits per CTA, at
-// most kDistMaxCluster CTAs, spans a multiple of 64 entries.
-static bool distill_shape(int V, size_t es, int* csize, int* span) {
-    const int base = static_cast<int>(kDistSpanBytes / (2 * es));
-    int c = (V + base - 1) / base;
-    if (c > kDistMaxCluster) c = kDistMaxCluster;
-    if (c < 1) c = 1;
-    int s = (V + c - 1) / c;
-    s = (s + 63) / 64 * 64;
-    c = (V + s - 1) / s;
-    if (2 * size_t(s) * es > size_t(kDistMaxSmem)) return false;
-    *csize = c;
-    *span = s;
-    return true;
-}
-
 // Shared by both entry points: argument checks, shape, and the launch.
 static osd_status distill_run(const void* draft_logits, const void* target_logits, osd_dtype dtype, int G,
                               int P, int V, int64_t d_stride_g, int64_t d_stride_p, int64_t t_stride_g,
@@ -801,7 +681,8 @@ static osd_status distill_run(const void* draft_logits, const void* target_logit
     if (kind == OSD_JSD && !(beta >= 0.f && beta <= 1.f)) return OSD_ERR_INVALID_ARG;
     const size_t es = dtype_size(dtype);
     int csize = 1, span = V;
-    if (!distill_shape(V, es, &csize, &span)) return OSD_ERR_UNSUPPORTED;
+    if (!row_span_shape(V, es, kDistSpanBytes, kDistMaxCluster, kDistMaxSmem, &csize, &span))
+        return OSD_ERR_UNSUPPORTED;
     const long long rows = static_cast<long long>(G) * P;
     if (rows * csize > INT_MAX) return OSD_ERR_UNSUPPORTED;
     cudaStream_t s = static_cast<cudaStream_t>(stream);

@@ -60,21 +60,6 @@ template <typename In> struct NegInfRaw;
 template <> struct NegInfRaw<float> { static constexpr uint32_t bits = 0xFF800000u; };
 template <> struct NegInfRaw<__nv_bfloat16> { static constexpr uint32_t bits = 0xFF80FF80u; };
 
-__device__ __forceinline__ double warp_sum_f64(double v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    return v;
-}
-__device__ __forceinline__ double warp_incl_scan_f64(double v) {
-    const int lane = threadIdx.x & 31;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const double y = __shfl_up_sync(0xffffffffu, v, o);
-        if (lane >= o) v += y;
-    }
-    return v;
-}
-
 template <typename In> __device__ __forceinline__ uint4 ninf_raw() {
     return make_uint4(NegInfRaw<In>::bits, NegInfRaw<In>::bits, NegInfRaw<In>::bits, NegInfRaw<In>::bits);
 }

@@ -95,6 +95,14 @@ def test_argument_errors_return_before_any_launch(lib):
               None) == osd.OSD_ERR_UNSUPPORTED
     assert fa(None, None, 1, 0, 2, 16, None, 0, 0.5, 1.0, None, None, None, None, None,
               None) == osd.OSD_OK
+    # mixed sampling: beta outside [0, 1], bad temperature, null uniforms, V beyond the limit
+    fm = lib.osd_mixed_sample
+    assert fm(fake, fake, 1, 2, 16, 16, 16, fake, 1.5, 1.0, fake, None, None, None) == osd.OSD_ERR_INVALID_ARG
+    assert fm(fake, fake, 1, 2, 16, 16, 16, fake, 0.5, 0.0, fake, None, None, None) == osd.OSD_ERR_INVALID_ARG
+    assert fm(fake, fake, 1, 2, 16, 16, 16, None, 0.5, 1.0, fake, None, None, None) == osd.OSD_ERR_INVALID_ARG
+    assert fm(fake, fake, 1, 2, 16, -16, 16, fake, 0.5, 1.0, fake, None, None, None) == osd.OSD_ERR_INVALID_ARG
+    assert fm(fake, fake, 1, 2, 500000, 0, 0, fake, 0.5, 1.0, fake, None, None, None) == osd.OSD_ERR_UNSUPPORTED
+    assert fm(None, None, 1, 0, 16, 16, 16, None, 0.5, 1.0, None, None, None, None) == osd.OSD_OK
 
 
 def test_product_path_fails_loudly_without_library(tmp_path, monkeypatch):
