@@ -71,6 +71,9 @@ def _load():
                                            ctypes.c_double, ctypes.c_double, dp, dp]
         lib.osd_oracle_log_softmax.restype = None
         lib.osd_oracle_log_softmax.argtypes = [dp, L, ctypes.c_double, dp]
+        lib.osd_oracle_verify_tree.restype = ctypes.c_int
+        lib.osd_oracle_verify_tree.argtypes = [dp, dp, L, L, L, i32p, i32p, dp, ctypes.c_double,
+                                               i32p, i32p, i32p, i32p, dp, dp]
         lib.osd_oracle_mixed_sample.restype = ctypes.c_int
         lib.osd_oracle_mixed_sample.argtypes = [dp, dp, L, L, L, L, dp, ctypes.c_double, ctypes.c_double,
                                                 i32p, dp]
@@ -232,3 +235,38 @@ def mixed_sample(draft_logits, target_logits, uniforms, beta, temperature=1.0):
     if rc != 0:
         raise ValueError("osd_oracle_mixed_sample rejected its arguments")
     return tok, gap
+
+
+def verify_tree(draft_logits, target_logits, parent, tokens, uniforms, temperature):
+    """Multi-candidate verification over a token tree (the tree-style decoding
+    of the paper's Medusa study), double precision.
+
+    draft_logits, target_logits [B, n_nodes, V]; parent [n_nodes] (parent[0] =
+    -1, parent[i] < i); tokens [B, n_nodes] (node 0 unused); uniforms
+    [B, n_nodes] (u[:, 0] drives the extra draw, u[:, i] tests node i).
+    Returns a dict with accepted [B], path [B, n_nodes], out_tokens
+    [B, n_nodes], last_node [B], margin [B, n_nodes], cdf_gap [B].
+    """
+    lib = _load()
+    z = _np(draft_logits, np.float64)
+    t = _np(target_logits, np.float64)
+    par = _np(parent, np.int32).reshape(-1)
+    y = _np(tokens, np.int32)
+    u = _np(uniforms, np.float64)
+    B, n, V = t.shape
+    assert z.shape == (B, n, V) and par.shape == (n,) and y.shape == (B, n) and u.shape == (B, n)
+    acc = np.empty(B, np.int32)
+    path = np.empty((B, n), np.int32)
+    out = np.empty((B, n), np.int32)
+    last = np.empty(B, np.int32)
+    margin = np.empty((B, n), np.float64)
+    gap = np.empty(B, np.float64)
+    rc = lib.osd_oracle_verify_tree(_ptr(z, ctypes.c_double), _ptr(t, ctypes.c_double), B, n, V,
+                                    _ptr(par, ctypes.c_int32), _ptr(y, ctypes.c_int32), _ptr(u, ctypes.c_double),
+                                    float(temperature), _ptr(acc, ctypes.c_int32), _ptr(path, ctypes.c_int32),
+                                    _ptr(out, ctypes.c_int32), _ptr(last, ctypes.c_int32),
+                                    _ptr(margin, ctypes.c_double), _ptr(gap, ctypes.c_double))
+    if rc != 0:
+        raise ValueError("osd_oracle_verify_tree rejected its arguments")
+    return {"accepted": acc, "path": path, "out_tokens": out, "last_node": last, "margin": margin,
+            "cdf_gap": gap}

@@ -11,6 +11,8 @@
  *                       variation distance, and the analytic gradient with
  *                       respect to the draft logits (Algorithm 1, "Update
  *                       q_theta ... analytically").
+ *   osd_oracle_verify_tree  multi-candidate verification over a token tree
+ *                       (the tree-style decoding of the paper's Medusa study).
  *   osd_oracle_mixed_sample  one draw per position from the mixture
  *                       beta p + (1 - beta) q_theta (Section 4.1, mixed
  *                       sampling of the tokens the distillation is run on).
@@ -341,5 +343,134 @@ int osd_oracle_mixed_sample(const double *draft, const double *target, long N, l
         }
     }
     free(lq); free(lp); free(w);
+    return 0;
+}
+
+/*
+ * Multi-candidate verification over a token tree: the tree-style speculative
+ * decoding the paper runs OSD on with Medusa, where several candidates are
+ * proposed per position.  Each node carries one candidate token; the children
+ * of a node are the alternatives for the next position, tried in increasing
+ * index order with the accept rule of Appendix A.1 applied to the current
+ * residual: child y is accepted iff u < r(y) / q(y), starting from r = p; a
+ * rejection replaces r by norm(max(0, r - q)) (multi-candidate speculative
+ * sampling, which keeps the output distributed as p).  Accepting a child moves
+ * the walk to it; when every child of the current node is rejected, or it has
+ * none, one more token is drawn from r by the inverse CDF of the verify
+ * oracle's extra token.  T = 0 is greedy: the first child equal to argmax p is
+ * taken, and the extra token is argmax p.
+ *
+ * parent [n_nodes]         parent[0] = -1, 0 <= parent[i] < i (static tree)
+ * draft  [B, n_nodes, V]   z at node i: the draft distribution q of node i's children
+ * target [B, n_nodes, V]   t at node i: the target distribution p after node i's path
+ * tokens [B, n_nodes]      candidate token of node i (node 0, the root, has none)
+ * uniforms [B, n_nodes]    u[b, i] tests node i; u[b, 0] drives the extra draw
+ * accepted [B]             accepted tokens (the depth reached); -1 if a token is
+ *                          outside [0, V)
+ * path [B, n_nodes]        the accepted nodes, root excluded, then -1
+ * out_tokens [B, n_nodes]  the accepted tokens, the extra token, then -1
+ * last_node [B]            the node where the walk stopped (-1 if bad)
+ * margin [B, n_nodes]      |u - r(y)/q(y)| of every test made; NaN elsewhere
+ * cdf_gap [B]              as in osd_oracle_verify; NaN at T = 0
+ * Returns 0, or -1 on bad arguments / allocation failure.
+ */
+int osd_oracle_verify_tree(const double *draft, const double *target, long B, long n_nodes, long V,
+                           const int32_t *parent, const int32_t *tokens, const double *uniforms,
+                           double T, int32_t *accepted, int32_t *path, int32_t *out_tokens,
+                           int32_t *last_node, double *margin, double *cdf_gap)
+{
+    if (B < 0 || n_nodes < 1 || V < 1 || !(T >= 0.0) || parent[0] != -1) return -1;
+    for (long i = 1; i < n_nodes; ++i)
+        if (parent[i] < 0 || parent[i] >= i) return -1;
+    double *lq = (double *)malloc(sizeof(double) * (size_t)V);
+    double *lp = (double *)malloc(sizeof(double) * (size_t)V);
+    double *q = (double *)malloc(sizeof(double) * (size_t)V);
+    double *r = (double *)malloc(sizeof(double) * (size_t)V);
+    if (!lq || !lp || !q || !r) { free(lq); free(lp); free(q); free(r); return -1; }
+
+    for (long b = 0; b < B; ++b) {
+        const int32_t *y = tokens + b * n_nodes;
+        const double *u = uniforms + b * n_nodes;
+        int32_t *pth = path + b * n_nodes;
+        int32_t *out = out_tokens + b * n_nodes;
+        for (long i = 0; i < n_nodes; ++i) {
+            pth[i] = -1;
+            out[i] = -1;
+            margin[b * n_nodes + i] = NAN;
+        }
+        cdf_gap[b] = NAN;
+        int bad = 0;
+        for (long i = 1; i < n_nodes; ++i)
+            if (y[i] < 0 || y[i] >= V) bad = 1;
+        if (bad) { accepted[b] = -1; last_node[b] = -1; continue; }
+
+        long node = 0, depth = 0, extra = -1;
+        for (;;) {
+            const double *trow = target + (b * n_nodes + node) * V;
+            long next = -1;
+            if (T == 0.0) {
+                long best = argmax_first(trow, V);
+                for (long c = node + 1; c < n_nodes && next < 0; ++c)
+                    if (parent[c] == node && y[c] == best) next = c;
+                if (next < 0) { extra = best; break; }
+            } else {
+                log_softmax(trow, V, T, lp);
+                log_softmax(draft + (b * n_nodes + node) * V, V, T, lq);
+                for (long j = 0; j < V; ++j) { r[j] = exp(lp[j]); q[j] = exp(lq[j]); }
+                for (long c = node + 1; c < n_nodes && next < 0; ++c) {
+                    if (parent[c] != node) continue;
+                    const double ry = r[y[c]], qy = q[y[c]];
+                    double ratio;
+                    if (qy > 0.0) ratio = ry / qy;
+                    else ratio = (ry > 0.0) ? INFINITY : 0.0;
+                    margin[b * n_nodes + c] = fabs(u[c] - ratio);
+                    if (u[c] < ratio) {
+                        next = c;
+                    } else {                          /* r <- norm(max(0, r - q)) */
+                        double W = 0.0;
+                        for (long j = 0; j < V; ++j) {
+                            const double d = r[j] - q[j];
+                            r[j] = d > 0.0 ? d : 0.0;
+                            W += r[j];
+                        }
+                        if (W > 0.0)
+                            for (long j = 0; j < V; ++j) r[j] /= W;
+                    }
+                }
+                if (next < 0) {                       /* the extra token from r */
+                    double W = 0.0;
+                    for (long j = 0; j < V; ++j) W += r[j];
+                    if (W > 0.0) {
+                        const double mass = u[0] * W;
+                        double C = 0.0, Cprev = 0.0;
+                        for (long j = 0; j < V; ++j) {
+                            Cprev = C;
+                            C += r[j];
+                            if (C > mass) { extra = j; break; }
+                        }
+                        if (extra < 0) {
+                            for (long j = V - 1; j >= 0; --j)
+                                if (r[j] > 0.0) { extra = j; break; }
+                            Cprev = W - r[extra];
+                            C = W;
+                        }
+                        const double g1 = C - mass, g0 = mass - Cprev;
+                        cdf_gap[b] = (g1 < g0 ? g1 : g0) / W;
+                    } else {
+                        extra = argmax_first(lp, V);
+                    }
+                    break;
+                }
+            }
+            pth[depth] = (int32_t)next;
+            out[depth] = y[next];
+            ++depth;
+            node = next;
+        }
+        out[depth] = (int32_t)extra;
+        accepted[b] = (int32_t)depth;
+        last_node[b] = (int32_t)node;
+    }
+    free(lq); free(lp); free(q); free(r);
     return 0;
 }

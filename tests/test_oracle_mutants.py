@@ -53,6 +53,12 @@ MUTANTS = [
      "if (C >= target_mass) { pick = j; break; }", 1),
     ("mixture_target_only", "w[j] = beta * exp(lp[j]) + (1.0 - beta) * exp(lq[j]);",
      "w[j] = exp(lp[j]);", 1),
+    ("tree_residual_not_updated", "const double d = r[j] - q[j];", "const double d = r[j];", 1),
+    ("tree_siblings_reversed",
+     "for (long c = node + 1; c < n_nodes && next < 0; ++c) {\n                    if (parent[c] != node) continue;",
+     "for (long c = n_nodes - 1; c > node && next < 0; --c) {\n                    if (parent[c] != node) continue;", 1),
+    ("tree_extra_uses_node_uniform", "const double mass = u[0] * W;", "const double mass = u[node] * W;", 1),
+    ("tree_ratio_inverted", "if (qy > 0.0) ratio = ry / qy;", "if (ry > 0.0) ratio = qy / ry;", 1),
 ]
 
 
@@ -67,6 +73,7 @@ def test_mutant_is_caught(tmp_path, name, old, new, count):
     r = subprocess.run([sys.executable, "-m", "pytest", "-x", "-q", "-p", "no:cacheprovider",
                         os.path.join(HERE, "test_oracle_distill.py"),
                         os.path.join(HERE, "test_oracle_verify.py"),
-                        os.path.join(HERE, "test_oracle_mixed.py")],
+                        os.path.join(HERE, "test_oracle_mixed.py"),
+                        os.path.join(HERE, "test_oracle_tree.py")],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
     assert r.returncode == 1, f"mutant {name} survived every pin:\n{r.stdout[-2000:]}"
