@@ -60,7 +60,8 @@ def _source_hash(files):
 
 DISTILL_SOURCES = ["paper_2310_07177_gb300/csrc/osd_distill.cu", "paper_2310_07177_gb300/csrc/osd_device.cuh",
                    "paper_2310_07177_gb300/csrc/osd_rowspan.cuh"]
-VERIFY_SOURCES = ["paper_2310_07177_gb300/csrc/osd_verify.cu", "paper_2310_07177_gb300/csrc/osd_device.cuh"]
+VERIFY_SOURCES = ["paper_2310_07177_gb300/csrc/osd_verify.cu", "paper_2310_07177_gb300/csrc/osd_device.cuh",
+                  "paper_2310_07177_gb300/csrc/osd_rowstats.cuh"]
 
 
 def _traffic(kernel: str, files):
@@ -317,6 +318,7 @@ def run_ours(args):
                                     "positions_per_s": sv.B * sv.k / (avg_g / 1e3)}
     if wl == "serving-32k" and not args.no_extras:
         kernels["mixed_sample"] = _time_mixed_sample(osd, d, sd, l2_flush, stream, reps=max(3, args.steps // 2))
+        kernels["tree_verify"] = _time_tree_verify(osd, dev, l2_flush, stream, reps=max(3, args.steps // 2))
     for kv in kernels.values():
         kv["frac_of_peak"] = kv["gbs"] / peak
     # the dominant kernel: distill on the default step, verify's row statistics at 128k
@@ -380,6 +382,37 @@ def _time_mixed_sample(osd, d, sd, l2_flush, stream, reps):
     alg = sd.N * sd.V * 2 * 2 + sd.N * 8  # both bf16 rows, the uniform and the token
     return {"us_per_call": avg * 1e3, "alg_bytes": alg, "gbs": alg / (avg / 1e3) / 1e9,
             "positions_per_s": sd.N / (avg / 1e3), "in_step": False, "beta": 0.5}
+
+
+def _time_tree_verify(osd, dev, l2_flush, stream, reps):
+    """Token-tree verification of B=32 sequences over the 27-node Medusa-style
+    tree at V=32000 bf16, T=1, timed on its own after the step loop."""
+    import torch
+    from paper_2310_07177_gb300 import workloads as W
+    par = W.MEDUSA_TREE
+    B, V = 32, 32000
+    inp = W.tree_inputs(B, par, V, torch.bfloat16, 1.0, seed=2310071778, device=dev, target_noise=0.8)
+    n = len(par)
+    ws = torch.empty(osd.osd_verify_tree_workspace_size(B, n, V), dtype=torch.uint8, device=dev)
+    res = osd.osd_verify_tree(inp["draft"], inp["target"], par, inp["tokens"], inp["uniforms"], 1.0, workspace=ws)
+    ms = []
+    for i in range(reps + 2):
+        l2_flush.zero_()
+        torch.cuda._sleep(SLEEP_CYCLES)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        osd.osd_verify_tree(inp["draft"], inp["target"], par, inp["tokens"], inp["uniforms"], 1.0,
+                            workspace=ws, out=res)
+        b.record(stream)
+        b.synchronize()
+        if i >= 2:
+            ms.append(a.elapsed_time(b))
+    avg = statistics.mean(ms)
+    alg = 2 * B * n * V * 2  # every node's draft and target row, read once by the statistics pass
+    acc = res.accepted.float().mean().item()
+    return {"us_per_call": avg * 1e3, "alg_bytes": alg, "gbs": alg / (avg / 1e3) / 1e9,
+            "positions_per_s": B * (acc + 1) / (avg / 1e3), "mean_accepted": round(acc, 3),
+            "nodes": n, "in_step": False}
 
 
 def run_e2e(args, osd, setup, dev, stream, positions, wl):

@@ -18,6 +18,8 @@
  *                and compacted on the device from its accepted counts.
  *   osd_mixed_sample  one token per position from beta p + (1 - beta) q
  *                (Section 4.1, mixed sampling).
+ *   osd_verify_tree  verification of several candidates per position laid
+ *                out as a token tree (the paper's Medusa combination).
  *
  * Conventions shared by every entry point:
  *   - All array arguments are DEVICE pointers to caller-owned memory on the
@@ -76,7 +78,8 @@ const char *osd_status_string(osd_status status);
 
 /* ABI version of this library: (major << 16) | minor.  2.0 added the
  * temperature argument of osd_distill and the OSD_CE loss; 2.1 added
- * osd_distill_accepted; 2.2 added osd_mixed_sample. */
+ * osd_distill_accepted; 2.2 added osd_mixed_sample; 2.3 added
+ * osd_verify_tree. */
 int osd_abi_version(void);
 
 /*
@@ -224,6 +227,64 @@ osd_status osd_distill_accepted(const void *draft_logits, const void *target_log
                                 osd_loss kind, float beta, float temperature,
                                 float *loss, float *dlogits, int32_t *seq_of_row, int32_t *count,
                                 int32_t *status, void *stream);
+
+/* Largest token tree osd_verify_tree accepts (nodes, root included). */
+#define OSD_TREE_MAX_NODES 64
+
+/*
+ * Bytes of device workspace osd_verify_tree needs for B trees of n_nodes
+ * nodes over a vocabulary of V (per-row softmax statistics).  Errors as
+ * osd_verify_workspace_size; OSD_ERR_UNSUPPORTED beyond OSD_TREE_MAX_NODES.
+ */
+osd_status osd_verify_tree_workspace_size(int B, int n_nodes, int V, size_t *bytes);
+
+/*
+ * Multi-candidate verification over a token tree: the tree-style speculative
+ * decoding the paper combines OSD with (its Medusa study), where several
+ * candidates are proposed per position.  Node i > 0 carries one candidate
+ * token; its children are the alternatives for the next position.
+ *
+ * At the current node (the root first), with q = softmax(draft row / T) and
+ * p = softmax(target row / T) of that node, the children are tried in
+ * increasing index order: child y passes iff u < r(y) / q(y), with r the
+ * current residual, starting from r = p; a rejection replaces r by
+ * norm(max(0, r - q)) (multi-candidate speculative sampling, which keeps the
+ * output distributed as p); a pass moves the walk to that child.  When every
+ * child is rejected, or the node has none, one more token is drawn from r by
+ * the inverse CDF of osd_verify's extra token (u = uniforms[b, 0]).
+ * T == 0 is greedy: the first child equal to argmax p (lowest index) passes;
+ * otherwise the extra token is argmax p.
+ *
+ * draft_logits   [B, n_nodes, V] dtype, contiguous: row i is the draft
+ *                distribution the children of node i were proposed from
+ *                (not read at T == 0; leaves' rows are not read)
+ * target_logits  [B, n_nodes, V] dtype, contiguous: row i is the target
+ *                distribution after the path to node i
+ * parent         [n_nodes] int32 HOST array, the static tree shared by the
+ *                batch: parent[0] = -1, 0 <= parent[i] < i
+ * tokens         [B, n_nodes] int32: candidate of node i (entry 0 unused)
+ * uniforms       [B, n_nodes] fp32 in [0, 1): u[b, i] tests node i, u[b, 0]
+ *                drives the extra draw (not read at T == 0)
+ * accepted       [B] out: accepted tokens (the depth reached), -1 if a token
+ *                lies outside [0, V)
+ * path           [B, n_nodes] out: the accepted nodes, root excluded, then -1
+ * out_tokens     [B, n_nodes] out: the accepted tokens, the extra token, then -1
+ * last_node      [B] out: the node where the walk stopped (its rows are the
+ *                ones a distillation step keeps when it has children)
+ * diag_margin    [B, n_nodes] out, nullable: |u - r(y)/q(y)| of every test made
+ *                (at node i's entry), NaN elsewhere and when T == 0
+ * diag_cdf_gap   [B] out, nullable: as in osd_verify
+ * workspace      >= osd_verify_tree_workspace_size() bytes, 16-byte aligned
+ * Limits: 1 <= n_nodes <= OSD_TREE_MAX_NODES, 1 <= V <= OSD_VERIFY_MAX_V.
+ * Returns OSD_ERR_INVALID_ARG for a malformed tree or the argument errors of
+ * osd_verify.
+ */
+osd_status osd_verify_tree(const void *draft_logits, const void *target_logits, osd_dtype dtype,
+                           int B, int n_nodes, int V, const int32_t *parent,
+                           const int32_t *tokens, const float *uniforms, float temperature,
+                           int32_t *accepted, int32_t *path, int32_t *out_tokens,
+                           int32_t *last_node, float *diag_margin, float *diag_cdf_gap,
+                           void *workspace, size_t workspace_bytes, void *stream);
 
 /*
  * Mixed-token sampling (Section 4.1): one token per position from the mixture

@@ -30,7 +30,7 @@ VERIFY_MAX_V = 1 << 21
 # every symbol include/osd.h declares
 EXPORTS = ("osd_status_string", "osd_abi_version", "osd_verify_workspace_size",
            "osd_verify", "osd_verify_noalloc", "osd_distill", "osd_distill_accepted",
-           "osd_mixed_sample")
+           "osd_mixed_sample", "osd_verify_tree_workspace_size", "osd_verify_tree")
 
 
 class OsdError(RuntimeError):
@@ -69,6 +69,11 @@ def load_library():
     lib.osd_distill.argtypes = [vp, vp, i32, i32, i32, i32, i64, i64, i64, i64, vp, i32, f32, f32, vp, vp, vp, vp]
     lib.osd_distill_accepted.restype = i32
     lib.osd_distill_accepted.argtypes = [vp, vp, i32, i32, i32, i32, vp, i32, f32, f32, vp, vp, vp, vp, vp, vp]
+    lib.osd_verify_tree_workspace_size.restype = i32
+    lib.osd_verify_tree_workspace_size.argtypes = [i32, i32, i32, ctypes.POINTER(sz)]
+    lib.osd_verify_tree.restype = i32
+    lib.osd_verify_tree.argtypes = [vp, vp, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_int32), vp, vp, f32,
+                                    vp, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.osd_mixed_sample.restype = i32
     lib.osd_mixed_sample.argtypes = [vp, vp, i32, i32, i32, i64, i64, vp, f32, f32, vp, vp, vp, vp]
     _lib = lib
@@ -322,3 +327,64 @@ def osd_mixed_sample(draft_logits: torch.Tensor, target_logits: torch.Tensor, un
     if st != OSD_OK:
         raise OsdError(st, "osd_mixed_sample")
     return tokens, cdf_gap
+
+
+def osd_verify_tree_workspace_size(B: int, n_nodes: int, V: int) -> int:
+    n = ctypes.c_size_t(0)
+    st = load_library().osd_verify_tree_workspace_size(int(B), int(n_nodes), int(V), ctypes.byref(n))
+    if st != OSD_OK:
+        raise OsdError(st, "osd_verify_tree_workspace_size")
+    return n.value
+
+
+class TreeResult(NamedTuple):
+    accepted: torch.Tensor      # [B] int32
+    path: torch.Tensor          # [B, n_nodes] int32
+    out_tokens: torch.Tensor    # [B, n_nodes] int32
+    last_node: torch.Tensor     # [B] int32
+    diag_margin: Optional[torch.Tensor]   # [B, n_nodes] fp32
+    diag_cdf_gap: Optional[torch.Tensor]  # [B] fp32
+
+
+def osd_verify_tree(draft_logits: Optional[torch.Tensor], target_logits: torch.Tensor, parent, tokens: torch.Tensor,
+                    uniforms: Optional[torch.Tensor], temperature: float, *, diagnostics: bool = True,
+                    workspace: Optional[torch.Tensor] = None, out: Optional[TreeResult] = None,
+                    stream: Optional[torch.cuda.Stream] = None) -> TreeResult:
+    """Multi-candidate verification over a token tree (see include/osd.h).
+
+    ``draft_logits`` and ``target_logits`` are contiguous [B, n_nodes, V];
+    ``parent`` is the static tree (a host sequence of n_nodes ints, parent[0] =
+    -1); ``tokens`` [B, n_nodes] int32; ``uniforms`` [B, n_nodes] fp32.  At
+    temperature 0 the draft logits and uniforms may be None.
+    """
+    lib = load_library()
+    B, n, V = target_logits.shape
+    dev = _need_cuda(draft_logits, target_logits, tokens, uniforms, workspace, *(out or ()))
+    par = (ctypes.c_int32 * n)(*[int(x) for x in (parent.tolist() if hasattr(parent, "tolist") else parent)])
+    if len(par) != n:
+        raise ValueError("parent must have n_nodes entries")
+    if not target_logits.is_contiguous() or (draft_logits is not None and (
+            tuple(draft_logits.shape) != (B, n, V) or not draft_logits.is_contiguous()
+            or draft_logits.dtype != target_logits.dtype)):
+        raise ValueError("draft/target logits must be contiguous [B, n_nodes, V] of one dtype")
+    if tokens.dtype != torch.int32 or tuple(tokens.shape) != (B, n) or not tokens.is_contiguous():
+        raise ValueError("tokens must be contiguous int32 [B, n_nodes]")
+    if uniforms is not None and (uniforms.dtype != torch.float32 or tuple(uniforms.shape) != (B, n)
+                                 or not uniforms.is_contiguous()):
+        raise ValueError("uniforms must be contiguous float32 [B, n_nodes]")
+    if workspace is None:
+        workspace = torch.empty(max(osd_verify_tree_workspace_size(B, n, V), 16), dtype=torch.uint8, device=dev)
+    if out is None:
+        i32 = torch.int32
+        out = TreeResult(torch.empty(B, dtype=i32, device=dev), torch.empty(B, n, dtype=i32, device=dev),
+                         torch.empty(B, n, dtype=i32, device=dev), torch.empty(B, dtype=i32, device=dev),
+                         torch.empty(B, n, dtype=torch.float32, device=dev) if diagnostics else None,
+                         torch.empty(B, dtype=torch.float32, device=dev) if diagnostics else None)
+    st = lib.osd_verify_tree(_ptr(draft_logits), _ptr(target_logits), _dtype_code(target_logits), B, n, V, par,
+                             _ptr(tokens), _ptr(uniforms), float(temperature), _ptr(out.accepted), _ptr(out.path),
+                             _ptr(out.out_tokens), _ptr(out.last_node), _ptr(out.diag_margin),
+                             _ptr(out.diag_cdf_gap), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                             _stream(dev, stream))
+    if st != OSD_OK:
+        raise OsdError(st, "osd_verify_tree")
+    return out

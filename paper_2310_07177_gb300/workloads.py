@@ -151,3 +151,54 @@ def accepted_inputs(B: int, k: int, seed: int, p_bad: float = 0.05, p_all: float
     a[u < p_all + p_bad] = k
     a[u < p_bad] = -1
     return a
+
+
+def tree_from_branching(branching) -> list:
+    """Parent array of a static candidate tree in breadth-first order.  branching
+    is a nested list: branching[d][i] is the number of children of the i-th
+    node at depth d (nodes of a depth in order); e.g. [[3], [2, 1, 0]] is a
+    root with three candidates, the first with two continuations, the second
+    with one."""
+    parent = [-1]
+    level = [0]
+    for counts in branching:
+        nxt = []
+        for node, c in zip(level, counts):
+            for _ in range(c):
+                parent.append(node)
+                nxt.append(len(parent) - 1)
+        level = nxt
+    return parent
+
+
+# A Medusa-style static tree of 26 candidates (27 nodes with the root): 4
+# candidates for the next token, 3 / 2 / 1 / 1 continuations of them, and so on
+# down to depth 5.
+MEDUSA_TREE = tree_from_branching([[4], [3, 2, 1, 1], [2, 1, 1, 1, 1, 0, 1], [2, 1, 1, 0, 1, 0, 1],
+                                   [1, 1, 0, 0, 0, 0]])
+
+
+def tree_inputs(B: int, parent, V: int, dtype, temperature: float, seed: int, device="cpu",
+                draft_std: float = 2.0, target_scale: float = 1.0, target_noise: float = 1.0) -> dict:
+    """draft [B,n,V], target [B,n,V], tokens [B,n] int32 and uniforms [B,n] for
+    the tree `parent`: the children of node i are independent draws from
+    softmax(draft row i / T), as a multi-candidate proposer makes them (at
+    T = 0 the first child is the draft argmax, the others draws at T = 1)."""
+    n = len(parent)
+    g = _gen(seed, device)
+    z = _randn((B, n, V), g, device).mul_(draft_std)
+    t = (z * target_scale + _randn((B, n, V), g, device).mul_(target_noise)).to(dtype)
+    z = z.to(dtype)
+    T = temperature if temperature > 0 else 1.0
+    tokens = torch.zeros(B, n, dtype=torch.int32, device=device)
+    for i in range(1, n):
+        u = torch.rand(B, V, generator=g, device=device).clamp_(min=1e-12)
+        gum = -torch.log(-torch.log(u))
+        first = parent.index(parent[i]) == i
+        if temperature == 0 and first:
+            tokens[:, i] = torch.argmax(z[:, parent[i]].float(), dim=-1).to(torch.int32)
+        else:
+            tokens[:, i] = torch.argmax(z[:, parent[i]].float() / T + gum, dim=-1).to(torch.int32)
+    uniforms = torch.rand(B, n, generator=g, device=device, dtype=torch.float32)
+    return {"draft": z.contiguous(), "target": t.contiguous(), "tokens": tokens, "uniforms": uniforms,
+            "parent": list(parent), "temperature": temperature}

@@ -95,6 +95,26 @@ def test_argument_errors_return_before_any_launch(lib):
               None) == osd.OSD_ERR_UNSUPPORTED
     assert fa(None, None, 1, 0, 2, 16, None, 0, 0.5, 1.0, None, None, None, None, None,
               None) == osd.OSD_OK
+    # tree verification: malformed trees, too many nodes, workspace too small, empty batch
+    ft = lib.osd_verify_tree
+    P = ctypes.c_int32 * 3
+    good, loop, root_kid = P(-1, 0, 1), P(-1, 1, 0), P(0, 0, 1)
+    for par in (loop, root_kid):
+        assert ft(fake, fake, 1, 2, 3, 16, par, fake, fake, 1.0, fake, fake, fake, fake, None, None, fake,
+                  1 << 20, None) == osd.OSD_ERR_INVALID_ARG
+    assert ft(fake, fake, 1, 2, 3, 16, good, fake, fake, -1.0, fake, fake, fake, fake, None, None, fake,
+              1 << 20, None) == osd.OSD_ERR_INVALID_ARG
+    assert ft(fake, fake, 1, 2, 3, 16, good, fake, fake, 1.0, fake, fake, fake, fake, None, None, fake,
+              8, None) == osd.OSD_ERR_INVALID_ARG
+    P65 = ctypes.c_int32 * 65
+    big = P65(-1, *range(64))
+    assert ft(fake, fake, 1, 2, 65, 16, big, fake, fake, 1.0, fake, fake, fake, fake, None, None, fake,
+              1 << 20, None) == osd.OSD_ERR_UNSUPPORTED
+    assert ft(None, None, 1, 0, 3, 16, good, None, None, 1.0, None, None, None, None, None, None, None,
+              0, None) == osd.OSD_OK
+    n = ctypes.c_size_t(0)
+    assert lib.osd_verify_tree_workspace_size(32, 27, 32000, ctypes.byref(n)) == osd.OSD_OK
+    assert n.value >= 2 * 32 * 27 * 16 and n.value % 256 == 0
     # mixed sampling: beta outside [0, 1], bad temperature, null uniforms, V beyond the limit
     fm = lib.osd_mixed_sample
     assert fm(fake, fake, 1, 2, 16, 16, 16, fake, 1.5, 1.0, fake, None, None, None) == osd.OSD_ERR_INVALID_ARG
