@@ -97,9 +97,6 @@ __device__ __forceinline__ float3 block_max_pivot(float mz, float tp, float mt, 
     }
     return r;
 }
-__device__ __forceinline__ float rescale(float m, float mb, float c) {
-    return (m == kNegInf) ? 0.f : ex2((m - mb) * c);
-}
 // CE label: the target maximum with the lowest index, and the draft logit there.
 struct Label {
     float m;
@@ -164,6 +161,13 @@ __device__ __forceinline__ void tvd_gradient(const In* zs, const In* ts, int n, 
                                              float* orow) {
     const int tid = threadIdx.x;
     auto g_of = [gpos, gneg](float q) { return q * (__float_as_int(q) < 0 ? gneg : gpos); };
+    // the factor of q': gpos, or gneg where the sign bit is set (one shift and one
+    // three-input logic op), so that the products go two at a time
+    const uint32_t fpos = __float_as_uint(gpos), fdiff = fpos ^ __float_as_uint(gneg);
+    auto factor = [fpos, fdiff](float q) {
+        const uint32_t neg = static_cast<uint32_t>(__float_as_int(q) >> 31);
+        return __uint_as_float(fpos ^ (neg & fdiff));
+    };
     if constexpr (kAligned) {
         constexpr int kVec = Elem<In>::kVec;
         const int nv = n / kVec;
@@ -181,9 +185,15 @@ __device__ __forceinline__ void tvd_gradient(const In* zs, const In* ts, int n, 
                     q[2 * i + 1] = __uint_as_float(prmt(tw[i], zw[i], 0x7632));
                 }
             }
+            float g[kVec];
 #pragma unroll
-            for (int e = 0; e < kVec; e += 4)
-                stg_v4(orow + v * kVec + e, g_of(q[e]), g_of(q[e + 1]), g_of(q[e + 2]), g_of(q[e + 3]));
+            for (int e = 0; e < kVec; e += 2) {
+                const float2 r = mul2(make_float2(q[e], q[e + 1]), make_float2(factor(q[e]), factor(q[e + 1])));
+                g[e] = r.x;
+                g[e + 1] = r.y;
+            }
+#pragma unroll
+            for (int e = 0; e < kVec; e += 4) stg_v4(orow + v * kVec + e, g[e], g[e + 1], g[e + 2], g[e + 3]);
         }
         const int r0 = nv * kVec;
         if (tid < n - r0) orow[r0 + tid] = g_of(load_q(zs, ts, r0 + tid));
@@ -203,6 +213,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     constexpr bool kClampZ = kClamp, kClampT = kClamp;
     constexpr bool kMoment = kKind == OSD_FKL || kKind == OSD_RKL;
     constexpr bool kNeedEt = kKind != OSD_CE;  // CE needs only the draft normaliser and the label
+    constexpr bool kFold = !kClamp;            // exponent arguments by one FMA (see pass 1)
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ __align__(8) uint64_t bar;
     __shared__ Stats1 s1_mine, s1_all;
@@ -306,7 +317,8 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         tpv = r.y;
         gtb = r.z;
     } else {
-        const float2 bm = block_max2(mz, mt, red_m);
+        // red_m has no readers yet: staging ended on a block barrier
+        const float2 bm = block_max2<false>(mz, mt, red_m);
         gzb = bm.x;
         gtb = bm.y;
         if constexpr (kKind == OSD_CE)
@@ -324,8 +336,16 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     float2 Ez2 = f2(0.f), Et2 = f2(0.f), X2 = f2(0.f);
     const bool zok = kClampZ || gzb != kNegInf;
     const bool tok = kNeedEt && (kClampT || gtb != kNegInf);
+    // Exponent arguments.  Unclamped kinds take (x - m) c as one FMA, x c - M with
+    // M = rn(m c): the rounding of M is a factor common to the whole row, so it
+    // cancels in the normalisation, and the row constants below add back its
+    // exact value fma(m, c, -M).  JSD keeps the exact difference, because its
+    // -1e30 clamp would make x c - M cancel catastrophically on an all-clamped span.
+    // A span with no mass gets M = 0: its logits are all -inf and so are x c - M.
+    const float Mz = zok ? __fmul_rn(gzb, c) : 0.f, Mt = tok ? __fmul_rn(gtb, c) : 0.f;
     if (!err_local) {
         const float2 gz2 = f2(gzb), gt2 = f2(gtb), tp2 = f2(tpv);
+        const float2 nMz2 = f2(-Mz), nMt2 = f2(-Mt);
         sweep<In, kAligned, kClampZ, kClampT, false, kMoment>(zs, ts, n, [&](const float* z, const float* t,
                                                                              auto tag, int, float, float,
                                                                              bool ninf) {
@@ -335,7 +355,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
 #pragma unroll
                 for (int e = 0; e < kCnt; ++e) {
                     if (zok) {
-                        const float ez = ex2((z[e] - gzb) * c);
+                        const float ez = kFold ? ex2(fmaf(z[e], c, -Mz)) : ex2((z[e] - gzb) * c);
                         Ez2.x += ez;
                         if (kKind == OSD_RKL && z[e] != kNegInf) {
                             if (t[e] == kNegInf) rkl_inf = true;  // q > 0 = p: the loss is +inf
@@ -343,39 +363,44 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                         }
                     }
                     if (tok) {
-                        const float et = ex2((t[e] - gtb) * c);
+                        const float et = kFold ? ex2(fmaf(t[e], c, -Mt)) : ex2((t[e] - gtb) * c);
                         Et2.x += et;
                         if (kKind == OSD_FKL && et > 0.f) X2.x = fmaf(et, t[e] - z[e], X2.x);
                     }
                 }
             } else {
-                if (zok) {
+                // no -inf in the chunk, and (unclamped) every span with finite logits has
+                // zok / tok set, so the sums need no per-chunk condition
 #pragma unroll
-                    for (int e = 0; e < kCnt; e += 2) {
-                        const float2 zd = sub2(make_float2(z[e], z[e + 1]), gz2);
-                        const float2 a = mul2(zd, f2(c));
-                        const float2 ez = make_float2(ex2(a.x), ex2(a.y));
-                        Ez2 = add2(Ez2, ez);
-                        if (kKind == OSD_RKL)
-                            X2 = fma2(ez, sub2(zd, sub2(make_float2(t[e], t[e + 1]), tp2)), X2);
-                    }
+                for (int e = 0; e < kCnt; e += 2) {
+                    const float2 zz = make_float2(z[e], z[e + 1]);
+                    float2 a;
+                    if constexpr (kFold) a = fma2(zz, f2(c), nMz2);
+                    else a = mul2(sub2(zz, gz2), f2(c));
+                    const float2 ez = make_float2(ex2(a.x), ex2(a.y));
+                    Ez2 = add2(Ez2, ez);
+                    if (kKind == OSD_RKL)
+                        X2 = fma2(ez, sub2(sub2(zz, gz2), sub2(make_float2(t[e], t[e + 1]), tp2)), X2);
                 }
-                if (tok) {
+                if constexpr (kNeedEt) {
 #pragma unroll
                     for (int e = 0; e < kCnt; e += 2) {
-                        const float2 a = mul2(sub2(make_float2(t[e], t[e + 1]), gt2), f2(c));
+                        const float2 tt = make_float2(t[e], t[e + 1]);
+                        float2 a;
+                        if constexpr (kFold) a = fma2(tt, f2(c), nMt2);
+                        else a = mul2(sub2(tt, gt2), f2(c));
                         const float2 et = make_float2(ex2(a.x), ex2(a.y));
                         Et2 = add2(Et2, et);
-                        if (kKind == OSD_FKL)
-                            X2 = fma2(et, sub2(make_float2(t[e], t[e + 1]), make_float2(z[e], z[e + 1])), X2);
+                        if (kKind == OSD_FKL) X2 = fma2(et, sub2(tt, make_float2(z[e], z[e + 1])), X2);
                     }
                 }
             }
         });
     }
     {
-        const float3 bs = block_sum3(Ez2.x + Ez2.y, Et2.x + Et2.y, X2.x + X2.y, red_s);
-        const int any_ninf = __syncthreads_or(row_ninf ? 1 : 0);
+        // red_s was last read by RKL's pivot merge; the other kinds have not used it yet
+        const float3 bs = block_sum3<kKind == OSD_RKL>(Ez2.x + Ez2.y, Et2.x + Et2.y, X2.x + X2.y, red_s);
+        const int any_ninf = kMoment ? __syncthreads_or(row_ninf ? 1 : 0) : 0;
         const int any_inf = (kKind == OSD_RKL) ? __syncthreads_or(rkl_inf ? 1 : 0) : 0;
         if (tid == 0)
             s1_mine = Stats1{gzb, bs.x, (kKind == OSD_CE) ? bl.m : gtb, bs.y, bs.z,
@@ -417,7 +442,12 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
             gt = fmaxf(gt, __shfl_xor_sync(0xffffffffu, gt, off));
             err |= __shfl_xor_sync(0xffffffffu, err, off);
         }
-        const float sz = rescale(o.mz, gz, c), st = rescale(o.mt, gt, c);
+        // each CTA's sums are against 2^(M_cta) (folded kinds) or 2^(m_cta c): bring them to the row's
+        auto to_row = [c](float m, float g) {
+            if (m == kNegInf) return 0.f;
+            return kFold ? ex2(__fmul_rn(m, c) - __fmul_rn(g, c)) : ex2((m - g) * c);
+        };
+        const float sz = to_row(o.mz, gz), st = to_row(o.mt, gt);
         float tg = 0.f;  // RKL: the row's pivot target logit
         if constexpr (kKind == OSD_RKL) {
             tg = (o.mz == gz && o.mz != kNegInf) ? o.zy : kNegInf;
@@ -438,16 +468,22 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
             s1_all = Stats1{gz, Ez, gt, Et, X, err, L.i, L.z};
             // row constants, computed once: log2 p = (t - m_t) c - log2(E_t) with
             // c = log2(e)/tau; the difference is exact, so the rounding never scales
-            // with the size of the logits
-            s_cu = -log2f(Et);
-            s_cv = -log2f(Ez);
-            const float lr = logf(Ez / Et);
+            // with the size of the logits.  Folded sums are against 2^M, M = rn(m c):
+            // E' = E 2^dm with dm = m c - M, taken exactly by an FMA
+            float dz = 0.f, dt = 0.f;
+            if (kFold) {
+                if (gz != kNegInf) dz = fmaf(gz, c, -__fmul_rn(gz, c));
+                if (gt != kNegInf) dt = fmaf(gt, c, -__fmul_rn(gt, c));
+            }
+            s_cu = -log2f(Et) + dt;
+            s_cv = -log2f(Ez) + dz;
+            const float lr = logf(Ez / Et) - kLn2 * (dz - dt);
             float l = 0.f;
             if (kKind == OSD_FKL) l = (X / Et - (gt - gz)) * inv_tau + lr;
             // RKL about the pivot: loss = log q - log p at the pivot + sum_j q_j D_j, with
             // D_j = ((z_j - m_z) - (t_j - t_pv)) / tau; s_K keeps the sum for pass 3
             if (kKind == OSD_RKL) l = (err & 4) ? __builtin_huge_valf() : (X / Ez + (gt - tg)) * inv_tau - lr;
-            if (kKind == OSD_CE) l = (gz - L.z) * inv_tau + logf(Ez);  // -log q(y*)
+            if (kKind == OSD_CE) l = (gz - L.z) * inv_tau + (logf(Ez) - kLn2 * dz);  // -log q(y*)
             s_loss = l;
             s_K = X / Ez * inv_tau;
             s_tp = tg;
@@ -479,18 +515,18 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                     const bool two = (e + 1 < kCnt);
                     const float2 u = log2p(make_float2(t[e], two ? t[e + 1] : t[e]));  // log2 p
                     const float2 v = log2q(make_float2(z[e], two ? z[e + 1] : z[e]));  // log2 q
-                    const float2 d = sub2(v, u);
                     float2 a, b, c2 = f2(0.f);
                     if (kKind == OSD_TVD) {
                         const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
-                        const float2 df = sub2(pj, qj);
+                        const float2 df = sub2(qj, pj);
                         a = make_float2(fabsf(df.x), fabsf(df.y));
-                        const float2 qq = make_float2(copysignf(qj.x, d.x), copysignf(qj.y, d.y));  // q sign(q - p)
+                        const float2 qq = make_float2(copysignf(qj.x, df.x), copysignf(qj.y, df.y));  // q sign(q - p)
                         qs[e] = qq.x;
                         if (e + 1 < kCnt) qs[e + 1] = qq.y;
                         b = add2(qj, qq);   // 2q where q >= p, else 0 (exact): into 2 Q+
                         c2 = sub2(qj, qq);  // 2q where q < p, else 0: into 2 Q-
                     } else {
+                        const float2 d = sub2(v, u);
                         float r[2][2];
                         const float uu[2] = {u.x, u.y}, vv[2] = {v.x, v.y}, dd[2] = {d.x, d.y};
 #pragma unroll
@@ -518,7 +554,8 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                 if constexpr (kKind == OSD_TVD) store_q<In, kCnt>(zs, ts, j0, qs);
             });
         }
-        const float3 bs = block_sum3(A2.x + A2.y, B2.x + B2.y, C2.x + C2.y, red_s);
+        // red_s was last read before the cluster merge's barriers
+        const float3 bs = block_sum3<false>(A2.x + A2.y, B2.x + B2.y, C2.x + C2.y, red_s);
         if (tid == 0) s2_mine = Stats2{bs.x, bs.y, bs.z};
         if (csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
         if (tid < 32) {

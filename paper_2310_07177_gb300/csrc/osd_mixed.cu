@@ -93,7 +93,7 @@ __global__ void __launch_bounds__(kRowThreads) mixed_sample_kernel(MixParams p) 
             mt = fmaxf(mt, ct);
         });
     }
-    const float2 bm = block_max2(mz, mt, red_m);
+    const float2 bm = block_max2<false>(mz, mt, red_m);  // red_m has no readers yet
     const float gzb = bm.x, gtb = bm.y;
     const bool zok = gzb != kNegInf, tok = gtb != kNegInf;  // a span of -inf has no mass
 

@@ -103,13 +103,17 @@ __device__ __forceinline__ void sweep(const In* zs, const In* ts, int n, F&& f) 
 
 // Block-wide max of two values, then sum of three: the cheap way to merge
 // softmax partials (every thread rescales its sums once to the block max).
+// kGuard adds the barrier that keeps a previous reduction's readers of
+// `scratch` ahead of the new writes; callers whose scratch has no readers
+// since the last block barrier leave it out.
+template <bool kGuard = true>
 __device__ __forceinline__ float2 block_max2(float a, float b, float2* scratch) {
     for (int o = 16; o > 0; o >>= 1) {
         a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
         b = fmaxf(b, __shfl_xor_sync(0xffffffffu, b, o));
     }
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    __syncthreads();
+    if (kGuard) __syncthreads();
     if (lane == 0) scratch[warp] = make_float2(a, b);
     __syncthreads();
     float2 r = scratch[0];
@@ -117,6 +121,7 @@ __device__ __forceinline__ float2 block_max2(float a, float b, float2* scratch) 
     for (int w = 1; w < kRowWarps; ++w) r = make_float2(fmaxf(r.x, scratch[w].x), fmaxf(r.y, scratch[w].y));
     return r;
 }
+template <bool kGuard = true>
 __device__ __forceinline__ float3 block_sum3(float a, float b, float c, float3* scratch) {
     for (int o = 16; o > 0; o >>= 1) {
         a += __shfl_xor_sync(0xffffffffu, a, o);
@@ -124,7 +129,7 @@ __device__ __forceinline__ float3 block_sum3(float a, float b, float c, float3* 
         c += __shfl_xor_sync(0xffffffffu, c, o);
     }
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    __syncthreads();
+    if (kGuard) __syncthreads();
     if (lane == 0) scratch[warp] = make_float3(a, b, c);
     __syncthreads();
     float3 r = scratch[0];
