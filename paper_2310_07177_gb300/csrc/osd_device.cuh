@@ -104,6 +104,17 @@ __device__ __forceinline__ float mul_c(float d, float c_hi, float c_lo) {
     return fmaf(d, c_hi, d * c_lo);
 }
 
+// The two bf16 halves (low = lower address) of a 32-bit word minus m: each half
+// converts to fp32 exactly and the difference is rounded once, as unpacking and
+// subtracting would give, by the mixed-precision subtract of sm_100+.
+__device__ __forceinline__ float2 bf16x2_minus(uint32_t w, float m) {
+    float a, b;
+    asm("{\n .reg .b16 lo, hi;\n mov.b32 {lo, hi}, %2;\n"
+        " sub.rn.f32.bf16 %0, lo, %3;\n sub.rn.f32.bf16 %1, hi, %3;\n}"
+        : "=f"(a), "=f"(b) : "r"(w), "f"(m));
+    return make_float2(a, b);
+}
+
 // ---------------------------------------------------------------- packed f32x2 (sm_100+)
 // Two fp32 lanes per instruction; the pack/unpack moves vanish in register allocation.
 __device__ __forceinline__ unsigned long long pk2(float a, float b) {

@@ -202,6 +202,17 @@ __device__ __forceinline__ void tvd_gradient(const In* zs, const In* ts, int n, 
     }
 }
 
+// The packed words of the 16-byte chunk at entry j0 of both staged rows (bf16),
+// clamped as the sweep clamps them.
+template <typename In, bool kClampZ, bool kClampT>
+__device__ __forceinline__ void raw_words(const In* zs, const In* ts, int j0, uint32_t* zw, uint32_t* tw) {
+    uint4 zr = lds_v4(zs + j0), tr = lds_v4(ts + j0);
+    if (kClampZ) Elem<In>::clamp_raw(zr);
+    if (kClampT) Elem<In>::clamp_raw(tr);
+    zw[0] = zr.x; zw[1] = zr.y; zw[2] = zr.z; zw[3] = zr.w;
+    tw[0] = tr.x; tw[1] = tr.y; tw[2] = tr.z; tw[3] = tr.w;
+}
+
 template <typename In, int kKind, bool kAligned>
 __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     // JSD clamps both rows to -1e30: a zero probability then stays exactly 0 and
@@ -495,7 +506,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     const bool has_ninf = (st.err & 2) != 0;  // some logit of the row is -inf
     const float cu = s_cu, cv = s_cv;
     const float2 mt2 = f2(st.mt), mz2 = f2(st.mz);
-    auto log2p = [&](float2 x) { return fma2(sub2(x, mt2), f2(c), f2(cu)); };
+    auto log2p = [&](float2 x) { return fma2(sub2(x, mt2), f2(c), f2(cu)); };  // pass 2
     auto log2q = [&](float2 x) { return fma2(sub2(x, mz2), f2(c), f2(cv)); };
     float loss = s_loss;
 
@@ -609,24 +620,37 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         sweep<In, kAligned, kClampZ, kClampT, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
                                                                     int j0, float, float, bool) {
             constexpr int kCnt = decltype(tag)::value;
+            // bf16 chunks of FKL/RKL, which need x - m of both rows, take the differences straight
+            // from the packed words (mixed-precision subtracts) instead of unpacking first;
+            // measured, CE and JSD do better unpacking
+            constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && (kKind == OSD_FKL || kKind == OSD_RKL);
+            uint32_t zw[4], tw[4];
+            if constexpr (kRaw) raw_words<In, kClampZ, kClampT>(zs, ts, j0, zw, tw);
+            // x - m of the pair at e, from the packed words or the unpacked values
+            auto zdiff = [&](int e, float m) {
+                if constexpr (kRaw) return bf16x2_minus(zw[e / 2], m);
+                else return sub2(make_float2(z[e], (e + 1 < kCnt) ? z[e + 1] : z[e]), f2(m));
+            };
+            auto tdiff = [&](int e, float m) {
+                if constexpr (kRaw) return bf16x2_minus(tw[e / 2], m);
+                else return sub2(make_float2(t[e], (e + 1 < kCnt) ? t[e + 1] : t[e]), f2(m));
+            };
             float gr[kCnt];
 #pragma unroll
             for (int e = 0; e < kCnt; e += 2) {
                 const bool two = (e + 1 < kCnt);
-                const float2 zz = make_float2(z[e], two ? z[e + 1] : z[e]);
-                const float2 tt = make_float2(t[e], two ? t[e + 1] : t[e]);
-                const float2 zd = sub2(zz, mz2);
+                const float2 zd = zdiff(e, st.mz);
                 const float2 v = fma2(zd, f2(c), cvs);  // log2 q + lg_scale
                 const float2 qj = make_float2(ex2(v.x), ex2(v.y));
                 float2 gg;
                 if (kKind == OSD_FKL) {  // (q - p) / tau
-                    const float2 u = fma2(sub2(tt, mt2), f2(c), cus);
+                    const float2 u = fma2(tdiff(e, st.mt), f2(c), cus);
                     gg = sub2(qj, make_float2(ex2(u.x), ex2(u.y)));
                 } else if (kKind == OSD_CE) {  // (q - onehot(y*)) / tau
                     const int j = e0 + j0 + e;
                     gg = sub2(qj, make_float2(j == label ? inv_tau : 0.f, j + 1 == label ? inv_tau : 0.f));
                 } else if (kKind == OSD_RKL) {  // q_j (D_j - sum_k q_k D_k) / tau
-                    const float2 dd = sub2(zd, sub2(tt, f2(tpg)));
+                    const float2 dd = sub2(zd, tdiff(e, tpg));
                     gg = mul2(qj, fma2(dd, f2(inv_tau), f2(-K)));
                     if (has_ninf) {  // q = 0 against an infinite log-ratio contributes 0
                         if (!(qj.x > 0.f)) gg.x = 0.f;
@@ -636,7 +660,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
                     if (jsd_trivial) {
                         gg = f2(0.f);
                     } else {
-                        const float2 d = sub2(v, fma2(sub2(tt, mt2), f2(c), cus));  // log2 q - log2 p
+                        const float2 d = sub2(v, fma2(tdiff(e, st.mt), f2(c), cus));  // log2 q - log2 p
                         const float dd[2] = {d.x, d.y};
                         float l2mq[2];
 #pragma unroll
