@@ -202,17 +202,6 @@ __device__ __forceinline__ void tvd_gradient(const In* zs, const In* ts, int n, 
     }
 }
 
-// The packed words of the 16-byte chunk at entry j0 of both staged rows (bf16),
-// clamped as the sweep clamps them.
-template <typename In, bool kClampZ, bool kClampT>
-__device__ __forceinline__ void raw_words(const In* zs, const In* ts, int j0, uint32_t* zw, uint32_t* tw) {
-    uint4 zr = lds_v4(zs + j0), tr = lds_v4(ts + j0);
-    if (kClampZ) Elem<In>::clamp_raw(zr);
-    if (kClampT) Elem<In>::clamp_raw(tr);
-    zw[0] = zr.x; zw[1] = zr.y; zw[2] = zr.z; zw[3] = zr.w;
-    tw[0] = tr.x; tw[1] = tr.y; tw[2] = tr.z; tw[3] = tr.w;
-}
-
 template <typename In, int kKind, bool kAligned>
 __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     // JSD clamps both rows to -1e30: a zero probability then stays exactly 0 and
@@ -292,7 +281,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     int jz = -1, jt = -1;
     if (!err_local) {
         sweep<In, kAligned, kClampZ, kClampT, true>(zs, ts, n, [&](const float*, const float*, auto, int j0,
-                                                                   float cz, float ct, bool) {
+                                                                   float cz, float ct, bool, const uint4&, const uint4&) {
             if (cz > mz) { mz = cz; jz = j0; }
             if (ct > mt) { mt = ct; jt = j0; }
         });
@@ -359,7 +348,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         const float2 nMz2 = f2(-Mz), nMt2 = f2(-Mt);
         sweep<In, kAligned, kClampZ, kClampT, false, kMoment>(zs, ts, n, [&](const float* z, const float* t,
                                                                              auto tag, int, float, float,
-                                                                             bool ninf) {
+                                                                             bool ninf, const uint4&, const uint4&) {
             constexpr int kCnt = decltype(tag)::value;
             row_ninf |= ninf;
             if (kCnt == 1 || ninf) {  // element-wise, with the guards a -inf needs
@@ -518,14 +507,24 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         float2 A2 = f2(0.f), B2 = f2(0.f), C2 = f2(0.f);
         if (!row_err && !jsd_trivial) {
             sweep<In, kAligned, kClampZ, kClampT, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
-                                                                        int j0, float, float, bool) {
+                                                                        int j0, float, float, bool, const uint4& zr, const uint4& tr) {
                 constexpr int kCnt = decltype(tag)::value;
+                // TVD's bf16 chunks: x - m straight from the packed words the sweep loaded
+                // (measured, JSD does as well unpacking)
+                constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && kKind == OSD_TVD;
+                const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw[4] = {tr.x, tr.y, tr.z, tr.w};
                 float qs[kCnt];  // TVD: q sign(q - p), kept for pass 3
 #pragma unroll
                 for (int e = 0; e < kCnt; e += 2) {
                     const bool two = (e + 1 < kCnt);
-                    const float2 u = log2p(make_float2(t[e], two ? t[e + 1] : t[e]));  // log2 p
-                    const float2 v = log2q(make_float2(z[e], two ? z[e + 1] : z[e]));  // log2 q
+                    float2 u, v;  // log2 p, log2 q
+                    if constexpr (kRaw) {
+                        u = fma2(bf16x2_minus(tw[e / 2], st.mt), f2(c), f2(cu));
+                        v = fma2(bf16x2_minus(zw[e / 2], st.mz), f2(c), f2(cv));
+                    } else {
+                        u = log2p(make_float2(t[e], two ? t[e + 1] : t[e]));
+                        v = log2q(make_float2(z[e], two ? z[e + 1] : z[e]));
+                    }
                     float2 a, b, c2 = f2(0.f);
                     if (kKind == OSD_TVD) {
                         const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
@@ -618,14 +617,13 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         const float2 cvs = f2(cv + p.lg_scale), cus = f2(cu + p.lg_scale);
         const int label = st.idx;
         sweep<In, kAligned, kClampZ, kClampT, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
-                                                                    int j0, float, float, bool) {
+                                                                    int j0, float, float, bool, const uint4& zr, const uint4& tr) {
             constexpr int kCnt = decltype(tag)::value;
             // bf16 chunks of FKL/RKL, which need x - m of both rows, take the differences straight
             // from the packed words (mixed-precision subtracts) instead of unpacking first;
             // measured, CE and JSD do better unpacking
             constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && (kKind == OSD_FKL || kKind == OSD_RKL);
-            uint32_t zw[4], tw[4];
-            if constexpr (kRaw) raw_words<In, kClampZ, kClampT>(zs, ts, j0, zw, tw);
+            const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw[4] = {tr.x, tr.y, tr.z, tr.w};
             // x - m of the pair at e, from the packed words or the unpacked values
             auto zdiff = [&](int e, float m) {
                 if constexpr (kRaw) return bf16x2_minus(zw[e / 2], m);

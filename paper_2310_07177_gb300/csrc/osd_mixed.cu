@@ -88,7 +88,7 @@ __global__ void __launch_bounds__(kRowThreads) mixed_sample_kernel(MixParams p) 
     float mz = kNegInf, mt = kNegInf;
     if (!err_local) {
         sweep<In, kAligned, false, false, true>(zs, ts, n, [&](const float*, const float*, auto, int, float cz,
-                                                               float ct, bool) {
+                                                               float ct, bool, const uint4&, const uint4&) {
             mz = fmaxf(mz, cz);
             mt = fmaxf(mt, ct);
         });

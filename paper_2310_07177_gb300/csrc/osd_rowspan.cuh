@@ -62,9 +62,9 @@ __device__ __forceinline__ int stage_span(In* zs, In* ts, const In* zsrc, const 
 
 // Visit this thread's entries of a staged span in chunks of one 16-byte vector
 // (or single entries on the element-wise path).  Clamping (to -1e30, see Elem)
-// happens on the packed words.  f(z[], t[], count_tag, j0, zmax, tmax, ninf)
-// gets the chunk maxima when kMax is set, and ninf = "the chunk holds a -inf"
-// when kMin is set.  Chunk v goes to thread v mod kRowThreads, so warp w sees
+// happens on the packed words.  f(z[], t[], count_tag, j0, zmax, tmax, ninf,
+// zraw, traw) gets the chunk maxima when kMax is set, ninf = "the chunk holds a
+// -inf" when kMin is set, and the (clamped) packed words of a full chunk.  Chunk v goes to thread v mod kRowThreads, so warp w sees
 // the 32-chunk groups w, w + kRowWarps, ... in order.
 template <typename In, bool kAligned, bool kClampZ, bool kClampT, bool kMax, bool kMin = false, typename F>
 __device__ __forceinline__ void sweep(const In* zs, const In* ts, int n, F&& f) {
@@ -82,21 +82,21 @@ __device__ __forceinline__ void sweep(const In* zs, const In* ts, int n, F&& f) 
             E::unpack(tr, t);
             const float cz = kMax ? E::max_raw(zr) : 0.f, ct = kMax ? E::max_raw(tr) : 0.f;
             const bool ninf = kMin ? (fminf(E::min_raw(zr), E::min_raw(tr)) == kNegInf) : false;
-            f(z, t, std::integral_constant<int, kVec>{}, v * kVec, cz, ct, ninf);
+            f(z, t, std::integral_constant<int, kVec>{}, v * kVec, cz, ct, ninf, zr, tr);
         }
         const int r0 = nv * kVec;
         if (tid < n - r0) {
             float z = E::lds(zs + r0 + tid), t = E::lds(ts + r0 + tid);
             if (kClampZ) z = E::clamp1(z);
             if (kClampT) t = E::clamp1(t);
-            f(&z, &t, std::integral_constant<int, 1>{}, r0 + tid, z, t, fminf(z, t) == kNegInf);
+            f(&z, &t, std::integral_constant<int, 1>{}, r0 + tid, z, t, fminf(z, t) == kNegInf, uint4{}, uint4{});
         }
     } else {
         for (int e = tid; e < n; e += kRowThreads) {
             float z = E::lds(zs + e), t = E::lds(ts + e);
             if (kClampZ) z = E::clamp1(z);
             if (kClampT) t = E::clamp1(t);
-            f(&z, &t, std::integral_constant<int, 1>{}, e, z, t, fminf(z, t) == kNegInf);
+            f(&z, &t, std::integral_constant<int, 1>{}, e, z, t, fminf(z, t) == kNegInf, uint4{}, uint4{});
         }
     }
 }
