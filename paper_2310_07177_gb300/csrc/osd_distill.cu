@@ -107,6 +107,12 @@ __device__ __forceinline__ Label merge_label(Label a, Label b) {
     return (b.m > a.m || (b.m == a.m && b.i < a.i)) ? b : a;
 }
 
+// Write one (exactly representable) value back to a staged row.
+__device__ __forceinline__ void store_elem(float* p, float x) { *p = x; }
+__device__ __forceinline__ void store_elem(__nv_bfloat16* p, float x) {
+    *reinterpret_cast<unsigned short*>(p) = static_cast<unsigned short>(__float_as_uint(x) >> 16);
+}
+
 // TVD keeps q' = q sign(q - p) (fp32) in the two 16-bit (bf16) or the first
 // 32-bit (fp32) staging slots of each entry once pass 2 has read its logits.
 __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
@@ -280,10 +286,20 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     float mz = kNegInf, mt = kNegInf;
     int jz = -1, jt = -1;
     if (!err_local) {
-        sweep<In, kAligned, kClampZ, kClampT, true>(zs, ts, n, [&](const float*, const float*, auto, int j0,
-                                                                   float cz, float ct, bool, const uint4&, const uint4&) {
+        sweep<In, kAligned, kClampZ, kClampT, true>(zs, ts, n, [&](const float* z, const float* t, auto tag,
+                                                                   int j0, float cz, float ct, bool,
+                                                                   const uint4& zr, const uint4& tr) {
             if (cz > mz) { mz = cz; jz = j0; }
             if (ct > mt) { mt = ct; jt = j0; }
+            if constexpr (kClamp) {  // clamp the staged logits once, for every later pass
+                if constexpr (decltype(tag)::value > 1) {
+                    *reinterpret_cast<uint4*>(zs + j0) = zr;
+                    *reinterpret_cast<uint4*>(ts + j0) = tr;
+                } else {
+                    store_elem(zs + j0, z[0]);
+                    store_elem(ts + j0, t[0]);
+                }
+            }
         });
     }
     // the entry that holds a maximum: RKL's pivot target logit, CE's label
@@ -346,7 +362,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     if (!err_local) {
         const float2 gz2 = f2(gzb), gt2 = f2(gtb), tp2 = f2(tpv);
         const float2 nMz2 = f2(-Mz), nMt2 = f2(-Mt);
-        sweep<In, kAligned, kClampZ, kClampT, false, kMoment>(zs, ts, n, [&](const float* z, const float* t,
+        sweep<In, kAligned, false, false, false, kMoment>(zs, ts, n, [&](const float* z, const float* t,
                                                                              auto tag, int, float, float,
                                                                              bool ninf, const uint4&, const uint4&) {
             constexpr int kCnt = decltype(tag)::value;
@@ -506,8 +522,8 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         // ---- pass 2: divergence terms with the global normalisers
         float2 A2 = f2(0.f), B2 = f2(0.f), C2 = f2(0.f);
         if (!row_err && !jsd_trivial) {
-            sweep<In, kAligned, kClampZ, kClampT, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
-                                                                        int j0, float, float, bool, const uint4& zr, const uint4& tr) {
+            sweep<In, kAligned, false, false, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
+                                                                    int j0, float, float, bool, const uint4& zr, const uint4& tr) {
                 constexpr int kCnt = decltype(tag)::value;
                 // TVD's bf16 chunks: x - m straight from the packed words the sweep loaded
                 // (measured, JSD does as well unpacking)
@@ -616,8 +632,8 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         // q and p of this pass come out multiplied by the gradient's constant factor
         const float2 cvs = f2(cv + p.lg_scale), cus = f2(cu + p.lg_scale);
         const int label = st.idx;
-        sweep<In, kAligned, kClampZ, kClampT, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
-                                                                    int j0, float, float, bool, const uint4& zr, const uint4& tr) {
+        sweep<In, kAligned, false, false, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
+                                                                int j0, float, float, bool, const uint4& zr, const uint4& tr) {
             constexpr int kCnt = decltype(tag)::value;
             // bf16 chunks of FKL/RKL, which need x - m of both rows, take the differences straight
             // from the packed words (mixed-precision subtracts) instead of unpacking first;
