@@ -79,7 +79,7 @@ const char *osd_status_string(osd_status status);
 /* ABI version of this library: (major << 16) | minor.  2.0 added the
  * temperature argument of osd_distill and the OSD_CE loss; 2.1 added
  * osd_distill_accepted; 2.2 added osd_mixed_sample; 2.3 added
- * osd_verify_tree. */
+ * osd_verify_tree; 2.4 added osd_check_bounded_wait. */
 int osd_abi_version(void);
 
 /*
@@ -315,6 +315,20 @@ osd_status osd_mixed_sample(const void *draft_logits, const void *target_logits,
                             int N, int V, int64_t d_stride, int64_t t_stride,
                             const float *uniforms, float beta, float temperature,
                             int32_t *tokens, float *cdf_gap, int32_t *status, void *stream);
+
+/*
+ * Health check of the failure path every staging kernel shares: a bounded
+ * wait on an mbarrier (the one that guards the bulk copies of osd_distill,
+ * osd_distill_accepted and osd_mixed_sample) is run against a barrier that
+ * nothing completes.  When limit_us microseconds have passed it writes
+ * OSD_ERR_TIMEOUT to the device int32 *status (OSD_OK would mean the wait
+ * completed, which cannot happen) and the nanoseconds it waited to the device
+ * uint64 *waited_ns (nullable).  The kernel then exits
+ * normally, so the context stays usable; no logits are read.
+ * Returns OSD_ERR_INVALID_ARG for a null `status`, misalignment, or limit_us
+ * outside [1, 10^7].
+ */
+osd_status osd_check_bounded_wait(uint32_t limit_us, int32_t *status, uint64_t *waited_ns, void *stream);
 
 #ifdef __cplusplus
 }

@@ -30,7 +30,7 @@ VERIFY_MAX_V = 1 << 21
 # every symbol include/osd.h declares
 EXPORTS = ("osd_status_string", "osd_abi_version", "osd_verify_workspace_size",
            "osd_verify", "osd_verify_noalloc", "osd_distill", "osd_distill_accepted",
-           "osd_mixed_sample", "osd_verify_tree_workspace_size", "osd_verify_tree")
+           "osd_mixed_sample", "osd_verify_tree_workspace_size", "osd_verify_tree", "osd_check_bounded_wait")
 
 
 class OsdError(RuntimeError):
@@ -74,6 +74,8 @@ def load_library():
     lib.osd_verify_tree.restype = i32
     lib.osd_verify_tree.argtypes = [vp, vp, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_int32), vp, vp, f32,
                                     vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.osd_check_bounded_wait.restype = i32
+    lib.osd_check_bounded_wait.argtypes = [ctypes.c_uint32, vp, vp, vp]
     lib.osd_mixed_sample.restype = i32
     lib.osd_mixed_sample.argtypes = [vp, vp, i32, i32, i32, i64, i64, vp, f32, f32, vp, vp, vp, vp]
     _lib = lib
@@ -388,3 +390,17 @@ def osd_verify_tree(draft_logits: Optional[torch.Tensor], target_logits: torch.T
     if st != OSD_OK:
         raise OsdError(st, "osd_verify_tree")
     return out
+
+
+def osd_check_bounded_wait(limit_us: int, *, device=None, stream: Optional[torch.cuda.Stream] = None):
+    """Run the shared bounded-wait failure path against a barrier nothing
+    completes; returns (status, waited_ns) read back from the device (status is
+    OSD_ERR_TIMEOUT when the path works)."""
+    lib = load_library()
+    dev = torch.device("cuda") if device is None else torch.device(device)
+    st = torch.full((1,), -1, dtype=torch.int32, device=dev)
+    waited = torch.zeros(1, dtype=torch.int64, device=dev)
+    rc = lib.osd_check_bounded_wait(int(limit_us), _ptr(st), _ptr(waited), _stream(dev, stream))
+    if rc != OSD_OK:
+        raise OsdError(rc, "osd_check_bounded_wait")
+    return int(st.item()), int(waited.item())

@@ -115,6 +115,10 @@ def test_argument_errors_return_before_any_launch(lib):
     n = ctypes.c_size_t(0)
     assert lib.osd_verify_tree_workspace_size(32, 27, 32000, ctypes.byref(n)) == osd.OSD_OK
     assert n.value >= 2 * 32 * 27 * 16 and n.value % 256 == 0
+    # the bounded-wait check: null status, zero or huge limit
+    assert lib.osd_check_bounded_wait(1000, None, None, None) == osd.OSD_ERR_INVALID_ARG
+    assert lib.osd_check_bounded_wait(0, fake, None, None) == osd.OSD_ERR_INVALID_ARG
+    assert lib.osd_check_bounded_wait(20_000_000, fake, None, None) == osd.OSD_ERR_INVALID_ARG
     # mixed sampling: beta outside [0, 1], bad temperature, null uniforms, V beyond the limit
     fm = lib.osd_mixed_sample
     assert fm(fake, fake, 1, 2, 16, 16, 16, fake, 1.5, 1.0, fake, None, None, None) == osd.OSD_ERR_INVALID_ARG
