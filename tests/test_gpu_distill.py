@@ -59,6 +59,8 @@ SHAPES = [  # (N, V, dtype)
     (3, 33001, torch.bfloat16),
     (2, 32128, torch.float32),
     (2, 128256, torch.bfloat16),
+    (2, 393216, torch.bfloat16),   # the largest vocabulary per dtype: 192 KB of staging per CTA
+    (2, 196608, torch.float32),
 ]
 
 

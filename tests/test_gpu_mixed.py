@@ -67,6 +67,8 @@ SHAPES = [  # (N, V, dtype)
     (6, 32128, torch.float32),
     (3, 128256, torch.bfloat16),
     (2, 65539, torch.float32),
+    (2, 393216, torch.bfloat16),   # the largest vocabulary per dtype
+    (2, 196608, torch.float32),
 ]
 
 

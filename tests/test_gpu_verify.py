@@ -50,6 +50,10 @@ CASES = [  # (B, k, V, dtype, T)
     (4, 4, 33001, torch.bfloat16, 0.7),
     (3, 6, 32000, torch.bfloat16, 1.0),
     (8, 2, 65539, torch.float32, 1.0),
+    (512, 4, 16, torch.bfloat16, 1.0),       # many sequences over a tiny vocabulary
+    (1024, 8, 64, torch.float32, 0.7),
+    (16, 64, 300, torch.bfloat16, 1.0),      # the largest k
+    (2, 3, 1 << 21, torch.bfloat16, 1.0),    # the largest vocabulary
 ]
 
 
