@@ -416,13 +416,17 @@ def _time_tree_verify(osd, dev, l2_flush, stream, reps):
 
 
 def run_e2e(args, osd, setup, dev, stream, positions, wl):
-    """Same step through the public API from pinned host buffers: inputs copied
-    host->device and results device->host inside the timed region."""
+    """Same step through the public API from pinned host buffers: every step's
+    inputs are copied host->device and its results read device->host inside
+    the timed region.  As a server would, the step pipelines: the upload of
+    step i+1's inputs (into the second of two device buffer sets, on a copy
+    stream) runs while step i's kernels run."""
     import torch
     v = setup["v"]
     sv = setup["spec_v"]
+    nbuf = 2
     host = {k: v[k].cpu().pin_memory() for k in ("draft", "target", "tokens", "greedy_tokens", "uniforms")}
-    dv = {k: torch.empty_like(v[k]) for k in host}
+    dv = [{k: torch.empty_like(v[k]) for k in host} for _ in range(nbuf)]
     h_out = {"acc": torch.empty(sv.B, dtype=torch.int32).pin_memory(),
              "tok": torch.empty(sv.B, sv.k + 1, dtype=torch.int32).pin_memory(),
              "mask": torch.empty(sv.B, sv.k, dtype=torch.uint8).pin_memory()}
@@ -439,52 +443,76 @@ def run_e2e(args, osd, setup, dev, stream, positions, wl):
              "count": torch.empty(1, dtype=torch.int32).pin_memory()}
     d2h = (h_out["acc"].numel() * 4 + h_out["tok"].numel() * 4 + h_out["mask"].numel()
            + sum(t.numel() * 4 for t in h_rej.values()))
+    hd, dd = {}, [{} for _ in range(nbuf)]
     if wl == "serving-32k":
         d = setup["d"]
         sd = setup["spec_d"]
         hd = {"draft": d["draft"].cpu().pin_memory(), "target": d["target"].cpu().pin_memory()}
-        dd = {k: torch.empty_like(d[k]) for k in hd}
+        dd = [{k: torch.empty_like(d[k]) for k in hd} for _ in range(nbuf)]
         loss = torch.empty(sd.N, dtype=torch.float32, device=dev)
         dl = torch.empty(sd.N, sd.V, dtype=torch.float32, device=dev)
         h_loss = torch.empty(2, sd.N, dtype=torch.float32).pin_memory()
         h2d += sum(t.numel() * t.element_size() for t in hd.values())
         d2h += h_out["acc"].numel() * 4 + h_out["tok"].numel() * 4 + h_out["mask"].numel() + h_loss.numel() * 4
 
-    def step():
-        for k in host:
-            dv[k].copy_(host[k], non_blocking=True)
-        r = osd.osd_verify(dv["draft"], dv["target"], dv["tokens"], dv["uniforms"], sv.temperature, workspace=ws)
+    copy_stream = torch.cuda.Stream(dev)
+    copied = [torch.cuda.Event() for _ in range(nbuf)]
+    free = [torch.cuda.Event() for _ in range(nbuf)]
+    for ev in free:
+        ev.record(stream)
+
+    def upload(i):
+        """Step i's inputs into buffer set i % 2, once step i-2's kernels are done with it."""
+        bi = i % nbuf
+        copy_stream.wait_event(free[bi])
+        with torch.cuda.stream(copy_stream):
+            for k in host:
+                dv[bi][k].copy_(host[k], non_blocking=True)
+            for k in hd:
+                dd[bi][k].copy_(hd[k], non_blocking=True)
+        copied[bi].record(copy_stream)
+
+    def compute(i):
+        bi = i % nbuf
+        stream.wait_event(copied[bi])
+        x, xd = dv[bi], dd[bi]
+        r = osd.osd_verify(x["draft"], x["target"], x["tokens"], x["uniforms"], sv.temperature, workspace=ws)
         h_out["acc"].copy_(r.accepted, non_blocking=True)
         h_out["tok"].copy_(r.out_tokens, non_blocking=True)
         h_out["mask"].copy_(r.mismatch_mask, non_blocking=True)
-        osd.osd_distill_accepted(dv["draft"], dv["target"], r.accepted, rej_kind, 0.5, out=rej)
+        osd.osd_distill_accepted(x["draft"], x["target"], r.accepted, rej_kind, 0.5, out=rej)
         h_rej["loss"].copy_(rej.loss, non_blocking=True)
         h_rej["seq"].copy_(rej.seq_of_row, non_blocking=True)
         h_rej["count"].copy_(rej.count, non_blocking=True)
         if wl == "serving-32k":
-            r0 = osd.osd_verify(None, dv["target"], dv["greedy_tokens"], None, 0.0, workspace=ws)
+            r0 = osd.osd_verify(None, x["target"], x["greedy_tokens"], None, 0.0, workspace=ws)
             h_out["acc"].copy_(r0.accepted, non_blocking=True)
             h_out["tok"].copy_(r0.out_tokens, non_blocking=True)
             h_out["mask"].copy_(r0.mismatch_mask, non_blocking=True)
-            for k in hd:
-                dd[k].copy_(hd[k], non_blocking=True)
-            for i, kind in enumerate(("rkl", "tvd")):
-                osd.osd_distill(dd["draft"], dd["target"], None, kind, 0.5, loss=loss, dlogits=dl)
-                h_loss[i].copy_(loss, non_blocking=True)
+            for i2, kind in enumerate(("rkl", "tvd")):
+                osd.osd_distill(xd["draft"], xd["target"], None, kind, 0.5, loss=loss, dlogits=dl)
+                h_loss[i2].copy_(loss, non_blocking=True)
+        free[bi].record(stream)
 
-    for _ in range(max(1, args.warmup)):
-        step()
+    def steps(count):
+        upload(0)
+        for i in range(count):
+            if i + 1 < count:
+                upload(i + 1)
+            compute(i)
+
+    steps(max(2, args.warmup))
     torch.cuda.synchronize()
     n = max(3, args.steps // 2)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(n):
-        step()
-    e1.record(stream)
+    e0.record(copy_stream)  # before the first upload
+    steps(n)
+    e1.record(stream)       # after the last step's kernels and read-backs
     e1.synchronize()
     ms = e0.elapsed_time(e1) / n
     return {"value": round(positions / (ms / 1e3), 1), "unit": "positions/s", "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "ms_per_step": round(ms, 3), "steps": n,
+            "pipelined": "step i+1's upload overlaps step i's kernels (two device buffer sets, a copy stream)",
             "note": "dlogits stays on the device, where the draft model's backward pass consumes it"}
 
 
