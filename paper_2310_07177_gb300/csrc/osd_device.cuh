@@ -256,6 +256,17 @@ __device__ __forceinline__ double warp_incl_scan_f64(double v) {
     return v;
 }
 
+// ---------------------------------------------------------------- programmatic dependent launch
+// A kernel lets the next kernel on its stream (launched with programmatic stream
+// serialisation) start; that kernel waits for this one's results and memory only
+// where it calls grid_dependency_wait.  Both are no-ops without the attribute.
+__device__ __forceinline__ void allow_dependent_launch() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dependency_wait() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 // ---------------------------------------------------------------- timers / errors
 __device__ __forceinline__ uint64_t global_ns() {
     uint64_t t;

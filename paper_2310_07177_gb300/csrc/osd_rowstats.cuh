@@ -71,6 +71,7 @@ row_stats_kernel(const In* __restrict__ draft, const In* __restrict__ target,
     __shared__ float red_s[kStatThreads / 32];
     __shared__ MaxIdx red_mi[kStatThreads / 32];
 
+    allow_dependent_launch();  // the consumer of the statistics waits for them in-kernel
     const long long item = blockIdx.x;
     const long long row = item / n_slices;
     const int slice = static_cast<int>(item - row * n_slices);

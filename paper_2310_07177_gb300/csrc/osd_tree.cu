@@ -105,6 +105,7 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
     }
     if (bad) return;  // uniform over the cluster, before any shared-memory exchange
     __syncthreads();  // the initialisation above lands before the walk writes its entries
+    grid_dependency_wait();  // the row statistics are complete from here on
 
     const int e0 = rank * p.span;
     const int cnt = max(0, min(p.span, V - e0));
@@ -461,9 +462,9 @@ static osd_status launch_tree(const TreeParams& base, int B, const void* draft, 
     if (smem > size_t(kTreeMaxSub) * sizeof(float)) return OSD_ERR_UNSUPPORTED;
     const dim3 grid2(unsigned(B) * unsigned(csize));
     if (vec)
-        e = launch(tree_walk_kernel<In, true>, grid2, dim3(kTreeThreads), smem, stream, csize, tp);
+        e = launch_ex(true, tree_walk_kernel<In, true>, grid2, dim3(kTreeThreads), smem, stream, csize, tp);
     else
-        e = launch(tree_walk_kernel<In, false>, grid2, dim3(kTreeThreads), smem, stream, csize, tp);
+        e = launch_ex(true, tree_walk_kernel<In, false>, grid2, dim3(kTreeThreads), smem, stream, csize, tp);
     return from_cuda(e);
 }
 

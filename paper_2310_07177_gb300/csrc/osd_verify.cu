@@ -106,6 +106,7 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
     }
     if (!greedy && warp == kWarps - 2)
         for (int i = lane; i <= k; i += 32) s_u[i] = p.uniforms[size_t(b) * (k + 1) + i];
+    grid_dependency_wait();  // the row statistics are complete from here on
     const int nrows = greedy ? (k + 1) : (2 * k + 1);
     const float ch0 = p.c_hi, cl0 = p.c_lo;
     auto srow_of = [&](int r) -> long long {
@@ -494,9 +495,9 @@ static osd_status launch_verify(const void* draft, const void* target, int B, in
     const size_t smem2 = greedy ? 0 : size_t((span + sub - 1) / sub) * sizeof(float);
     if (smem2 > size_t(kFinMaxSub) * sizeof(float)) return OSD_ERR_UNSUPPORTED;
     if (vec)
-        e = launch(verify_finalize_kernel<In, true>, grid2, dim3(kFinThreads), smem2, stream, csize, fp);
+        e = launch_ex(true, verify_finalize_kernel<In, true>, grid2, dim3(kFinThreads), smem2, stream, csize, fp);
     else
-        e = launch(verify_finalize_kernel<In, false>, grid2, dim3(kFinThreads), smem2, stream, csize, fp);
+        e = launch_ex(true, verify_finalize_kernel<In, false>, grid2, dim3(kFinThreads), smem2, stream, csize, fp);
     return from_cuda(e);
 }
 
