@@ -34,6 +34,8 @@ namespace osd {
 constexpr int kMixMaxCluster = 8;
 constexpr int kMixSpanBytes = 32768;     // target bytes of both rows per CTA
 constexpr int kMixMaxSmem = 192 * 1024;  // largest staging buffer per CTA
+constexpr int kGroups = 8;               // CDF pieces per warp range (kRowWarps * kGroups = 32)
+static_assert(kRowWarps * kGroups == 32, "one CDF piece per lane of the picking warp");
 
 struct MixParams {
     const void* draft;
@@ -65,6 +67,7 @@ __global__ void __launch_bounds__(kRowThreads) mixed_sample_kernel(MixParams p) 
     __shared__ int s_err;
     __shared__ float2 red_m[kRowWarps];
     __shared__ float2 s_rng[kRowWarps];  // (sum 2^((t-m)c), sum 2^((z-m)c)) of each warp's range
+    __shared__ float2 s_piece[kRowWarps * kGroups];  // the same over each run of steps
     __shared__ MixStats s_mine;
     __shared__ int s_owner, s_mode, s_bad;
     __shared__ float s_a, s_b;
@@ -118,35 +121,62 @@ __global__ void __launch_bounds__(kRowThreads) mixed_sample_kernel(MixParams p) 
     };
     auto exp_one = [&](float x, float m) { return ex2(mul_c(x - m, ch, cl)); };
 
-    // ---- pass 1: sums over each warp's contiguous range [lo(w), lo(w + 1))
+    // ---- pass 1: each warp's contiguous range [lo(w), lo(w + 1)) in steps of 32 chunks,
+    // the steps split into kGroups runs whose sums stay in registers until the loop ends:
+    // kRowWarps x kGroups pieces of the CDF, with no shuffle inside the loop
     const int nchunks = (n + kVec - 1) / kVec;
     const int range_len = (nchunks + kRowWarps - 1) / kRowWarps * kVec;
     auto range_lo = [&](int w) { return min(n, w * range_len); };
+    const int steps = (range_len / kVec + 31) / 32;      // per warp
+    const int per_group = (steps + kGroups - 1) / kGroups;
+    // a span with no mass: its logits are -inf, and so are x - 0
+    const float gz_ref = zok ? gzb : 0.f, gt_ref = tok ? gtb : 0.f;
     {
-        float2 T2 = f2(0.f), Z2 = f2(0.f);
-        if (!err_local) {
-            const int hi = range_lo(warp + 1);
-            for (int j = range_lo(warp) + lane * kVec; j < hi; j += 32 * kVec) {
-                float z[kVec], t[kVec];
-                load_chunk(j, hi, z, t);
-                if constexpr (kVec == 1) {
-                    if (tok) T2.x += exp_one(t[0], gtb);
-                    if (zok) Z2.x += exp_one(z[0], gzb);
-                } else {
+        const int lo_w = range_lo(warp), hi_w = range_lo(warp + 1);
+        float Tg[kGroups], Zg[kGroups];
 #pragma unroll
-                    for (int e = 0; e < kVec; e += 2) {
-                        if (tok) T2 = add2(T2, exp_pair(t[e], t[e + 1], gtb));
-                        if (zok) Z2 = add2(Z2, exp_pair(z[e], z[e + 1], gzb));
+        for (int g = 0; g < kGroups; ++g) {
+            float2 T2 = f2(0.f), Z2 = f2(0.f);
+            if (!err_local) {
+                const int s_end = min((g + 1) * per_group, steps);
+                for (int st = g * per_group; st < s_end; ++st) {
+                    const int j = lo_w + (st * 32 + lane) * kVec;
+                    if (j < hi_w) {
+                        float z[kVec], t[kVec];
+                        load_chunk(j, hi_w, z, t);
+                        if constexpr (kVec == 1) {
+                            T2.x += exp_one(t[0], gt_ref);
+                            Z2.x += exp_one(z[0], gz_ref);
+                        } else {
+#pragma unroll
+                            for (int e = 0; e < kVec; e += 2) {
+                                T2 = add2(T2, exp_pair(t[e], t[e + 1], gt_ref));
+                                Z2 = add2(Z2, exp_pair(z[e], z[e + 1], gz_ref));
+                            }
+                        }
                     }
                 }
             }
+            Tg[g] = T2.x + T2.y;
+            Zg[g] = Z2.x + Z2.y;
         }
-        float Tw = T2.x + T2.y, Zw = Z2.x + Z2.y;
         for (int o = 16; o > 0; o >>= 1) {
-            Tw += __shfl_xor_sync(0xffffffffu, Tw, o);
-            Zw += __shfl_xor_sync(0xffffffffu, Zw, o);
+#pragma unroll
+            for (int g = 0; g < kGroups; ++g) {
+                Tg[g] += __shfl_xor_sync(0xffffffffu, Tg[g], o);
+                Zg[g] += __shfl_xor_sync(0xffffffffu, Zg[g], o);
+            }
         }
-        if (lane == 0) s_rng[warp] = make_float2(Tw, Zw);
+        if (lane == 0) {
+            float Tw = 0.f, Zw = 0.f;
+#pragma unroll
+            for (int g = 0; g < kGroups; ++g) {
+                s_piece[warp * kGroups + g] = make_float2(Tg[g], Zg[g]);
+                Tw += Tg[g];
+                Zw += Zg[g];
+            }
+            s_rng[warp] = make_float2(Tw, Zw);
+        }
     }
     __syncthreads();
     if (tid == 0) {
@@ -230,46 +260,50 @@ __global__ void __launch_bounds__(kRowThreads) mixed_sample_kernel(MixParams p) 
             if (p.status) atomicExch(p.status, static_cast<int32_t>(OSD_ERR_TIMEOUT));
         }
     } else if (rank == s_owner && warp == 0) {
-        // ---- pick: the range, then the entry, in fp64
+        // ---- pick: the piece (lane l holds piece l, in vocabulary order), then the entry, in fp64
         const float a = s_a, b = s_b;
         const double tau = s_tau, W = s_W;
         int mode = s_mode;
-        double run = s_base;
-        int rsel = -1;
+        const double mass = double(a) * double(s_piece[lane].x) + double(b) * double(s_piece[lane].y);
+        const double incl = s_base + warp_incl_scan_f64(mass);
+        int piece = -1;
+        double run = 0.0;
         if (mode == 0) {
-            for (int w = 0; w < kRowWarps; ++w) {
-                const double m = double(a) * double(s_rng[w].x) + double(b) * double(s_rng[w].y);
-                if (run + m > tau) { rsel = w; break; }
-                run += m;
+            const unsigned h = __ballot_sync(0xffffffffu, incl - mass <= tau && incl > tau);
+            if (h) {
+                piece = __ffs(h) - 1;
+                run = __shfl_sync(0xffffffffu, incl - mass, piece);
+            } else {
+                mode = 1;
             }
-            if (rsel < 0) mode = 1;
         }
-        if (mode == 1) {
-            for (int w = kRowWarps - 1; w >= 0; --w)
-                if (double(a) * double(s_rng[w].x) + double(b) * double(s_rng[w].y) > 0.0) { rsel = w; break; }
-            if (rsel < 0) rsel = 0;
+        if (mode == 1) {  // the last piece with positive mass
+            const unsigned pos = __ballot_sync(0xffffffffu, mass > 0.0);
+            piece = pos ? 31 - __clz(pos) : 0;
         }
-        const int lo = range_lo(rsel), hi = range_lo(rsel + 1);
+        const int pw = piece / kGroups, pg = piece % kGroups;
+        const int lo = range_lo(pw), hi = range_lo(pw + 1);
+        const int s_end = min((pg + 1) * per_group, steps);
         int pick = -1, last_pos = -1;
         double gap = 0.0;
         bool found = false;
-        for (int j0 = lo; j0 < hi; j0 += 32 * kVec) {  // warp-uniform trip count
-            const int j = j0 + lane * kVec;
+        for (int st = pg * per_group; st < s_end; ++st) {  // warp-uniform trip count
+            const int j = lo + (st * 32 + lane) * kVec;
             float z[kVec], t[kVec], w[kVec];
-            load_chunk(j, hi, z, t);
+            load_chunk(j, hi, z, t);  // past the range end the entries read as -inf: weight 0
 #pragma unroll
             for (int e = 0; e < kVec; ++e) {
-                const float pt = tok ? exp_one(t[e], gtb) : 0.f;
-                const float qz = zok ? exp_one(z[e], gzb) : 0.f;
+                const float pt = exp_one(t[e], gt_ref);
+                const float qz = exp_one(z[e], gz_ref);
                 w[e] = fmaf(a, pt, b * qz);
                 if (w[e] > 0.f) last_pos = j + e;
             }
             double mine = 0.0;
 #pragma unroll
             for (int e = 0; e < kVec; ++e) mine += double(w[e]);
-            const double incl = warp_incl_scan_f64(mine);
+            const double wincl = warp_incl_scan_f64(mine);
             if (mode == 0) {
-                const double excl = run + incl - mine;
+                const double excl = run + wincl - mine;
                 const unsigned h = __ballot_sync(0xffffffffu, excl <= tau && excl + mine > tau);
                 if (h) {
                     if (lane == __ffs(h) - 1) {
@@ -292,9 +326,9 @@ __global__ void __launch_bounds__(kRowThreads) mixed_sample_kernel(MixParams p) 
                 }
             }
             if (found) break;
-            run += __shfl_sync(0xffffffffu, incl, 31);
+            run += __shfl_sync(0xffffffffu, wincl, 31);
         }
-        if (!found) {  // mode 1, or rounding left tau beyond the range: the largest j with w_j > 0
+        if (!found) {  // mode 1, or rounding left tau past the piece: the largest j with w_j > 0
             int lp = last_pos;
             for (int off = 16; off > 0; off >>= 1) lp = max(lp, __shfl_xor_sync(0xffffffffu, lp, off));
             if (lane == 0) {
