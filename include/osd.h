@@ -79,7 +79,8 @@ const char *osd_status_string(osd_status status);
 /* ABI version of this library: (major << 16) | minor.  2.0 added the
  * temperature argument of osd_distill and the OSD_CE loss; 2.1 added
  * osd_distill_accepted; 2.2 added osd_mixed_sample; 2.3 added
- * osd_verify_tree; 2.4 added osd_check_bounded_wait. */
+ * osd_verify_tree; 2.4 added osd_check_bounded_wait; 2.5 raised
+ * osd_mixed_sample's vocabulary limit to OSD_VERIFY_MAX_V. */
 int osd_abi_version(void);
 
 /*
@@ -305,9 +306,11 @@ osd_status osd_verify_tree(const void *draft_logits, const void *target_logits, 
  * cdf_gap        [N] fp32 out, nullable: distance of u W to the nearest edge of
  *                the chosen CDF step, divided by W (<= 0 when rounding left
  *                no step above u W).
- * status         nullable device int32: 0, or OSD_ERR_TIMEOUT if a bounded
- *                wait for a bulk copy gave up (that row's token is then -1).
- * Limits as osd_distill's: V <= 393216 (bf16) or 196608 (fp32).
+ * status         nullable device int32, set to 0 (OSD_OK): the kernel
+ *                streams both rows with plain loads and has no wait that can
+ *                run out; kept so that every staging entry point reports the
+ *                same way.
+ * Limits: 1 <= V <= OSD_VERIFY_MAX_V, N >= 0.
  * Argument errors: OSD_ERR_INVALID_ARG (null pointers with N > 0, negative
  * sizes or strides, beta outside [0, 1], bad temperature, misalignment).
  */
@@ -318,8 +321,8 @@ osd_status osd_mixed_sample(const void *draft_logits, const void *target_logits,
 
 /*
  * Health check of the failure path every staging kernel shares: a bounded
- * wait on an mbarrier (the one that guards the bulk copies of osd_distill,
- * osd_distill_accepted and osd_mixed_sample) is run against a barrier that
+ * wait on an mbarrier (the one that guards the bulk copies of osd_distill
+ * and osd_distill_accepted) is run against a barrier that
  * nothing completes.  When limit_us microseconds have passed it writes
  * OSD_ERR_TIMEOUT to the device int32 *status (OSD_OK would mean the wait
  * completed, which cannot happen) and the nanoseconds it waited to the device

@@ -12,4 +12,4 @@ extern "C" const char* osd_status_string(osd_status status) {
     return "OSD_ERR_UNKNOWN";
 }
 
-extern "C" int osd_abi_version(void) { return (2 << 16) | 4; }
+extern "C" int osd_abi_version(void) { return (2 << 16) | 5; }

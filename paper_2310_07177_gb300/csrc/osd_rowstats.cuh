@@ -29,35 +29,6 @@ inline int stats_slice_len(long long rows) {
     return rows >= 2048 ? 32768 : (rows >= 512 ? 16384 : 8192);
 }
 
-// Sentinel for vector slots past the end of a slice: -inf never raises a
-// maximum and adds 0 to a sum.
-template <typename In> struct NegInfRaw;
-template <> struct NegInfRaw<float> { static constexpr uint32_t bits = 0xFF800000u; };
-template <> struct NegInfRaw<__nv_bfloat16> { static constexpr uint32_t bits = 0xFF80FF80u; };
-
-template <typename In> __device__ __forceinline__ uint4 ninf_raw() {
-    return make_uint4(NegInfRaw<In>::bits, NegInfRaw<In>::bits, NegInfRaw<In>::bits, NegInfRaw<In>::bits);
-}
-// kW values of type In held in (the low bytes of) a 16-byte register block.
-template <typename In, int kW>
-__device__ __forceinline__ uint4 pack_raw(const float* v) {
-    if constexpr (kW == 1) {
-        return make_uint4(__float_as_uint(v[0]), 0u, 0u, 0u);
-    } else if constexpr (sizeof(In) == 4) {
-        return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]), __float_as_uint(v[3]));
-    } else {  // bf16: the values are exact bf16 numbers, so truncation keeps them
-        uint32_t w[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) w[i] = (__float_as_uint(v[2 * i]) >> 16) | (__float_as_uint(v[2 * i + 1]) & 0xffff0000u);
-        return make_uint4(w[0], w[1], w[2], w[3]);
-    }
-}
-template <typename In, int kW>
-__device__ __forceinline__ void unpack_raw(const uint4& r, float* v) {
-    if constexpr (kW == 1) v[0] = __uint_as_float(r.x);
-    else Elem<In>::unpack(r, v);
-}
-
 // ------------------------------------------------------------------ pass 1
 template <typename In, bool kGreedy>
 __global__ void __launch_bounds__(kStatThreads)

@@ -125,7 +125,7 @@ def test_argument_errors_return_before_any_launch(lib):
     assert fm(fake, fake, 1, 2, 16, 16, 16, fake, 0.5, 0.0, fake, None, None, None) == osd.OSD_ERR_INVALID_ARG
     assert fm(fake, fake, 1, 2, 16, 16, 16, None, 0.5, 1.0, fake, None, None, None) == osd.OSD_ERR_INVALID_ARG
     assert fm(fake, fake, 1, 2, 16, -16, 16, fake, 0.5, 1.0, fake, None, None, None) == osd.OSD_ERR_INVALID_ARG
-    assert fm(fake, fake, 1, 2, 500000, 0, 0, fake, 0.5, 1.0, fake, None, None, None) == osd.OSD_ERR_UNSUPPORTED
+    assert fm(fake, fake, 1, 2, (1 << 21) + 1, 0, 0, fake, 0.5, 1.0, fake, None, None, None) == osd.OSD_ERR_UNSUPPORTED
     assert fm(None, None, 1, 0, 16, 16, 16, None, 0.5, 1.0, None, None, None, None) == osd.OSD_OK
 
 

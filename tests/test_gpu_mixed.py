@@ -67,8 +67,10 @@ SHAPES = [  # (N, V, dtype)
     (6, 32128, torch.float32),
     (3, 128256, torch.bfloat16),
     (2, 65539, torch.float32),
-    (2, 393216, torch.bfloat16),   # the largest vocabulary per dtype
-    (2, 196608, torch.float32),
+    (1, 33001, torch.bfloat16),    # one row: 16-byte loads with a ragged last chunk
+    (1, 4099, torch.float32),
+    (2, 1 << 21, torch.bfloat16),  # the largest vocabulary
+    (2, 1 << 21, torch.float32),
 ]
 
 
@@ -99,6 +101,13 @@ def test_strided_and_broadcast_rows(osd):
     tok, _ = osd.osd_mixed_sample(big_z.to(dev)[:, 1], big_t.to(dev)[:, 2], u.to(dev), 0.3)
     torch.cuda.synchronize()
     ref, gap = oracle.mixed_sample(z, t, u, 0.3)
+    assert np.array_equal(tok.cpu().numpy()[gap >= TIE], ref[gap >= TIE])
+    # padded rows: 16-byte aligned strides around a ragged vocabulary of 5003
+    pz = torch.randn(6, 5008, generator=g).to(torch.bfloat16)
+    pt = torch.randn(6, 5008, generator=g).to(torch.bfloat16)
+    tok, _ = osd.osd_mixed_sample(pz.to(dev)[:, :5003], pt.to(dev)[:, :5003], u.to(dev), 0.6)
+    torch.cuda.synchronize()
+    ref, gap = oracle.mixed_sample(pz[:, :5003].contiguous(), pt[:, :5003].contiguous(), u, 0.6)
     assert np.array_equal(tok.cpu().numpy()[gap >= TIE], ref[gap >= TIE])
     # stride 0: one row repeated
     zr = z[:1].expand(6, -1)
@@ -144,7 +153,7 @@ def test_invalid_arguments_are_rejected(osd):
         with pytest.raises(osd.OsdError) as ei:
             osd.osd_mixed_sample(z, z, u, beta, temperature=tau)
         assert ei.value.status == osd.OSD_ERR_INVALID_ARG
-    big = torch.zeros(1, 500000, dtype=torch.bfloat16, device=dev)
+    big = torch.zeros(1, (1 << 21) + 1, dtype=torch.bfloat16, device=dev)
     with pytest.raises(osd.OsdError) as ei:
         osd.osd_mixed_sample(big, big, u[:1], 0.5)
     assert ei.value.status == osd.OSD_ERR_UNSUPPORTED
