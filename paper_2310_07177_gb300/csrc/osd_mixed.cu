@@ -39,14 +39,15 @@ struct MixParams {
     long long dstride, tstride;  // elements between consecutive rows
     const float* uniforms;
     float beta;
-    float c_hi, c_lo;  // log2(e) / tau as a float pair (c_lo > 0)
+    float c;  // log2(e) / tau, rounded to fp32
     int32_t* tokens;
     float* cdf_gap;
 };
 
-// Online max and sum of 2^((x - max) c) of both rows over one piece.
+// Online sums of both rows over one piece, each as (M, s) with M = rn(max c)
+// and s = sum 2^(x c - M).
 struct Piece {
-    float mt, st, mz, sz;
+    float Mt, st, Mz, sz;
 };
 
 template <typename In, bool kVecPath>
@@ -60,7 +61,7 @@ __global__ void __launch_bounds__(kMixThreads, 16) mixed_sample_kernel(MixParams
     const In* zrow = static_cast<const In*>(p.draft) + row * p.dstride;
     const In* trow = static_cast<const In*>(p.target) + row * p.tstride;
     const int V = p.V;
-    const float ch = p.c_hi, cl = p.c_lo;
+    const float c = p.c;
     // chunks of the row, the warp ranges and the runs (pieces) of steps in them
     const int nch = (V + kW - 1) / kW;
     const int rch = (nch + kMixWarps - 1) / kMixWarps;  // chunks per warp range
@@ -69,15 +70,15 @@ __global__ void __launch_bounds__(kMixThreads, 16) mixed_sample_kernel(MixParams
     auto range_lo = [&](int w) { return min(nch, w * rch); };
 
     // the kW raw entries of chunk c (past the row end they read as -inf)
-    auto load_chunk = [&](const In* rp, int c) -> uint4 {
+    auto load_chunk = [&](const In* rp, int ci) -> uint4 {
         if constexpr (kVecPath) {
-            if ((c + 1) * kW <= V) return ldg_stream(rp + size_t(c) * kW);
+            if ((ci + 1) * kW <= V) return ldg_stream(rp + size_t(ci) * kW);
             float v[kW];  // the ragged last chunk of the row
 #pragma unroll
-            for (int e = 0; e < kW; ++e) v[e] = (c * kW + e < V) ? E::load(rp + c * kW + e) : kNegInf;
+            for (int e = 0; e < kW; ++e) v[e] = (ci * kW + e < V) ? E::load(rp + ci * kW + e) : kNegInf;
             return pack_raw<In, kW>(v);
         } else {
-            float v[1] = {c < V ? E::load(rp + c) : kNegInf};
+            float v[1] = {ci < V ? E::load(rp + ci) : kNegInf};
             return pack_raw<In, 1>(v);
         }
     };
@@ -87,41 +88,44 @@ __global__ void __launch_bounds__(kMixThreads, 16) mixed_sample_kernel(MixParams
         if constexpr (kVecPath) return E::max_raw(r);
         else return __uint_as_float(r.x);
     };
-    // sum over the chunk of 2^((x - m) c), the exponent from the exact difference times c_hi + c_lo
-    auto chunk_sum = [&](const uint4& r, float m) {
+    // Exponent arguments are x c - M as one FMA, M = rn(m c): the FMA rounds
+    // once, after the cancellation, so the terms that carry the mass come out
+    // as exact as from the difference (x - m) c, and the rounding of M is a
+    // factor common to all the sums it scales.  Rescaling between two
+    // references is 2^(M - M'), a difference of two floats.
+    auto chunk_sum = [&](const uint4& r, float M) {
         float x[kW];
         unpack_raw<In, kW>(r, x);
         if constexpr (kW == 1) {
-            return ex2(mul_c(x[0] - m, ch, cl));
+            return ex2(fmaf(x[0], c, -M));
         } else {
             float2 s2 = f2(0.f);
 #pragma unroll
             for (int e = 0; e < kW; e += 2) {
-                const float2 d = sub2(make_float2(x[e], x[e + 1]), f2(m));
-                const float2 g = fma2(d, f2(ch), mul2(d, f2(cl)));
+                const float2 g = fma2(make_float2(x[e], x[e + 1]), f2(c), f2(-M));
                 s2 = add2(s2, make_float2(ex2(g.x), ex2(g.y)));
             }
             return s2.x + s2.y;
         }
     };
-    // one lane's running (max, sum) absorbs a chunk: rescale when the max rises
-    // (rarely, once the first chunks are in), then add; a lane that has seen
-    // only -inf keeps s = 0 and skips the sum
-    auto absorb = [&](float& m, float& s, const uint4& r) {
-        const float cm = chunk_max(r);
-        if (cm > m) {
-            s = (m == kNegInf) ? 0.f : s * ex2(mul_c(m - cm, ch, cl));
-            m = cm;
+    // one lane's running (reference M, sum s) absorbs a chunk: rescale when the
+    // reference rises (rarely, once the first chunks are in), then add; a lane
+    // that has seen only -inf keeps s = 0 and skips the sum
+    auto absorb = [&](float& M, float& s, const uint4& r) {
+        const float cM = __fmul_rn(chunk_max(r), c);
+        if (cM > M) {
+            s = (M == kNegInf) ? 0.f : s * ex2(M - cM);
+            M = cM;
         }
-        if (m != kNegInf) s += chunk_sum(r, m);
+        if (M != kNegInf) s += chunk_sum(r, M);
     };
-    // the warp's merge of every lane's (max, sum)
-    auto warp_merge = [&](float& m, float& s) {
-        float gm = m;
-        for (int o = 16; o > 0; o >>= 1) gm = fmaxf(gm, __shfl_xor_sync(0xffffffffu, gm, o));
-        s = (m == kNegInf) ? 0.f : s * ex2(mul_c(m - gm, ch, cl));
+    // the warp's merge of every lane's (M, s); M = -inf marks a lane without mass
+    auto warp_merge = [&](float& M, float& s) {
+        float gM = M;
+        for (int o = 16; o > 0; o >>= 1) gM = fmaxf(gM, __shfl_xor_sync(0xffffffffu, gM, o));
+        s = (M == kNegInf) ? 0.f : s * ex2(M - gM);
         for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-        m = gm;
+        M = gM;
     };
 
     // ---- pass: the warp's steps, one step of loads in flight ahead
@@ -134,7 +138,7 @@ __global__ void __launch_bounds__(kMixThreads, 16) mixed_sample_kernel(MixParams
             tc = load_chunk(trow, chunk_of(0));
         }
         for (int g = 0; g < kPieces; ++g) {
-            float mt = kNegInf, st_ = 0.f, mz = kNegInf, sz = 0.f;
+            float Mt = kNegInf, st_ = 0.f, Mz = kNegInf, sz = 0.f;
             const int s_end = min((g + 1) * per_piece, steps);
             for (int st = g * per_piece; st < s_end; ++st) {
                 uint4 zn = none, tn = none;
@@ -142,14 +146,14 @@ __global__ void __launch_bounds__(kMixThreads, 16) mixed_sample_kernel(MixParams
                     zn = load_chunk(zrow, chunk_of(st + 1));
                     tn = load_chunk(trow, chunk_of(st + 1));
                 }
-                absorb(mt, st_, tc);
-                absorb(mz, sz, zc);
+                absorb(Mt, st_, tc);
+                absorb(Mz, sz, zc);
                 zc = zn;
                 tc = tn;
             }
-            warp_merge(mt, st_);
-            warp_merge(mz, sz);
-            if (lane == 0) s_piece[warp * kPieces + g] = Piece{mt, st_, mz, sz};
+            warp_merge(Mt, st_);
+            warp_merge(Mz, sz);
+            if (lane == 0) s_piece[warp * kPieces + g] = Piece{Mt, st_, Mz, sz};
         }
     }
     __syncthreads();
@@ -157,20 +161,20 @@ __global__ void __launch_bounds__(kMixThreads, 16) mixed_sample_kernel(MixParams
 
     // ---- pick: lane l holds piece l (in vocabulary order)
     const Piece pc = s_piece[lane];
-    float gt = pc.mt, gz = pc.mz;
+    float Gt = pc.Mt, Gz = pc.Mz;  // rn(row max c): rounding is monotone, so the max of the M
     for (int o = 16; o > 0; o >>= 1) {
-        gt = fmaxf(gt, __shfl_xor_sync(0xffffffffu, gt, o));
-        gz = fmaxf(gz, __shfl_xor_sync(0xffffffffu, gz, o));
+        Gt = fmaxf(Gt, __shfl_xor_sync(0xffffffffu, Gt, o));
+        Gz = fmaxf(Gz, __shfl_xor_sync(0xffffffffu, Gz, o));
     }
-    // each piece's sums against the row maxima (a piece of -inf only has none)
-    const float rt = (pc.mt == kNegInf) ? 0.f : pc.st * ex2(mul_c(pc.mt - gt, ch, cl));
-    const float rz = (pc.mz == kNegInf) ? 0.f : pc.sz * ex2(mul_c(pc.mz - gz, ch, cl));
+    // each piece's sums against the row references (a piece of -inf only has none)
+    const float rt = (pc.Mt == kNegInf) ? 0.f : pc.st * ex2(pc.Mt - Gt);
+    const float rz = (pc.Mz == kNegInf) ? 0.f : pc.sz * ex2(pc.Mz - Gz);
     float Et = rt, Ez = rz;
     for (int o = 16; o > 0; o >>= 1) {
         Et += __shfl_xor_sync(0xffffffffu, Et, o);
         Ez += __shfl_xor_sync(0xffffffffu, Ez, o);
     }
-    // weights w_j = a 2^((t_j - m_t)c) + b 2^((z_j - m_z)c) against the row maxima
+    // weights w_j = a 2^(t_j c - G_t) + b 2^(z_j c - G_z) against the row references
     const float a = (Et > 0.f) ? p.beta / Et : 0.f;
     const float b = (Ez > 0.f) ? (1.f - p.beta) / Ez : 0.f;
     const double mass = double(a) * double(rt) + double(b) * double(rz);
@@ -188,7 +192,8 @@ __global__ void __launch_bounds__(kMixThreads, 16) mixed_sample_kernel(MixParams
         const unsigned pos = __ballot_sync(0xffffffffu, mass > 0.0);
         piece = pos ? 31 - __clz(pos) : 0;
     }
-    const float gt_ref = (gt == kNegInf) ? 0.f : gt, gz_ref = (gz == kNegInf) ? 0.f : gz;
+    // a row without mass: its logits are -inf, and so are x c - 0
+    const float Gt_ref = (Gt == kNegInf) ? 0.f : Gt, Gz_ref = (Gz == kNegInf) ? 0.f : Gz;
     const int pw = piece / kPieces, pg = piece % kPieces;
     const int c0 = range_lo(pw), c1 = range_lo(pw + 1);
     const int s_end = min((pg + 1) * per_piece, steps);
@@ -196,16 +201,16 @@ __global__ void __launch_bounds__(kMixThreads, 16) mixed_sample_kernel(MixParams
     double gap = 0.0;
     bool found = false;
     for (int st = pg * per_piece; st < s_end; ++st) {  // warp-uniform trip count
-        const int c = c0 + st * 32 + lane;
+        const int ci = c0 + st * 32 + lane;
         float z[kW], t[kW], w[kW];
-        unpack_raw<In, kW>(c < c1 ? load_chunk(zrow, c) : none, z);
-        unpack_raw<In, kW>(c < c1 ? load_chunk(trow, c) : none, t);
+        unpack_raw<In, kW>(ci < c1 ? load_chunk(zrow, ci) : none, z);
+        unpack_raw<In, kW>(ci < c1 ? load_chunk(trow, ci) : none, t);
 #pragma unroll
         for (int e = 0; e < kW; ++e) {
-            const float pt = ex2(mul_c(t[e] - gt_ref, ch, cl));
-            const float qz = ex2(mul_c(z[e] - gz_ref, ch, cl));
+            const float pt = ex2(fmaf(t[e], c, -Gt_ref));
+            const float qz = ex2(fmaf(z[e], c, -Gz_ref));
             w[e] = fmaf(a, pt, b * qz);
-            if (w[e] > 0.f) last_pos = c * kW + e;
+            if (w[e] > 0.f) last_pos = ci * kW + e;
         }
         double mine = 0.0;
 #pragma unroll
@@ -221,7 +226,7 @@ __global__ void __launch_bounds__(kMixThreads, 16) mixed_sample_kernel(MixParams
                         const double Cprev = C;
                         C += double(w[e]);
                         if (C > tau) {
-                            pick = c * kW + e;
+                            pick = ci * kW + e;
                             gap = fmin(C - tau, tau - Cprev) / W;
                             break;
                         }
@@ -286,7 +291,7 @@ extern "C" osd_status osd_mixed_sample(const void* draft_logits, const void* tar
     mp.tstride = t_stride;
     mp.uniforms = uniforms;
     mp.beta = beta;
-    split_scale(temperature, &mp.c_hi, &mp.c_lo);
+    mp.c = static_cast<float>(1.4426950408889634074 / static_cast<double>(temperature));
     mp.tokens = tokens;
     mp.cdf_gap = cdf_gap;
     const dim3 grid(static_cast<unsigned>(N)), block(kMixThreads);
