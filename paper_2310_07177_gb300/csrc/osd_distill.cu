@@ -220,6 +220,8 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     constexpr bool kMoment = kKind == OSD_FKL || kKind == OSD_RKL;
     constexpr bool kNeedEt = kKind != OSD_CE;  // CE needs only the draft normaliser and the label
     constexpr bool kFold = !kClamp;            // exponent arguments by one FMA (see pass 1)
+    // chunk loops unrolled by two where that measured faster (TVD, JSD, CE: +2-3 %; FKL, RKL: -1 %)
+    constexpr int kUn = (kKind == OSD_FKL || kKind == OSD_RKL) ? 1 : 2;
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ __align__(8) uint64_t bar;
     __shared__ Stats1 s1_mine, s1_all;
@@ -286,7 +288,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     float mz = kNegInf, mt = kNegInf;
     int jz = -1, jt = -1;
     if (!err_local) {
-        sweep<In, kAligned, kClampZ, kClampT, true>(zs, ts, n, [&](const float* z, const float* t, auto tag,
+        sweep<In, kAligned, kClampZ, kClampT, true, false, kUn>(zs, ts, n, [&](const float* z, const float* t, auto tag,
                                                                    int j0, float cz, float ct, bool,
                                                                    const uint4& zr, const uint4& tr) {
             if (cz > mz) { mz = cz; jz = j0; }
@@ -362,7 +364,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     if (!err_local) {
         const float2 gz2 = f2(gzb), gt2 = f2(gtb), tp2 = f2(tpv);
         const float2 nMz2 = f2(-Mz), nMt2 = f2(-Mt);
-        sweep<In, kAligned, false, false, false, kMoment>(zs, ts, n, [&](const float* z, const float* t,
+        sweep<In, kAligned, false, false, false, kMoment, kUn>(zs, ts, n, [&](const float* z, const float* t,
                                                                              auto tag, int, float, float,
                                                                              bool ninf, const uint4&, const uint4&) {
             constexpr int kCnt = decltype(tag)::value;
@@ -522,8 +524,9 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         // ---- pass 2: divergence terms with the global normalisers
         float2 A2 = f2(0.f), B2 = f2(0.f), C2 = f2(0.f);
         if (!row_err && !jsd_trivial) {
-            sweep<In, kAligned, false, false, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
-                                                                    int j0, float, float, bool, const uint4& zr, const uint4& tr) {
+            sweep<In, kAligned, false, false, false, false, kUn>(zs, ts, n, [&](const float* z, const float* t,
+                                                                               auto tag, int j0, float, float, bool,
+                                                                               const uint4& zr, const uint4& tr) {
                 constexpr int kCnt = decltype(tag)::value;
                 // TVD's bf16 chunks: x - m straight from the packed words the sweep loaded
                 // (measured, JSD does as well unpacking)
@@ -632,8 +635,9 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         // q and p of this pass come out multiplied by the gradient's constant factor
         const float2 cvs = f2(cv + p.lg_scale), cus = f2(cu + p.lg_scale);
         const int label = st.idx;
-        sweep<In, kAligned, false, false, false>(zs, ts, n, [&](const float* z, const float* t, auto tag,
-                                                                int j0, float, float, bool, const uint4& zr, const uint4& tr) {
+        sweep<In, kAligned, false, false, false, false, kUn>(zs, ts, n, [&](const float* z, const float* t,
+                                                                           auto tag, int j0, float, float, bool,
+                                                                           const uint4& zr, const uint4& tr) {
             constexpr int kCnt = decltype(tag)::value;
             // bf16 chunks of FKL/RKL, which need x - m of both rows, take the differences straight
             // from the packed words (mixed-precision subtracts) instead of unpacking first;

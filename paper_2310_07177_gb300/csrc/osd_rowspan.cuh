@@ -64,15 +64,19 @@ __device__ __forceinline__ int stage_span(In* zs, In* ts, const In* zsrc, const 
 // (or single entries on the element-wise path).  Clamping (to -1e30, see Elem)
 // happens on the packed words.  f(z[], t[], count_tag, j0, zmax, tmax, ninf,
 // zraw, traw) gets the chunk maxima when kMax is set, ninf = "the chunk holds a
-// -inf" when kMin is set, and the (clamped) packed words of a full chunk.  Chunk v goes to thread v mod kRowThreads, so warp w sees
-// the 32-chunk groups w, w + kRowWarps, ... in order.
-template <typename In, bool kAligned, bool kClampZ, bool kClampT, bool kMax, bool kMin = false, typename F>
+// -inf" when kMin is set, and the (clamped) packed words of a full chunk.
+// Chunk v goes to thread v mod kRowThreads, so warp w sees the 32-chunk groups
+// w, w + kRowWarps, ... in order.  kUnroll unrolls the chunk loop (two chunks
+// a trip halve the loop overhead, at some registers).
+template <typename In, bool kAligned, bool kClampZ, bool kClampT, bool kMax, bool kMin = false, int kUnroll = 1,
+          typename F>
 __device__ __forceinline__ void sweep(const In* zs, const In* ts, int n, F&& f) {
     using E = Elem<In>;
     constexpr int kVec = E::kVec;
     const int tid = threadIdx.x;
     if constexpr (kAligned) {
         const int nv = n / kVec;
+#pragma unroll kUnroll
         for (int v = tid; v < nv; v += kRowThreads) {
             uint4 zr = lds_v4(zs + v * kVec), tr = lds_v4(ts + v * kVec);
             if (kClampZ) E::clamp_raw(zr);
