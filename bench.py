@@ -88,6 +88,7 @@ class ClockSampler:
         self.gpu_id = gpu_id
         self.proc = None
         self.lines = []
+        self.first = 0
 
     def __enter__(self):
         try:
@@ -104,6 +105,22 @@ class ClockSampler:
         for line in self.proc.stdout:
             self.lines.append(line.strip())
 
+    def wait_lines(self, n: int, timeout_s: float) -> None:
+        """Wait (bounded) until at least n sample lines have arrived."""
+        t_end = time.perf_counter() + timeout_s
+        while self.proc is not None and len(self.lines) < n and time.perf_counter() < t_end:
+            time.sleep(0.002)
+
+    def start_region(self) -> None:
+        """Mark the start of the timed region once the sampler is running: keep
+        the sample just before it, so that a region shorter than the sampling
+        period still has the clocks on both sides of it."""
+        self.wait_lines(1, 3.0)
+        self.first = max(0, len(self.lines) - 1)
+
+    def end_region(self) -> None:
+        self.wait_lines(len(self.lines) + 1, 1.0)  # and the sample just after it
+
     def __exit__(self, *exc):
         if self.proc is not None:
             self.proc.terminate()
@@ -115,7 +132,7 @@ class ClockSampler:
     def summary(self):
         sm, mx, reasons = [], None, set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in self.lines:
+        for line in self.lines[self.first:]:
             parts = [p.strip() for p in line.split(",")]
             if len(parts) < 7:
                 continue
@@ -266,11 +283,13 @@ def run_ours(args):
         torch.distributed.barrier()
     torch.cuda.synchronize()
     with ClockSampler(gpu_id) as clk:
+        clk.start_region()
         t0 = time.perf_counter()
         for _ in range(args.steps):
             step(recs)
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
+        clk.end_region()
     if world > 1:
         torch.distributed.barrier()
 

@@ -36,11 +36,14 @@ constexpr int kTreeThreads = 128;
 constexpr int kTreeWarps = kTreeThreads / 32;
 constexpr int kTreeMaxCluster = 8;
 constexpr int kTreeMaxSub = 8192;  // sub-tiles of one CTA's vocabulary span
+constexpr int kTreeUnroll = 4;     // sub-tiles of loads in flight per warp in a mass pass
 
-// Children lists of the static tree: first child and next sibling, increasing index.
+// Children lists of the static tree: first child and next sibling, increasing
+// index; and each node's parent (-1 at the root).
 struct TreeTopo {
     int8_t first_child[OSD_TREE_MAX_NODES];
     int8_t next_sibling[OSD_TREE_MAX_NODES];
+    int8_t parent[OSD_TREE_MAX_NODES];
 };
 
 struct TreeParams {
@@ -72,8 +75,13 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
     __shared__ double s_span_total;            // read by the other CTAs of the cluster
     __shared__ double s_cta_incl[kTreeMaxCluster];  // inclusive prefix of the CTA masses, rank order
     __shared__ double s_W;
-    __shared__ float s_mt, s_st, s_mz, s_sz;
-    __shared__ int s_idx, s_next, s_extra;
+    __shared__ int s_next, s_extra;
+    // per node: merged statistics of its target (0) and draft (1) rows, or the target argmax at T = 0
+    __shared__ float s_nm[2][OSD_TREE_MAX_NODES], s_ns[2][OSD_TREE_MAX_NODES];
+    __shared__ int s_nidx[OSD_TREE_MAX_NODES];
+    // per child c: its token's logits in the draft and target rows of its parent, and its uniform
+    __shared__ float s_zy[OSD_TREE_MAX_NODES], s_ty[OSD_TREE_MAX_NODES], s_u[OSD_TREE_MAX_NODES];
+    __shared__ double s_nratio[OSD_TREE_MAX_NODES];  // per node with children: E_z / E_t
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int csize = p.csize;
@@ -87,9 +95,21 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
     int32_t* out = p.out_tokens + size_t(b) * n;
     const float ch = p.c_hi, cl = p.c_lo;
 
+    // Prologue, before the statistics are ready: check the tokens and gather the two
+    // logits every child's accept test needs, all in one round of loads.
     int bad = 0;
-    for (int i = 1 + tid; i < n; i += kTreeThreads)
-        if (y[i] < 0 || y[i] >= V) bad = 1;
+    if (!greedy)
+        for (int i = tid; i < n; i += kTreeThreads) s_u[i] = u[i];
+    for (int i = 1 + tid; i < n; i += kTreeThreads) {
+        const int yi = y[i];
+        if (yi < 0 || yi >= V) {
+            bad = 1;
+        } else if (!greedy) {
+            const size_t prow = size_t(b) * n + p.topo.parent[i];
+            s_zy[i] = E::load(static_cast<const In*>(p.draft) + prow * V + yi);
+            s_ty[i] = E::load(static_cast<const In*>(p.target) + prow * V + yi);
+        }
+    }
     bad = __syncthreads_or(bad);
     if (rank == 0) {
         for (int i = tid; i < n; i += kTreeThreads) {
@@ -106,6 +126,37 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
     if (bad) return;  // uniform over the cluster, before any shared-memory exchange
     __syncthreads();  // the initialisation above lands before the walk writes its entries
     grid_dependency_wait();  // the row statistics are complete from here on
+
+    // Every node's row statistics, merged from their slices up front (one thread per
+    // node and row, all loads in one round) instead of one dependent round per node
+    // on the walk.  Draft rows matter only where children are tested.
+    for (int t = tid; t < 2 * n; t += kTreeThreads) {
+        const int nd = t >> 1, which = t & 1;
+        if (greedy) {
+            if (which == 0) {
+                const RowStat* st = p.stats + (size_t(b) * n + nd) * p.n_slices;
+                MaxIdx acc{kNegInf, INT_MAX};
+#pragma unroll 4
+                for (int sl = 0; sl < p.n_slices; ++sl) acc = merge_mi(acc, MaxIdx{st[sl].m, st[sl].idx});
+                s_nidx[nd] = (acc.i == INT_MAX) ? 0 : acc.i;
+            }
+        } else if (which == 0 || p.topo.first_child[nd] >= 0) {
+            const RowStat* st = p.stats + ((which == 0 ? p.n_draft_rows : 0) + size_t(b) * n + nd) * p.n_slices;
+            MaxSum acc{kNegInf, 0.f};
+#pragma unroll 4
+            for (int sl = 0; sl < p.n_slices; ++sl) acc = merge_ms(acc, MaxSum{st[sl].m, st[sl].s}, ch, cl);
+            s_nm[which][nd] = acc.m;
+            s_ns[which][nd] = acc.s;
+        }
+    }
+    __syncthreads();
+    // the sum ratio of each accept test's p/q, once per node (fp64 divisions are slow here)
+    if (!greedy) {
+        for (int nd = tid; nd < n; nd += kTreeThreads)
+            if (p.topo.first_child[nd] >= 0) s_nratio[nd] = double(s_ns[1][nd]) / double(s_ns[0][nd]);
+        __syncthreads();
+    }
+    float cur_mt = 0.f, cur_st = 1.f, cur_mz = 0.f, cur_sz = 1.f;  // the current node's statistics
 
     const int e0 = rank * p.span;
     const int cnt = max(0, min(p.span, V - e0));
@@ -134,11 +185,11 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
         }
     };
     auto weights = [&](const Raw& r, bool use_q, float s, float* w) {
-        const float mt = s_mt, inv_st = 1.0f / s_st;
+        const float mt = cur_mt, inv_st = 1.0f / cur_st;
         float tv[kW], zv[kW];
         unpack_raw<In, kW>(r.t, tv);
         unpack_raw<In, kW>(r.z, zv);
-        const float mz = s_mz, inv_sz = use_q ? 1.0f / s_sz : 0.f;
+        const float mz = cur_mz, inv_sz = use_q ? 1.0f / cur_sz : 0.f;
 #pragma unroll
         for (int e = 0; e < kW; ++e) {
             const float pj = ex2(mul_c(tv[e] - mt, ch, cl)) * inv_st;
@@ -154,16 +205,24 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
     // the CTA masses' inclusive prefix into s_cta_incl, and the row's mass W (returned).
     auto mass_pass = [&](const In* trow, const In* zrow, bool use_q, float s) -> double {
         if (pending) cluster_wait();  // every peer has read the previous pass's total
-        for (int sb = warp; sb < nsub; sb += kTreeWarps) {
-            Raw r;
-            load_sub(trow, zrow, use_q, sb, r);
-            float w[kW];
-            weights(r, use_q, s, w);
-            float sum = 0.f;
+        for (int sb0 = warp; sb0 < nsub; sb0 += kTreeWarps * kTreeUnroll) {
+            Raw r[kTreeUnroll];  // the loads of kTreeUnroll sub-tiles go out together
 #pragma unroll
-            for (int e = 0; e < kW; ++e) sum += w[e];
-            for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-            if (lane == 0) s_sub[sb] = sum;
+            for (int u2 = 0; u2 < kTreeUnroll; ++u2)
+                if (sb0 + u2 * kTreeWarps < nsub) load_sub(trow, zrow, use_q, sb0 + u2 * kTreeWarps, r[u2]);
+#pragma unroll
+            for (int u2 = 0; u2 < kTreeUnroll; ++u2) {
+                const int sb = sb0 + u2 * kTreeWarps;
+                if (sb < nsub) {
+                    float w[kW];
+                    weights(r[u2], use_q, s, w);
+                    float sum = 0.f;
+#pragma unroll
+                    for (int e = 0; e < kW; ++e) sum += w[e];
+                    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+                    if (lane == 0) s_sub[sb] = sum;
+                }
+            }
         }
         __syncthreads();
         if (warp == 0) {
@@ -194,37 +253,16 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
         const In* zrow = static_cast<const In*>(p.draft) + (size_t(b) * n + node) * V;
         const bool has_child = p.topo.first_child[node] >= 0;
         const bool need_q = !greedy && has_child;
-        // statistics of the node's rows, merged from their slices by warp 0
-        if (warp == 0) {
-            const RowStat* ts = p.stats + (p.n_draft_rows + size_t(b) * n + node) * p.n_slices;
-            if (greedy) {
-                MaxIdx acc{kNegInf, INT_MAX};
-                for (int sl = lane; sl < p.n_slices; sl += 32) acc = merge_mi(acc, MaxIdx{ts[sl].m, ts[sl].idx});
-                acc = warp_reduce(acc, [](MaxIdx x, MaxIdx z) { return merge_mi(x, z); });
-                if (lane == 0) s_idx = (acc.i == INT_MAX) ? 0 : acc.i;
-            } else {
-                auto merge = [ch, cl](MaxSum x, MaxSum z) { return merge_ms(x, z, ch, cl); };
-                MaxSum at{kNegInf, 0.f}, az{kNegInf, 0.f};
-                const RowStat* zs = p.stats + (size_t(b) * n + node) * p.n_slices;
-                for (int sl = lane; sl < p.n_slices; sl += 32) {
-                    at = merge(at, MaxSum{ts[sl].m, ts[sl].s});
-                    if (need_q) az = merge(az, MaxSum{zs[sl].m, zs[sl].s});
-                }
-                at = warp_reduce(at, merge);
-                az = warp_reduce(az, merge);
-                if (lane == 0) {
-                    s_mt = at.m;
-                    s_st = at.s;
-                    s_mz = az.m;
-                    s_sz = az.s;
-                }
-            }
+        cur_mt = s_nm[0][node];
+        cur_st = s_ns[0][node];
+        if (need_q) {
+            cur_mz = s_nm[1][node];
+            cur_sz = s_ns[1][node];
         }
-        __syncthreads();
 
         int next = -1;
         if (greedy) {
-            const int best = s_idx;
+            const int best = s_nidx[node];
             for (int c = p.topo.first_child[node]; c >= 0; c = p.topo.next_sibling[c])
                 if (y[c] == best) { next = c; break; }
             if (next < 0) {
@@ -237,20 +275,21 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
             bool passed = false;  // a mass pass of the current residual has run
             for (int c = p.topo.first_child[node]; c >= 0; c = p.topo.next_sibling[c]) {
                 if (tid == 0) {
-                    // p(y)/q(y) from the logit differences and the two sums, as the verifier forms it
-                    const int yc = y[c];
-                    const float zt = E::load(zrow + yc), tt = E::load(trow + yc);
-                    double r;
+                    // p(y)/q(y) from the logit differences and the two sums, as the verifier
+                    // forms it; the test u < max(0, p/q - s) / N is taken as u N < max(0, p/q - s)
+                    const float zt = s_zy[c], tt = s_ty[c];
+                    double rn;  // max(0, p(y)/q(y) - s_j)
                     if (zt == kNegInf) {
-                        r = (tt > kNegInf) ? INFINITY : 0.0;
+                        rn = (tt > kNegInf) ? INFINITY : 0.0;
                     } else {
-                        const float D = (tt - s_mt) - (zt - s_mz);
-                        const double rho = double(ex2(mul_c(D, ch, cl))) * (double(s_sz) / double(s_st));
-                        r = fmax(rho - double(s), 0.0) / N;
+                        const float D = (tt - cur_mt) - (zt - cur_mz);
+                        const double rho = double(ex2(mul_c(D, ch, cl))) * s_nratio[node];
+                        rn = fmax(rho - double(s), 0.0);
                     }
-                    const float uc = u[c];
-                    if (rank == 0 && p.diag_margin) p.diag_margin[size_t(b) * n + c] = float(fabs(double(uc) - r));
-                    s_next = (double(uc) < r) ? c : -1;
+                    const float uc = s_u[c];
+                    if (rank == 0 && p.diag_margin)  // |u - r|, a diagnostic: fp32 is enough
+                        p.diag_margin[size_t(b) * n + c] = fabsf(uc - float(rn) / float(N));
+                    s_next = (double(uc) * N < rn) ? c : -1;
                 }
                 __syncthreads();
                 next = s_next;
@@ -264,7 +303,7 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
                 // ---- the extra token from w = max(0, p - s q) (p itself when nothing was rejected)
                 const bool use_q = passed;
                 const double W = passed ? N : mass_pass(trow, zrow, false, 0.f);
-                const double tau = double(u[0]) * W;
+                const double tau = double(s_u[0]) * W;
                 int owner = -1, mode = 0;  // mode 0: inverse CDF, 1: largest positive entry, 2: argmax p
                 double base = 0.0;
                 if (W > 0.0) {
@@ -414,9 +453,11 @@ static bool tree_topology(const int32_t* parent, int n, TreeTopo* topo) {
     }
     int8_t last_child[OSD_TREE_MAX_NODES];
     for (int i = 0; i < OSD_TREE_MAX_NODES; ++i) last_child[i] = -1;
+    for (int i = 0; i < OSD_TREE_MAX_NODES; ++i) topo->parent[i] = -1;
     for (int i = 1; i < n; ++i) {
         const int par = parent[i];
         if (par < 0 || par >= i) return false;
+        topo->parent[i] = static_cast<int8_t>(par);
         if (last_child[par] < 0) topo->first_child[par] = static_cast<int8_t>(i);
         else topo->next_sibling[last_child[par]] = static_cast<int8_t>(i);
         last_child[par] = static_cast<int8_t>(i);
