@@ -441,9 +441,13 @@ static int verify_slices(int B, int k, int V) {
     return (V + len - 1) / len;
 }
 
-static void finalize_shape(int V, int* csize, int* span) {
+// CTAs per sequence: up to 8 for few sequences (short spans, low latency); 4 past
+// 128 sequences, where 8 would leave more clusters than fit on the GPU at once and
+// the second wave would wait out the first one's latency phases.
+static void finalize_shape(int B, int V, int* csize, int* span) {
+    const int cmax = (B > 128) ? kFinMaxCluster / 2 : kFinMaxCluster;
     int c = (V + 4095) / 4096;
-    c = c < 1 ? 1 : (c > kFinMaxCluster ? kFinMaxCluster : c);
+    c = c < 1 ? 1 : (c > cmax ? cmax : c);
     int s = (V + c - 1) / c;
     s = (s + 63) / 64 * 64;
     c = (V + s - 1) / s;
@@ -485,7 +489,7 @@ static osd_status launch_verify(const void* draft, const void* target, int B, in
     fp.accepted = accepted; fp.out_tokens = out_tokens; fp.mask = mask;
     fp.diag_margin = diag_margin; fp.diag_gap = diag_gap;
     int csize = 1, span = V;
-    if (!greedy) finalize_shape(V, &csize, &span);
+    if (!greedy) finalize_shape(B, V, &csize, &span);
     fp.csize = csize;
     fp.span = span;
     const bool vec = !greedy && aligned_to(draft, 16) && aligned_to(target, 16) &&

@@ -53,6 +53,8 @@ CASES = [  # (B, k, V, dtype, T)
     (512, 4, 16, torch.bfloat16, 1.0),       # many sequences over a tiny vocabulary
     (1024, 8, 64, torch.float32, 0.7),
     (16, 64, 300, torch.bfloat16, 1.0),      # the largest k
+    (160, 2, 20000, torch.bfloat16, 1.0),    # past 128 sequences: 4 finalize CTAs per sequence
+    (130, 3, 40961, torch.float32, 0.7),     # the same, element-wise path
     (2, 3, 1 << 21, torch.bfloat16, 1.0),    # the largest vocabulary
 ]
 
