@@ -33,6 +33,7 @@ namespace osd {
 constexpr int kDistThreads = kRowThreads;
 constexpr int kDistMaxCluster = 8;
 constexpr int kDistSpanBytes = 32768;         // target bytes of both rows per CTA
+constexpr int kDistSpanBytesJsd = 49152;      // JSD, bound by its ex2/lg2 work, does best with fewer, longer spans
 constexpr int kDistMaxSmem = 192 * 1024;      // largest staging buffer per CTA
 
 struct DistParams {
@@ -763,7 +764,8 @@ static osd_status distill_run(const void* draft_logits, const void* target_logit
     if (kind == OSD_JSD && !(beta >= 0.f && beta <= 1.f)) return OSD_ERR_INVALID_ARG;
     const size_t es = dtype_size(dtype);
     int csize = 1, span = V;
-    if (!row_span_shape(V, es, kDistSpanBytes, kDistMaxCluster, kDistMaxSmem, &csize, &span))
+    const size_t span_bytes = (kind == OSD_JSD) ? kDistSpanBytesJsd : kDistSpanBytes;
+    if (!row_span_shape(V, es, span_bytes, kDistMaxCluster, kDistMaxSmem, &csize, &span))
         return OSD_ERR_UNSUPPORTED;
     const long long rows = static_cast<long long>(G) * P;
     if (rows * csize > INT_MAX) return OSD_ERR_UNSUPPORTED;
