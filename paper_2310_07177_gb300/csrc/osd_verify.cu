@@ -9,14 +9,18 @@
 //                       exp((x - max)/T) of the slice (or the argmax for T = 0).
 //                       This pass reads every logit once and carries almost all
 //                       of the operation's HBM traffic.
-//   verify_finalize     one thread-block cluster per sequence: merges the slice
-//                       statistics, runs the k accept tests u_i < p_i(y_i)/q_i(y_i)
-//                       in order, then draws the extra token from
+//   verify_finalize     (T > 0) one thread-block cluster per sequence: merges the slice
+//                       statistics, runs the k accept tests u_i < p_i(y_i)/q_i(y_i),
+//                       all at once (a is the first failure), then draws the extra token from
 //                       norm(max(0, p_a - q_a)) (or p_k when all k pass) by inverse
 //                       CDF.  Each CTA of the cluster sums the residual weights of
 //                       its part of the vocabulary per tile; the partial sums meet
 //                       through distributed shared memory and the CTA whose part
 //                       holds u*W rescans that one tile with an fp64 block scan.
+//
+//   verify_greedy       (T = 0) one warp per sequence: the argmax of every target
+//                       row from its slices, the matches in order, the target
+//                       argmax at the first mismatch.
 //
 // The log-ratio of the accept test is formed from differences of raw logits and
 // maxima, (t_y - m_t) - (z_y - m_z), and the ratio of the two sums, so no
@@ -59,6 +63,70 @@ struct FinParams {
 };
 
 
+// T = 0: the accept tests are argmax matches, and the extra token is the target
+// argmax at the first mismatch.  One warp per sequence, a small kernel of its
+// own: at serving batch sizes this pass is latency-bound, and a compact kernel
+// starts faster than the sampling kernel with its greedy branch would.
+constexpr int kGreedyWarps = 4;
+__global__ void __launch_bounds__(kGreedyWarps * 32) verify_greedy_kernel(FinParams p) {
+    const int lane = threadIdx.x & 31;
+    const int b = blockIdx.x * kGreedyWarps + (threadIdx.x >> 5);
+    if (b >= p.B) return;
+    const int k = p.k, V = p.V;
+    const int32_t* y = p.tokens + size_t(b) * k;
+    // the draft tokens before the statistics are needed (one round of loads)
+    constexpr int kC = (OSD_VERIFY_MAX_K + 1 + 31) / 32;
+    int yv[kC];
+    bool bad = false;
+#pragma unroll
+    for (int c = 0; c < kC; ++c) {
+        const int i = c * 32 + lane;
+        yv[c] = (i < k) ? y[i] : 0;
+        bad |= (i < k) && (yv[c] < 0 || yv[c] >= V);
+    }
+    grid_dependency_wait();  // the row statistics are complete from here on
+    // row i <= k of the sequence: its target argmax, lowest index on ties, merged
+    // from the slices by the lane that owns the row
+    int idx[kC];
+    unsigned fail = 0;
+    int a = k;
+#pragma unroll
+    for (int c = 0; c < kC; ++c) {
+        const int i = c * 32 + lane;
+        idx[c] = 0;
+        if (i <= k) {
+            const RowStat* st = p.stats + ((long long)b * (k + 1) + i) * p.n_slices;
+            MaxIdx acc{kNegInf, INT_MAX};
+            for (int sl = 0; sl < p.n_slices; ++sl) acc = merge_mi(acc, MaxIdx{st[sl].m, st[sl].idx});
+            idx[c] = (acc.i == INT_MAX) ? 0 : acc.i;
+        }
+        fail = __ballot_sync(0xffffffffu, i < k && yv[c] != idx[c]);
+        if (fail && a == k) a = c * 32 + __ffs(fail) - 1;
+    }
+    bad = __any_sync(0xffffffffu, bad);
+    int32_t* out = p.out_tokens + size_t(b) * (k + 1);
+    if (lane == 0) {
+        p.accepted[b] = bad ? -1 : a;
+        if (p.diag_gap) p.diag_gap[b] = __int_as_float(0x7fc00000);
+    }
+    // the token at a is the target argmax there, held by lane a % 32 in slot a / 32
+    int at = 0;
+#pragma unroll
+    for (int c = 0; c < kC; ++c) {
+        const int v = __shfl_sync(0xffffffffu, idx[c], a & 31);
+        if (c == a / 32) at = v;
+    }
+#pragma unroll
+    for (int c = 0; c < kC; ++c) {
+        const int i = c * 32 + lane;
+        if (i <= k) out[i] = bad ? -1 : (i < a ? yv[c] : (i == a ? at : -1));
+        if (i < k) {
+            p.mask[size_t(b) * k + i] = (!bad && i == a) ? 1 : 0;
+            if (p.diag_margin) p.diag_margin[size_t(b) * k + i] = __int_as_float(0x7fc00000);
+        }
+    }
+}
+
 template <typename In, bool kVecPath>
 __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams p) {
     using E = Elem<In>;
@@ -68,7 +136,6 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
 
     __shared__ float s_m[2 * OSD_VERIFY_MAX_K + 1];
     __shared__ float s_s[2 * OSD_VERIFY_MAX_K + 1];
-    __shared__ int s_idx[OSD_VERIFY_MAX_K + 1];
     __shared__ float s_zy[OSD_VERIFY_MAX_K], s_ty[OSD_VERIFY_MAX_K];
     __shared__ int s_y[OSD_VERIFY_MAX_K];
     __shared__ float s_u[OSD_VERIFY_MAX_K + 1];
@@ -81,7 +148,6 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
     const int rank = (p.csize > 1) ? static_cast<int>(cluster_rank()) : 0;
     const int b = blockIdx.x / p.csize;
     const int k = p.k, V = p.V;
-    const bool greedy = (p.T == 0.f);
     const int32_t* y = p.tokens + size_t(b) * k;
     const In* draft = static_cast<const In*>(p.draft);
     const In* target = static_cast<const In*>(p.target);
@@ -98,16 +164,16 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
             s_y[i] = t;
             if (t < 0 || t >= V) {
                 bad = 1;
-            } else if (!greedy) {
+            } else {
                 s_zy[i] = E::load(draft + (size_t(b) * k + i) * V + t);
                 s_ty[i] = E::load(target + (size_t(b) * (k + 1) + i) * V + t);
             }
         }
     }
-    if (!greedy && warp == kWarps - 2)
+    if (warp == kWarps - 2)
         for (int i = lane; i <= k; i += 32) s_u[i] = p.uniforms[size_t(b) * (k + 1) + i];
     grid_dependency_wait();  // the row statistics are complete from here on
-    const int nrows = greedy ? (k + 1) : (2 * k + 1);
+    const int nrows = 2 * k + 1;
     const float ch0 = p.c_hi, cl0 = p.c_lo;
     auto srow_of = [&](int r) -> long long {
         return (r <= k) ? (p.n_draft_rows + (long long)b * (k + 1) + r) : ((long long)b * k + (r - k - 1));
@@ -126,20 +192,12 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
             const int r = r0 + q * kWarps;
             if (r >= nrows) break;  // uniform across the warp
             const RowStat* st = p.stats + srow_of(r) * p.n_slices;
-            if (greedy) {
-                MaxIdx acc{kNegInf, INT_MAX};
-                if (have[q]) acc = MaxIdx{part[q][0].m, part[q][0].idx};
-                for (int sl = lane + 32; sl < p.n_slices; sl += 32) acc = merge_mi(acc, MaxIdx{st[sl].m, st[sl].idx});
-                acc = warp_reduce(acc, [](MaxIdx x, MaxIdx z) { return merge_mi(x, z); });
-                if (lane == 0) { s_m[r] = acc.m; s_idx[r] = (acc.i == INT_MAX) ? 0 : acc.i; }
-            } else {
-                auto merge = [ch0, cl0](MaxSum x, MaxSum z) { return merge_ms(x, z, ch0, cl0); };
-                MaxSum acc{kNegInf, 0.f};
-                if (have[q]) acc = MaxSum{part[q][0].m, part[q][0].s};
-                for (int sl = lane + 32; sl < p.n_slices; sl += 32) acc = merge(acc, MaxSum{st[sl].m, st[sl].s});
-                acc = warp_reduce(acc, merge);
-                if (lane == 0) { s_m[r] = acc.m; s_s[r] = acc.s; }
-            }
+            auto merge = [ch0, cl0](MaxSum x, MaxSum z) { return merge_ms(x, z, ch0, cl0); };
+            MaxSum acc{kNegInf, 0.f};
+            if (have[q]) acc = MaxSum{part[q][0].m, part[q][0].s};
+            for (int sl = lane + 32; sl < p.n_slices; sl += 32) acc = merge(acc, MaxSum{st[sl].m, st[sl].s});
+            acc = warp_reduce(acc, merge);
+            if (lane == 0) { s_m[r] = acc.m; s_s[r] = acc.s; }
         }
     }
     bad = __syncthreads_or(bad);
@@ -157,23 +215,34 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
         return;
     }
 
-    // ---- accept tests, in order, stopping at the first rejection
-    if (tid == 0) {
-        int a = 0;
-        if (greedy) {
-            while (a < k && s_y[a] == s_idx[a]) ++a;
-        } else {
-            for (; a < k; ++a) {
-                const float mt = s_m[a], st = s_s[a];
-                const float mz = s_m[k + 1 + a], sz = s_s[k + 1 + a];
-                const float D = (s_ty[a] - mt) - (s_zy[a] - mz);
-                const float r = expf(__fdiv_rn(D, p.T)) * __fdiv_rn(sz, st);
-                const float u = s_u[a];
-                if (rank == 0 && p.diag_margin) p.diag_margin[size_t(b) * k + a] = fabsf(u - r);
-                if (!(u < r)) break;
+    // ---- accept tests: warp 0 runs them all at once, one position per lane, and
+    // the first failing position is a (the tests after it are not decided)
+    if (warp == 0) {
+        int a = k;
+        float r_all[(OSD_VERIFY_MAX_K + 31) / 32];
+#pragma unroll
+        for (int c = 0; c < (OSD_VERIFY_MAX_K + 31) / 32; ++c) {
+            const int i = c * 32 + lane;
+            bool fail = false;
+            r_all[c] = 0.f;
+            if (i < k) {
+                const float mt = s_m[i], st = s_s[i];
+                const float mz = s_m[k + 1 + i], sz = s_s[k + 1 + i];
+                const float D = (s_ty[i] - mt) - (s_zy[i] - mz);
+                r_all[c] = expf(__fdiv_rn(D, p.T)) * __fdiv_rn(sz, st);
+                fail = !(s_u[i] < r_all[c]);
+            }
+            const unsigned f = __ballot_sync(0xffffffffu, fail);
+            if (f && a == k) a = c * 32 + __ffs(f) - 1;
+        }
+        if (rank == 0 && p.diag_margin) {
+#pragma unroll
+            for (int c = 0; c < (OSD_VERIFY_MAX_K + 31) / 32; ++c) {
+                const int i = c * 32 + lane;
+                if (i < k && i <= a) p.diag_margin[size_t(b) * k + i] = fabsf(s_u[i] - r_all[c]);
             }
         }
-        s_a = a;
+        if (lane == 0) s_a = a;
     }
     __syncthreads();
     const int a = s_a;
@@ -184,15 +253,8 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
             else if (i > a) out[i] = -1;
         for (int i = tid; i < k; i += kFinThreads) {
             p.mask[size_t(b) * k + i] = (i == a) ? 1 : 0;
-            if (p.diag_margin && (greedy || i > a)) p.diag_margin[size_t(b) * k + i] = __int_as_float(0x7fc00000);
+            if (p.diag_margin && i > a) p.diag_margin[size_t(b) * k + i] = __int_as_float(0x7fc00000);
         }
-    }
-    if (greedy) {  // launched with one CTA per sequence
-        if (tid == 0) {
-            out[a] = s_idx[a];
-            if (p.diag_gap) p.diag_gap[b] = __int_as_float(0x7fc00000);
-        }
-        return;
     }
 
     // ---- extra token: inverse CDF of w = max(0, p_a - q_a) (a < k) or p_k (a == k)
@@ -488,15 +550,20 @@ static osd_status launch_verify(const void* draft, const void* target, int B, in
     fp.stats = stats; fp.n_slices = n_slices; fp.n_draft_rows = n_draft_rows;
     fp.accepted = accepted; fp.out_tokens = out_tokens; fp.mask = mask;
     fp.diag_margin = diag_margin; fp.diag_gap = diag_gap;
+    if (greedy) {
+        fp.csize = 1;
+        fp.span = V;
+        const dim3 grid_g(unsigned((B + kGreedyWarps - 1) / kGreedyWarps));
+        return from_cuda(launch_ex(true, verify_greedy_kernel, grid_g, dim3(kGreedyWarps * 32), 0, stream, 1, fp));
+    }
     int csize = 1, span = V;
-    if (!greedy) finalize_shape(B, V, &csize, &span);
+    finalize_shape(B, V, &csize, &span);
     fp.csize = csize;
     fp.span = span;
-    const bool vec = !greedy && aligned_to(draft, 16) && aligned_to(target, 16) &&
-                     ((size_t)V * sizeof(In)) % 16 == 0;
+    const bool vec = aligned_to(draft, 16) && aligned_to(target, 16) && ((size_t)V * sizeof(In)) % 16 == 0;
     const dim3 grid2(unsigned(B) * unsigned(csize));
     const int sub = 32 * (vec ? Elem<In>::kVec : 1);
-    const size_t smem2 = greedy ? 0 : size_t((span + sub - 1) / sub) * sizeof(float);
+    const size_t smem2 = size_t((span + sub - 1) / sub) * sizeof(float);
     if (smem2 > size_t(kFinMaxSub) * sizeof(float)) return OSD_ERR_UNSUPPORTED;
     if (vec)
         e = launch_ex(true, verify_finalize_kernel<In, true>, grid2, dim3(kFinThreads), smem2, stream, csize, fp);
