@@ -30,7 +30,9 @@
 
 namespace osd {
 
-constexpr int kDistThreads = kRowThreads;
+constexpr int kDistThreads = kRowThreads;      // threads per CTA ...
+constexpr int kDistThreadsWide = 256;          // ... and for spans of kDistWideSpan entries or more, where
+constexpr int kDistWideSpan = 12288;           // FKL, RKL, CE and JSD measured 5-10 % faster (V = 128256)
 constexpr int kDistMaxCluster = 8;
 constexpr int kDistSpanBytes = 32768;         // target bytes of both rows per CTA
 constexpr int kDistSpanBytesJsd = 49152;      // JSD, bound by its ex2/lg2 work, does best with fewer, longer spans
@@ -79,6 +81,7 @@ struct Stats2 {
 __device__ __forceinline__ bool pivot_wins(float m, float t, float m0, float t0) {
     return m > m0 || (m == m0 && t > t0);
 }
+template <int kT>
 __device__ __forceinline__ float3 block_max_pivot(float mz, float tp, float mt, float3* scratch) {
     for (int o = 16; o > 0; o >>= 1) {
         const float m2 = __shfl_xor_sync(0xffffffffu, mz, o), t2 = __shfl_xor_sync(0xffffffffu, tp, o);
@@ -91,7 +94,7 @@ __device__ __forceinline__ float3 block_max_pivot(float mz, float tp, float mt, 
     __syncthreads();
     float3 r = scratch[0];
 #pragma unroll
-    for (int w = 1; w < kDistThreads / 32; ++w) {
+    for (int w = 1; w < kT / 32; ++w) {
         const float3 x = scratch[w];
         if (pivot_wins(x.x, x.y, r.x, r.y)) { r.x = x.x; r.y = x.y; }
         r.z = fmaxf(r.z, x.z);
@@ -163,7 +166,7 @@ __device__ __forceinline__ float load_q(const In* zs, const In* ts, int j) {
 // gradient q (s/2 - G) / tau is q Q- / tau where q >= p and -q Q+ / tau where
 // q < p: both products of positive sums, so nothing cancels when one side
 // holds almost all the mass.
-template <typename In, bool kAligned>
+template <typename In, bool kAligned, int kT>
 __device__ __forceinline__ void tvd_gradient(const In* zs, const In* ts, int n, float gpos, float gneg,
                                              float* orow) {
     const int tid = threadIdx.x;
@@ -178,7 +181,7 @@ __device__ __forceinline__ void tvd_gradient(const In* zs, const In* ts, int n, 
     if constexpr (kAligned) {
         constexpr int kVec = Elem<In>::kVec;
         const int nv = n / kVec;
-        for (int v = tid; v < nv; v += kDistThreads) {
+        for (int v = tid; v < nv; v += kT) {
             float q[kVec];
             if constexpr (sizeof(In) == 4) {
                 const float4 f = *reinterpret_cast<const float4*>(zs + v * kVec);
@@ -205,12 +208,12 @@ __device__ __forceinline__ void tvd_gradient(const In* zs, const In* ts, int n, 
         const int r0 = nv * kVec;
         if (tid < n - r0) orow[r0 + tid] = g_of(load_q(zs, ts, r0 + tid));
     } else {
-        for (int e = tid; e < n; e += kDistThreads) orow[e] = g_of(load_q(zs, ts, e));
+        for (int e = tid; e < n; e += kT) orow[e] = g_of(load_q(zs, ts, e));
     }
 }
 
-template <typename In, int kKind, bool kAligned>
-__global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
+template <typename In, int kKind, bool kAligned, int kT>
+__global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
     // JSD clamps both rows to -1e30: a zero probability then stays exactly 0 and
     // every logit difference finite, so no entry needs a guard.  TVD needs none
     // either: a -inf gives p or q = 0, and the sign it picks multiplies q = 0.
@@ -230,12 +233,12 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     __shared__ __align__(8) uint64_t bar;
     __shared__ Stats1 s1_mine, s1_all;
     __shared__ Stats2 s2_mine, s2_all;
-    __shared__ float2 red_m[kDistThreads / 32];
-    __shared__ float3 red_s[kDistThreads / 32];
+    __shared__ float2 red_m[kT / 32];
+    __shared__ float3 red_s[kT / 32];
     __shared__ int s_err;
     __shared__ float s_cu, s_cv, s_loss, s_K, s_tp;
-    __shared__ Label red_l[kDistThreads / 32];
-    __shared__ int2 red_i[kDistThreads / 32];
+    __shared__ Label red_l[kT / 32];
+    __shared__ int2 red_i[kT / 32];
 
     const int tid = threadIdx.x;
     const int csize = p.csize;
@@ -249,13 +252,13 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         const int b = static_cast<int>(row), a = p.accepted[b];
         const bool active = a >= 0 && a < p.k;
         int2 cnt = make_int2(0, 0);  // (active before b, active in total)
-        for (int i = tid; i < p.G; i += kDistThreads) {
+        for (int i = tid; i < p.G; i += kT) {
             const int ai = p.accepted[i];
             const int act = (ai >= 0 && ai < p.k) ? 1 : 0;
             cnt.x += (i < b) ? act : 0;
             cnt.y += act;
         }
-        cnt = block_reduce<kDistThreads>(cnt, [](int2 u, int2 v) { return make_int2(u.x + v.x, u.y + v.y); },
+        cnt = block_reduce<kT>(cnt, [](int2 u, int2 v) { return make_int2(u.x + v.x, u.y + v.y); },
                                          red_i);
         const long long slot = active ? cnt.x : cnt.y + (b - cnt.x);
         if (rank == 0 && tid == 0) {
@@ -286,13 +289,13 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     In* ts = zs + p.span;
 
     // ---- stage the span of both rows in shared memory
-    const int err_local = stage_span<In, kAligned>(zs, ts, zrow + e0, trow + e0, n, &bar, &s_err);
+    const int err_local = stage_span<In, kAligned, kT>(zs, ts, zrow + e0, trow + e0, n, &bar, &s_err);
 
     // ---- pass 0: this thread's maxima, and the chunk where each first appears
     float mz = kNegInf, mt = kNegInf;
     int jz = -1, jt = -1;
     if (!err_local) {
-        sweep<In, kAligned, kClampZ, kClampT, true, false, kUn>(zs, ts, n, [&](const float* z, const float* t, auto tag,
+        sweep<In, kAligned, kClampZ, kClampT, true, false, kUn, kT>(zs, ts, n, [&](const float* z, const float* t, auto tag,
                                                                    int j0, float cz, float ct, bool,
                                                                    const uint4& zr, const uint4& tr) {
             if (cz > mz) { mz = cz; jz = j0; }
@@ -334,17 +337,17 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     float gzb, gtb, tpv = 0.f;
     Label bl{kNegInf, INT_MAX, 0.f};
     if constexpr (kKind == OSD_RKL) {
-        const float3 r = block_max_pivot(mz, tp, mt, red_s);
+        const float3 r = block_max_pivot<kT>(mz, tp, mt, red_s);
         gzb = r.x;
         tpv = r.y;
         gtb = r.z;
     } else {
         // red_m has no readers yet: staging ended on a block barrier
-        const float2 bm = block_max2<false>(mz, mt, red_m);
+        const float2 bm = block_max2<false, kT>(mz, mt, red_m);
         gzb = bm.x;
         gtb = bm.y;
         if constexpr (kKind == OSD_CE)
-            bl = block_reduce<kDistThreads>(lab, [](Label a, Label b) { return merge_label(a, b); }, red_l);
+            bl = block_reduce<kT>(lab, [](Label a, Label b) { return merge_label(a, b); }, red_l);
     }
 
     // ---- pass 1: sums of 2^((x - m) c) against the block maxima (+ the FKL/RKL moment)
@@ -368,7 +371,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     if (!err_local) {
         const float2 gz2 = f2(gzb), gt2 = f2(gtb), tp2 = f2(tpv);
         const float2 nMz2 = f2(-Mz), nMt2 = f2(-Mt);
-        sweep<In, kAligned, false, false, false, kMoment, kUn>(zs, ts, n, [&](const float* z, const float* t,
+        sweep<In, kAligned, false, false, false, kMoment, kUn, kT>(zs, ts, n, [&](const float* z, const float* t,
                                                                              auto tag, int, float, float,
                                                                              bool ninf, const uint4&, const uint4&) {
             constexpr int kCnt = decltype(tag)::value;
@@ -421,7 +424,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     }
     {
         // red_s was last read by RKL's pivot merge; the other kinds have not used it yet
-        const float3 bs = block_sum3<kKind == OSD_RKL>(Ez2.x + Ez2.y, Et2.x + Et2.y, X2.x + X2.y, red_s);
+        const float3 bs = block_sum3<kKind == OSD_RKL, kT>(Ez2.x + Ez2.y, Et2.x + Et2.y, X2.x + X2.y, red_s);
         const int any_ninf = kMoment ? __syncthreads_or(row_ninf ? 1 : 0) : 0;
         const int any_inf = (kKind == OSD_RKL) ? __syncthreads_or(rkl_inf ? 1 : 0) : 0;
         if (tid == 0)
@@ -528,7 +531,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
         // ---- pass 2: divergence terms with the global normalisers
         float2 A2 = f2(0.f), B2 = f2(0.f), C2 = f2(0.f);
         if (!row_err && !jsd_trivial) {
-            sweep<In, kAligned, false, false, false, false, kUn>(zs, ts, n, [&](const float* z, const float* t,
+            sweep<In, kAligned, false, false, false, false, kUn, kT>(zs, ts, n, [&](const float* z, const float* t,
                                                                                auto tag, int j0, float, float, bool,
                                                                                const uint4& zr, const uint4& tr) {
                 constexpr int kCnt = decltype(tag)::value;
@@ -588,7 +591,7 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
             });
         }
         // red_s was last read before the cluster merge's barriers
-        const float3 bs = block_sum3<false>(A2.x + A2.y, B2.x + B2.y, C2.x + C2.y, red_s);
+        const float3 bs = block_sum3<false, kT>(A2.x + A2.y, B2.x + B2.y, C2.x + C2.y, red_s);
         if (tid == 0) s2_mine = Stats2{bs.x, bs.y, bs.z};
         if (csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
         if (tid < 32) {
@@ -632,14 +635,14 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
     // ---- pass 3: d loss / d draft logits of the span
     if (kKind == OSD_TVD && !row_err) {
         // from the stored q' = q sign(q - p): q' Q- / tau, or q' Q+ / tau where q' < 0
-        tvd_gradient<In, kAligned>(zs, ts, n, s2.c * inv_tau, s2.b * inv_tau, p.dlogits + row * V + e0);
+        tvd_gradient<In, kAligned, kT>(zs, ts, n, s2.c * inv_tau, s2.b * inv_tau, p.dlogits + row * V + e0);
     } else if (kKind != OSD_TVD && !row_err) {
         float* orow = p.dlogits + row * V + e0;
         const float K = s_K, tpg = s_tp;
         // q and p of this pass come out multiplied by the gradient's constant factor
         const float2 cvs = f2(cv + p.lg_scale), cus = f2(cu + p.lg_scale);
         const int label = st.idx;
-        sweep<In, kAligned, false, false, false, false, kUn3>(zs, ts, n, [&](const float* z, const float* t,
+        sweep<In, kAligned, false, false, false, false, kUn3, kT>(zs, ts, n, [&](const float* z, const float* t,
                                                                             auto tag, int j0, float, float, bool,
                                                                             const uint4& zr, const uint4& tr) {
             constexpr int kCnt = decltype(tag)::value;
@@ -713,9 +716,9 @@ __global__ void __launch_bounds__(kDistThreads) distill_kernel(DistParams p) {
 }
 
 // ------------------------------------------------------------------ host
-template <typename In, int kKind, bool kAligned>
+template <typename In, int kKind, bool kAligned, int kT>
 static cudaError_t launch_distill_kind(const DistParams& dp, long long rows, size_t smem, cudaStream_t s) {
-    auto kern = distill_kernel<In, kKind, kAligned>;
+    auto kern = distill_kernel<In, kKind, kAligned, kT>;
     if (smem > 48 * 1024) {
         // the opt-in is per device and kernel; set it once, so that later calls
         // (including ones under stream capture) make no attribute call
@@ -734,19 +737,34 @@ static cudaError_t launch_distill_kind(const DistParams& dp, long long rows, siz
             }
         }
     }
-    return launch(kern, dim3(static_cast<unsigned>(rows * dp.csize)), dim3(kDistThreads), smem, s,
+    return launch(kern, dim3(static_cast<unsigned>(rows * dp.csize)), dim3(kT), smem, s,
                   dp.csize, dp);
 }
 
+// Wide CTAs only on the 16-byte path (TVD, whose extra cluster exchange costs
+// more with them, always takes kDistThreads).
 template <typename In, bool kAligned>
 static cudaError_t launch_distill_dtype(osd_loss kind, const DistParams& dp, long long rows, size_t smem,
                                         cudaStream_t s) {
+    constexpr int kN = kDistThreads;
+    if constexpr (kAligned) {
+        constexpr int kWd = kDistThreadsWide;
+        if (dp.span >= kDistWideSpan) {
+            switch (kind) {
+                case OSD_FKL: return launch_distill_kind<In, OSD_FKL, true, kWd>(dp, rows, smem, s);
+                case OSD_RKL: return launch_distill_kind<In, OSD_RKL, true, kWd>(dp, rows, smem, s);
+                case OSD_JSD: return launch_distill_kind<In, OSD_JSD, true, kWd>(dp, rows, smem, s);
+                case OSD_CE: return launch_distill_kind<In, OSD_CE, true, kWd>(dp, rows, smem, s);
+                default: break;
+            }
+        }
+    }
     switch (kind) {
-        case OSD_FKL: return launch_distill_kind<In, OSD_FKL, kAligned>(dp, rows, smem, s);
-        case OSD_RKL: return launch_distill_kind<In, OSD_RKL, kAligned>(dp, rows, smem, s);
-        case OSD_JSD: return launch_distill_kind<In, OSD_JSD, kAligned>(dp, rows, smem, s);
-        case OSD_CE: return launch_distill_kind<In, OSD_CE, kAligned>(dp, rows, smem, s);
-        default: return launch_distill_kind<In, OSD_TVD, kAligned>(dp, rows, smem, s);
+        case OSD_FKL: return launch_distill_kind<In, OSD_FKL, kAligned, kN>(dp, rows, smem, s);
+        case OSD_RKL: return launch_distill_kind<In, OSD_RKL, kAligned, kN>(dp, rows, smem, s);
+        case OSD_JSD: return launch_distill_kind<In, OSD_JSD, kAligned, kN>(dp, rows, smem, s);
+        case OSD_CE: return launch_distill_kind<In, OSD_CE, kAligned, kN>(dp, rows, smem, s);
+        default: return launch_distill_kind<In, OSD_TVD, kAligned, kN>(dp, rows, smem, s);
     }
 }
 

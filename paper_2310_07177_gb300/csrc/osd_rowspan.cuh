@@ -1,7 +1,8 @@
 // osd_rowspan.cuh -- building blocks of the kernels that stage one span of a
 // draft row and a target row in shared memory and sweep it several times
 // (distillation and mixed sampling).  One thread-block cluster per row, each
-// CTA of kRowThreads threads owns a contiguous span of the vocabulary.
+// CTA of kRowThreads (or a template's kT) threads owns a contiguous span of the
+// vocabulary.
 #pragma once
 
 #include <cstddef>
@@ -26,7 +27,7 @@ __device__ __forceinline__ void copy_raw(In* dst, const In* src) {
 // aligned path the 16-byte body goes by two bulk copies completing on `bar`
 // and the ragged tail by plain loads.  Every thread calls it; it returns
 // non-zero (for every thread) when the bounded wait for the copies gave up.
-template <typename In, bool kAligned>
+template <typename In, bool kAligned, int kT = kRowThreads>
 __device__ __forceinline__ int stage_span(In* zs, In* ts, const In* zsrc, const In* tsrc, int n, uint64_t* bar,
                                           int* s_err) {
     const int tid = threadIdx.x;
@@ -41,7 +42,7 @@ __device__ __forceinline__ int stage_span(In* zs, In* ts, const In* zsrc, const 
             bulk_g2s(zs, zsrc, bytes, bar);
             bulk_g2s(ts, tsrc, bytes, bar);
         }
-        for (int e = nb + tid; e < n; e += kRowThreads) {
+        for (int e = nb + tid; e < n; e += kT) {
             copy_raw(zs + e, zsrc + e);
             copy_raw(ts + e, tsrc + e);
         }
@@ -51,7 +52,7 @@ __device__ __forceinline__ int stage_span(In* zs, In* ts, const In* zsrc, const 
         }
     } else {
         __syncthreads();
-        for (int e = tid; e < n; e += kRowThreads) {
+        for (int e = tid; e < n; e += kT) {
             copy_raw(zs + e, zsrc + e);
             copy_raw(ts + e, tsrc + e);
         }
@@ -65,11 +66,11 @@ __device__ __forceinline__ int stage_span(In* zs, In* ts, const In* zsrc, const 
 // happens on the packed words.  f(z[], t[], count_tag, j0, zmax, tmax, ninf,
 // zraw, traw) gets the chunk maxima when kMax is set, ninf = "the chunk holds a
 // -inf" when kMin is set, and the (clamped) packed words of a full chunk.
-// Chunk v goes to thread v mod kRowThreads, so warp w sees the 32-chunk groups
-// w, w + kRowWarps, ... in order.  kUnroll unrolls the chunk loop (two chunks
-// a trip halve the loop overhead, at some registers).
+// Chunk v goes to thread v mod kT (the CTA's threads), so warp w sees the
+// 32-chunk groups w, w + kT/32, ... in order.  kUnroll unrolls the chunk loop
+// (two chunks a trip halve the loop overhead, at some registers).
 template <typename In, bool kAligned, bool kClampZ, bool kClampT, bool kMax, bool kMin = false, int kUnroll = 1,
-          typename F>
+          int kT = kRowThreads, typename F>
 __device__ __forceinline__ void sweep(const In* zs, const In* ts, int n, F&& f) {
     using E = Elem<In>;
     constexpr int kVec = E::kVec;
@@ -77,7 +78,7 @@ __device__ __forceinline__ void sweep(const In* zs, const In* ts, int n, F&& f) 
     if constexpr (kAligned) {
         const int nv = n / kVec;
 #pragma unroll kUnroll
-        for (int v = tid; v < nv; v += kRowThreads) {
+        for (int v = tid; v < nv; v += kT) {
             uint4 zr = lds_v4(zs + v * kVec), tr = lds_v4(ts + v * kVec);
             if (kClampZ) E::clamp_raw(zr);
             if (kClampT) E::clamp_raw(tr);
@@ -96,7 +97,7 @@ __device__ __forceinline__ void sweep(const In* zs, const In* ts, int n, F&& f) 
             f(&z, &t, std::integral_constant<int, 1>{}, r0 + tid, z, t, fminf(z, t) == kNegInf, uint4{}, uint4{});
         }
     } else {
-        for (int e = tid; e < n; e += kRowThreads) {
+        for (int e = tid; e < n; e += kT) {
             float z = E::lds(zs + e), t = E::lds(ts + e);
             if (kClampZ) z = E::clamp1(z);
             if (kClampT) t = E::clamp1(t);
@@ -110,7 +111,7 @@ __device__ __forceinline__ void sweep(const In* zs, const In* ts, int n, F&& f) 
 // kGuard adds the barrier that keeps a previous reduction's readers of
 // `scratch` ahead of the new writes; callers whose scratch has no readers
 // since the last block barrier leave it out.
-template <bool kGuard = true>
+template <bool kGuard = true, int kT = kRowThreads>
 __device__ __forceinline__ float2 block_max2(float a, float b, float2* scratch) {
     for (int o = 16; o > 0; o >>= 1) {
         a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
@@ -122,10 +123,10 @@ __device__ __forceinline__ float2 block_max2(float a, float b, float2* scratch) 
     __syncthreads();
     float2 r = scratch[0];
 #pragma unroll
-    for (int w = 1; w < kRowWarps; ++w) r = make_float2(fmaxf(r.x, scratch[w].x), fmaxf(r.y, scratch[w].y));
+    for (int w = 1; w < kT / 32; ++w) r = make_float2(fmaxf(r.x, scratch[w].x), fmaxf(r.y, scratch[w].y));
     return r;
 }
-template <bool kGuard = true>
+template <bool kGuard = true, int kT = kRowThreads>
 __device__ __forceinline__ float3 block_sum3(float a, float b, float c, float3* scratch) {
     for (int o = 16; o > 0; o >>= 1) {
         a += __shfl_xor_sync(0xffffffffu, a, o);
@@ -138,7 +139,7 @@ __device__ __forceinline__ float3 block_sum3(float a, float b, float c, float3* 
     __syncthreads();
     float3 r = scratch[0];
 #pragma unroll
-    for (int w = 1; w < kRowWarps; ++w) r = make_float3(r.x + scratch[w].x, r.y + scratch[w].y, r.z + scratch[w].z);
+    for (int w = 1; w < kT / 32; ++w) r = make_float3(r.x + scratch[w].x, r.y + scratch[w].y, r.z + scratch[w].z);
     return r;
 }
 

@@ -58,7 +58,9 @@ SHAPES = [  # (N, V, dtype)
     (2, 32000, torch.float32),
     (3, 33001, torch.bfloat16),
     (2, 32128, torch.float32),
-    (2, 128256, torch.bfloat16),
+    (2, 128256, torch.bfloat16),   # spans of 16032: 256-thread CTAs for every kind but TVD
+    (2, 100000, torch.bfloat16),   # the wide path with 12544-entry spans
+    (2, 100003, torch.bfloat16),   # the same length off the 16-byte path: 128-thread CTAs
     (2, 393216, torch.bfloat16),   # the largest vocabulary per dtype: 192 KB of staging per CTA
     (2, 196608, torch.float32),
 ]
