@@ -353,6 +353,11 @@ __device__ __forceinline__ double ld_dsmem_f64(uint32_t addr) {
     asm volatile("ld.shared::cluster.f64 %0, [%1];" : "=d"(v) : "r"(addr) : "memory");
     return v;
 }
+__device__ __forceinline__ unsigned long long ld_dsmem_u64(uint32_t addr) {
+    unsigned long long v;
+    asm volatile("ld.shared::cluster.u64 %0, [%1];" : "=l"(v) : "r"(addr) : "memory");
+    return v;
+}
 __device__ __forceinline__ int ld_dsmem_s32(uint32_t addr) {
     int v;
     asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
@@ -386,6 +391,51 @@ template <typename In, int kW>
 __device__ __forceinline__ void unpack_raw(const uint4& r, float* v) {
     if constexpr (kW == 1) v[0] = __uint_as_float(r.x);
     else Elem<In>::unpack(r, v);
+}
+
+// ---------------------------------------------------------------- exact CDF sums
+// Non-negative weights below 8 as unsigned 64-bit fixed point with kFixBits
+// fraction bits, truncated.  Sums of them are exact, so a prefix sum does not
+// depend on the order of its adds; and an integer add takes a few cycles where
+// a dependent fp64 add takes about 64 on this GPU.  Truncation loses less than
+// 2^-60 per weight.
+constexpr int kFixBits = 60;
+__device__ __forceinline__ unsigned long long fix_of(float x) {
+    const uint32_t bits = __float_as_uint(x);
+    const int e = static_cast<int>(bits >> 23);  // x >= 0: no sign bit
+    if (e == 0) return 0ull;                     // zero or subnormal, below 2^-126
+    const unsigned long long m = (bits & 0x7fffffu) | 0x800000u;
+    const int sh = e - (127 + 23) + kFixBits;    // x = m 2^(e - 150)
+    return sh >= 0 ? (m << sh) : (sh > -64 ? (m >> -sh) : 0ull);
+}
+__device__ __forceinline__ float fix_to_float(unsigned long long v) {
+    return __ull2float_rn(v) * (1.0f / static_cast<float>(1ull << kFixBits));
+}
+// floor(u W) for u in [0, 1) (u >= 1 gives W): u as a 64-bit binary fraction,
+// exact for u >= 2^-40, times W, high half.
+__device__ __forceinline__ unsigned long long fix_scale(float u, unsigned long long W) {
+    const uint32_t bits = __float_as_uint(u);
+    const int e = static_cast<int>(bits >> 23);
+    if (e == 0 || (bits >> 31)) return 0ull;
+    if (e >= 127) return W;
+    const unsigned long long m = (bits & 0x7fffffu) | 0x800000u;
+    const int sh = e - 150 + 64;  // <= 40 for u < 1
+    const unsigned long long U = sh >= 0 ? (m << sh) : (sh > -64 ? (m >> -sh) : 0ull);
+    return __umul64hi(U, W);
+}
+__device__ __forceinline__ unsigned long long warp_sum_u64(unsigned long long v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ unsigned long long warp_incl_scan_u64(unsigned long long v) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const unsigned long long y = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += y;
+    }
+    return v;
 }
 
 }  // namespace osd

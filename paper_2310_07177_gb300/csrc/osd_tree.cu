@@ -72,9 +72,10 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
     constexpr int kW = kVecPath ? E::kVec : 1;  // entries per lane per sub-tile
     constexpr int kSub = 32 * kW;
     extern __shared__ float s_sub[];           // mass of every sub-tile of this CTA's span (last pass)
-    __shared__ double s_span_total;            // read by the other CTAs of the cluster
-    __shared__ double s_cta_incl[kTreeMaxCluster];  // inclusive prefix of the CTA masses, rank order
-    __shared__ double s_W;
+    // masses in exact 64-bit fixed point (fix_of): a dependent fp64 add is slow here
+    __shared__ unsigned long long s_span_total;            // read by the other CTAs of the cluster
+    __shared__ unsigned long long s_cta_incl[kTreeMaxCluster];  // inclusive prefix of the CTA masses, rank order
+    __shared__ unsigned long long s_W;
     __shared__ int s_next, s_extra;
     // per node: merged statistics of its target (0) and draft (1) rows, or the target argmax at T = 0
     __shared__ float s_nm[2][OSD_TREE_MAX_NODES], s_ns[2][OSD_TREE_MAX_NODES];
@@ -202,8 +203,9 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
         }
     };
     // One cluster-wide pass: the mass of every sub-tile of w = max(0, p - s q) into s_sub,
-    // the CTA masses' inclusive prefix into s_cta_incl, and the row's mass W (returned).
-    auto mass_pass = [&](const In* trow, const In* zrow, bool use_q, float s) -> double {
+    // the CTA masses' inclusive prefix into s_cta_incl, and the row's mass W (returned,
+    // fixed point).
+    auto mass_pass = [&](const In* trow, const In* zrow, bool use_q, float s) -> unsigned long long {
         if (pending) cluster_wait();  // every peer has read the previous pass's total
         for (int sb0 = warp; sb0 < nsub; sb0 += kTreeWarps * kTreeUnroll) {
             Raw r[kTreeUnroll];  // the loads of kTreeUnroll sub-tiles go out together
@@ -226,16 +228,16 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
         }
         __syncthreads();
         if (warp == 0) {
-            double part = 0.0;
-            for (int sb = lane; sb < nsub; sb += 32) part += double(s_sub[sb]);
-            part = warp_sum_f64(part);
+            unsigned long long part = 0ull;
+            for (int sb = lane; sb < nsub; sb += 32) part += fix_of(s_sub[sb]);
+            part = warp_sum_u64(part);
             if (lane == 0) s_span_total = part;
         }
         if (csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
         if (warp == 0) {
-            double tot = 0.0;
-            if (lane < csize) tot = (lane == rank) ? s_span_total : ld_dsmem_f64(map_rank(&s_span_total, lane));
-            const double incl = warp_incl_scan_f64(tot);
+            unsigned long long tot = 0ull;
+            if (lane < csize) tot = (lane == rank) ? s_span_total : ld_dsmem_u64(map_rank(&s_span_total, lane));
+            const unsigned long long incl = warp_incl_scan_u64(tot);
             if (lane < csize) s_cta_incl[lane] = incl;
             if (lane == 31) s_W = incl;
         }
@@ -272,6 +274,7 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
         } else {
             float s = 0.f;  // residual shift s_j
             double N = 1.0;  // residual mass N_j (p itself has mass 1)
+            unsigned long long Nfix = 0ull;  // the same, in fixed point, after a mass pass
             bool passed = false;  // a mass pass of the current residual has run
             for (int c = p.topo.first_child[node]; c >= 0; c = p.topo.next_sibling[c]) {
                 if (tid == 0) {
@@ -296,25 +299,26 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
                 __syncthreads();  // s_next is rewritten by the next test
                 if (next >= 0) break;
                 s = static_cast<float>(double(s) + N);  // rejected: s_{j+1} = s_j + N_j
-                N = mass_pass(trow, zrow, true, s);
+                Nfix = mass_pass(trow, zrow, true, s);
+                N = __ull2double_rn(Nfix) * (1.0 / static_cast<double>(1ull << kFixBits));
                 passed = true;
             }
             if (next < 0) {
                 // ---- the extra token from w = max(0, p - s q) (p itself when nothing was rejected)
                 const bool use_q = passed;
-                const double W = passed ? N : mass_pass(trow, zrow, false, 0.f);
-                const double tau = double(s_u[0]) * W;
+                const unsigned long long W = passed ? Nfix : mass_pass(trow, zrow, false, 0.f);
+                const unsigned long long tau = fix_scale(s_u[0], W);  // floor(u W)
                 int owner = -1, mode = 0;  // mode 0: inverse CDF, 1: largest positive entry, 2: argmax p
-                double base = 0.0;
-                if (W > 0.0) {
+                unsigned long long base = 0ull;
+                if (W > 0ull) {
                     for (int r = 0; r < csize; ++r)
                         if (s_cta_incl[r] > tau) { owner = r; break; }
                     if (owner >= 0) {
-                        base = owner > 0 ? s_cta_incl[owner - 1] : 0.0;
+                        base = owner > 0 ? s_cta_incl[owner - 1] : 0ull;
                     } else {
                         mode = 1;
                         for (int r = csize - 1; r >= 0 && owner < 0; --r)
-                            if (s_cta_incl[r] > (r > 0 ? s_cta_incl[r - 1] : 0.0)) owner = r;
+                            if (s_cta_incl[r] > (r > 0 ? s_cta_incl[r - 1] : 0ull)) owner = r;
                         if (owner < 0) owner = csize - 1;
                     }
                 } else {
@@ -323,7 +327,7 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
                 }
                 if (rank == owner && warp == 0) {
                     int pick = -1;
-                    double gap = __int_as_float(0x7fc00000);
+                    float gap = __int_as_float(0x7fc00000);
                     if (mode == 2) {  // no residual mass: argmax of p over the row, lowest index
                         MaxIdx acc{kNegInf, INT_MAX};
                         for (int j = lane; j < V; j += 32) {
@@ -336,23 +340,23 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
                         // the sub-tile: lane l owns the run [s_lo, s_hi) of sub-tiles
                         const int per = (nsub + 31) / 32;
                         const int s_lo = min(nsub, lane * per), s_hi = min(nsub, s_lo + per);
-                        double mine = 0.0;
-                        for (int sb = s_lo; sb < s_hi; ++sb) mine += double(s_sub[sb]);
-                        const double excl = base + warp_incl_scan_f64(mine) - mine;
+                        unsigned long long mine = 0ull;
+                        for (int sb = s_lo; sb < s_hi; ++sb) mine += fix_of(s_sub[sb]);
+                        const unsigned long long excl = base + warp_incl_scan_u64(mine) - mine;
                         int tile = -1;
-                        double tbase = 0.0;
+                        unsigned long long tbase = 0ull;
                         if (mode == 0) {
                             const unsigned h = __ballot_sync(0xffffffffu, excl <= tau && excl + mine > tau);
                             if (h) {
                                 const int l = __ffs(h) - 1;
-                                if (lane == l) {
-                                    double c2 = excl;
+                                if (lane == l) {  // the sums are exact: the run holds tau in one sub-tile
+                                    unsigned long long c2 = excl;
                                     for (int sb = s_lo; sb < s_hi; ++sb) {
-                                        if (c2 + double(s_sub[sb]) > tau) { tile = sb; break; }
-                                        c2 += double(s_sub[sb]);
+                                        const unsigned long long v = fix_of(s_sub[sb]);
+                                        if (c2 + v > tau) { tile = sb; break; }
+                                        c2 += v;
                                     }
                                     tbase = c2;
-                                    if (tile < 0) { tile = s_hi - 1; tbase = c2 - double(s_sub[s_hi - 1]); }
                                 }
                                 tile = __shfl_sync(0xffffffffu, tile, l);
                                 tbase = __shfl_sync(0xffffffffu, tbase, l);
@@ -374,19 +378,19 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
                         const int j0 = e0 + tile * kSub + lane * kW;
                         bool done = false;
                         if (mode == 0) {
-                            double wsum = 0.0;
+                            unsigned long long wsum = 0ull;
 #pragma unroll
-                            for (int e = 0; e < kW; ++e) wsum += double(w[e]);
-                            const double wex = tbase + warp_incl_scan_f64(wsum) - wsum;
+                            for (int e = 0; e < kW; ++e) wsum += fix_of(w[e]);
+                            const unsigned long long wex = tbase + warp_incl_scan_u64(wsum) - wsum;
                             const bool hit = wex <= tau && wex + wsum > tau;
                             if (hit) {
-                                double C = wex;
+                                unsigned long long C = wex;
                                 for (int e = 0; e < kW; ++e) {
-                                    const double Cprev = C;
-                                    C += double(w[e]);
+                                    const unsigned long long Cprev = C;
+                                    C += fix_of(w[e]);
                                     if (C > tau) {
                                         pick = j0 + e;
-                                        gap = fmin(C - tau, tau - Cprev) / W;
+                                        gap = fminf(fix_to_float(C - tau), fix_to_float(tau - Cprev)) / fix_to_float(W);
                                         break;
                                     }
                                 }
@@ -404,7 +408,8 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
                             pick = -1;
                             if (jb >= 0 && best == jb) {
                                 pick = jb;
-                                gap = fmin(W - tau, tau - (W - double(wbest))) / W;
+                                const float Wf = fix_to_float(W), tf = fix_to_float(tau);
+                                gap = fminf(Wf - tf, tf - (Wf - wbest)) / Wf;
                             } else if (jb < 0 && lane == 0) {
                                 pick = j0;  // no positive entry: cannot happen when W > 0
                             }
@@ -412,7 +417,7 @@ __global__ void __launch_bounds__(kTreeThreads) tree_walk_kernel(TreeParams p) {
                     }
                     if (pick >= 0 && (mode != 2 || lane == 0)) {
                         out[depth] = pick;
-                        if (p.diag_gap && mode != 2) p.diag_gap[b] = float(gap);
+                        if (p.diag_gap && mode != 2) p.diag_gap[b] = gap;
                     }
                 }
                 if (tid == 0) s_extra = -1;  // written by the owner
