@@ -15,8 +15,9 @@
 //                       norm(max(0, p_a - q_a)) (or p_k when all k pass) by inverse
 //                       CDF.  Each CTA of the cluster sums the residual weights of
 //                       its part of the vocabulary per tile; the partial sums meet
-//                       through distributed shared memory and the CTA whose part
-//                       holds u*W rescans that one tile with an fp64 block scan.
+//                       through distributed shared memory as exact 64-bit fixed
+//                       point, and the CTA whose part holds u*W rescans that one
+//                       tile with an exact warp scan.
 //
 //   verify_greedy       (T = 0) one warp per sequence: the argmax of every target
 //                       row from its slices, the matches in order, the target
@@ -141,8 +142,9 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
     __shared__ float s_u[OSD_VERIFY_MAX_K + 1];
     __shared__ int s_a, s_owner, s_mode, s_tile;
     extern __shared__ float s_sub[];  // one residual sum per sub-tile of this CTA's span
-    __shared__ double s_span_total;  // read by the other CTAs of the cluster
-    __shared__ double s_tau, s_W, s_base;
+    // residual masses in exact 64-bit fixed point (fix_of): a dependent fp64 add is slow here
+    __shared__ unsigned long long s_span_total;  // read by the other CTAs of the cluster
+    __shared__ unsigned long long s_tau, s_W, s_base;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int rank = (p.csize > 1) ? static_cast<int>(cluster_rank()) : 0;
@@ -345,34 +347,34 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
         }
     }
     __syncthreads();
-    // span total in fp64, reduced across warp 0 (no serial chain of fp64 adds)
+    // span total, exact, reduced across warp 0
     if (warp == 0) {
-        double part = 0.0;
-        for (int s2 = lane; s2 < nsub; s2 += 32) part += double(s_sub[s2]);
-        part = warp_sum_f64(part);
+        unsigned long long part = 0ull;
+        for (int s2 = lane; s2 < nsub; s2 += 32) part += fix_of(s_sub[s2]);
+        part = warp_sum_u64(part);
         if (lane == 0) s_span_total = part;
     }
     if (p.csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
 
-    // warp 0 of every CTA derives W, tau and the owning CTA identically: lane r
-    // holds CTA r's total, an fp64 warp scan gives the prefix in rank order
+    // warp 0 of every CTA derives W, tau = floor(u W) and the owning CTA identically:
+    // lane r holds CTA r's total, a warp scan gives the prefix in rank order
     if (warp == 0) {
         const float u = s_u[k];
-        double tot = 0.0;
-        if (lane < p.csize) tot = (lane == rank) ? s_span_total : ld_dsmem_f64(map_rank(&s_span_total, lane));
-        const double incl = warp_incl_scan_f64(tot);
-        const double W = __shfl_sync(0xffffffffu, incl, 31);
-        const double tau = double(u) * W;
+        unsigned long long tot = 0ull;
+        if (lane < p.csize) tot = (lane == rank) ? s_span_total : ld_dsmem_u64(map_rank(&s_span_total, lane));
+        const unsigned long long incl = warp_incl_scan_u64(tot);
+        const unsigned long long W = __shfl_sync(0xffffffffu, incl, 31);
+        const unsigned long long tau = fix_scale(u, W);
         int owner, mode = 0;  // mode 0: inverse CDF, 1: largest positive entry, 2: argmax p
-        double base = 0.0;
-        if (W > 0.0) {
+        unsigned long long base = 0ull;
+        if (W > 0ull) {
             const unsigned hit = __ballot_sync(0xffffffffu, lane < p.csize && incl > tau);
             if (hit) {
                 owner = __ffs(hit) - 1;
                 base = __shfl_sync(0xffffffffu, incl - tot, owner);
             } else {  // tau >= W (u >= 1 or rounding): largest j with w_j > 0
                 mode = 1;
-                const unsigned pos = __ballot_sync(0xffffffffu, lane < p.csize && tot > 0.0);
+                const unsigned pos = __ballot_sync(0xffffffffu, lane < p.csize && tot > 0ull);
                 owner = 31 - __clz(pos);
             }
         } else {
@@ -384,21 +386,21 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
             // sub-tile holding tau: each lane owns a run of consecutive sub-tiles
             const int per = (nsub + 31) / 32;
             const int s_lo = min(nsub, lane * per), s_hi = min(nsub, s_lo + per);
-            double mine = 0.0;
-            for (int s2 = s_lo; s2 < s_hi; ++s2) mine += double(s_sub[s2]);
-            const double excl = base + warp_incl_scan_f64(mine) - mine;
+            unsigned long long mine = 0ull;
+            for (int s2 = s_lo; s2 < s_hi; ++s2) mine += fix_of(s_sub[s2]);
+            const unsigned long long excl = base + warp_incl_scan_u64(mine) - mine;
             if (mode == 0) {
                 const unsigned hit = __ballot_sync(0xffffffffu, excl <= tau && excl + mine > tau);
                 if (hit) {
                     const int l = __ffs(hit) - 1;
-                    if (lane == l) {
-                        double c = excl;
+                    if (lane == l) {  // the sums are exact: the run holds tau in one sub-tile
+                        unsigned long long c = excl;
                         for (int s2 = s_lo; s2 < s_hi; ++s2) {
-                            if (c + double(s_sub[s2]) > tau) { tile = s2; break; }
-                            c += double(s_sub[s2]);
+                            const unsigned long long v = fix_of(s_sub[s2]);
+                            if (c + v > tau) { tile = s2; break; }
+                            c += v;
                         }
                         base = c;
-                        if (tile < 0) { tile = s_hi - 1; base = c - double(s_sub[s_hi - 1]); }
                     }
                     tile = __shfl_sync(0xffffffffu, tile, l);
                     base = __shfl_sync(0xffffffffu, base, l);
@@ -420,7 +422,7 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
     if (p.csize > 1) cluster_arrive_relaxed();  // done reading the other CTAs' shared memory
 
     if (rank == s_owner && warp == 0) {
-        const double tau = s_tau, W = s_W;
+        const unsigned long long tau = s_tau, W = s_W;
         const int mode = s_mode, s = s_tile;
         if (mode == 0 || mode == 1) {
             float w[kW];
@@ -433,26 +435,21 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
             const int j0 = e0 + max(s, 0) * kSub + lane * kW;
             bool done = false;
             if (mode == 0) {
-                // fp64 scan of the sub-tile across the warp, then within the lane
-                double mine = 0.0;
+                // exact scan of the sub-tile across the warp, then within the lane
+                unsigned long long mine = 0ull;
 #pragma unroll
-                for (int e = 0; e < kW; ++e) mine += double(w[e]);
-                double incl = mine;
-#pragma unroll
-                for (int o = 1; o < 32; o <<= 1) {
-                    const double y = __shfl_up_sync(0xffffffffu, incl, o);
-                    if (lane >= o) incl += y;
-                }
-                const double excl = s_base + incl - mine;
+                for (int e = 0; e < kW; ++e) mine += fix_of(w[e]);
+                const unsigned long long excl = s_base + warp_incl_scan_u64(mine) - mine;
                 const bool hit = excl <= tau && excl + mine > tau;
                 if (hit) {
-                    double C = excl;
+                    unsigned long long C = excl;
                     for (int e = 0; e < kW; ++e) {
-                        const double Cprev = C;
-                        C += double(w[e]);
+                        const unsigned long long Cprev = C;
+                        C += fix_of(w[e]);
                         if (C > tau) {
                             out[a] = j0 + e;
-                            if (p.diag_gap) p.diag_gap[b] = float(fmin(C - tau, tau - Cprev) / W);
+                            if (p.diag_gap)
+                                p.diag_gap[b] = fminf(fix_to_float(C - tau), fix_to_float(tau - Cprev)) / fix_to_float(W);
                             break;
                         }
                     }
@@ -471,8 +468,8 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
                 if (jb >= 0 && best == jb) {
                     out[a] = jb;
                     if (p.diag_gap) {
-                        const double g1 = W - tau, g0 = tau - (W - double(wbest));
-                        p.diag_gap[b] = float(fmin(g1, g0) / W);
+                        const float Wf = fix_to_float(W), tf = fix_to_float(tau);
+                        p.diag_gap[b] = fminf(Wf - tf, tf - (Wf - wbest)) / Wf;
                     }
                 } else if (jb < 0 && lane == 0) {
                     out[a] = e0;  // no positive entry found: cannot happen when W > 0
