@@ -35,8 +35,10 @@
  *     fp32 or bf16 (OSD_F32 / OSD_BF16).  Any alignment to the element size
  *     is accepted; rows that start on 16-byte boundaries take the fast
  *     vectorised path.
- *   - Accumulation is fp32 inside a thread with fp64 where it decides a
- *     sample position; exponentials use the hardware ex2 unit.
+ *   - Accumulation is fp32 inside a thread.  Where a sum decides a sample
+ *     position it is carried exactly, in 64-bit fixed point with 60
+ *     fraction bits (verification, tree verification), or in fp64 (mixed
+ *     sampling); exponentials use the hardware ex2 unit.
  */
 #ifndef OSD_H_
 #define OSD_H_
