@@ -239,13 +239,7 @@ __device__ __forceinline__ T block_reduce(T v, F f, T* scratch) {
     return r;
 }
 
-// fp64 sum and inclusive prefix sum across a warp (used where a sum decides a
-// sample position)
-__device__ __forceinline__ double warp_sum_f64(double v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    return v;
-}
+// fp64 inclusive prefix sum across a warp (the mixed sampler's CDF scans)
 __device__ __forceinline__ double warp_incl_scan_f64(double v) {
     const int lane = threadIdx.x & 31;
 #pragma unroll
@@ -346,11 +340,6 @@ __device__ __forceinline__ uint32_t map_rank(const void* p, uint32_t rank) {
 __device__ __forceinline__ float ld_dsmem_f32(uint32_t addr) {
     float v;
     asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
-    return v;
-}
-__device__ __forceinline__ double ld_dsmem_f64(uint32_t addr) {
-    double v;
-    asm volatile("ld.shared::cluster.f64 %0, [%1];" : "=d"(v) : "r"(addr) : "memory");
     return v;
 }
 __device__ __forceinline__ unsigned long long ld_dsmem_u64(uint32_t addr) {
