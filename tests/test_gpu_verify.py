@@ -187,6 +187,20 @@ def test_gpu_output_distribution_equals_target(osd, T, V, k):
         assert abs(acc / reach - alpha) < 5 * math.sqrt(alpha * (1 - alpha) / reach)
 
 
+def test_gpu_expected_length_eq1(osd):
+    """Eq. 1 on the GPU's own decisions: the same (p, q) at every position gives
+    E[a + 1] = (1 - alpha^(k+1)) / (1 - alpha), alpha = sum min(p, q)."""
+    rng = np.random.default_rng(88)
+    V, k = 6, 4
+    zrow = rng.normal(0, 1.0, V)
+    trow = rng.normal(0, 1.0, V)
+    a, _ = _mc(osd, np.tile(zrow, (k, 1)), np.tile(trow, (k + 1, 1)), 1.0, 1_000_000, seed=89)
+    alpha = np.minimum(softmax(trow), softmax(zrow)).sum()
+    want = (1 - alpha ** (k + 1)) / (1 - alpha)
+    L = a + 1.0
+    assert abs(L.mean() - want) < 5 * L.std() / math.sqrt(len(L)), (L.mean(), want)
+
+
 # ----------------------------------------------------------------- full-size workloads
 @pytest.mark.parametrize("cfg", [1, 2])
 def test_workload_small_configs_full(osd, cfg):
