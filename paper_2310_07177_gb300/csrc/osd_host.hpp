@@ -4,6 +4,7 @@
 
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 
@@ -30,6 +31,18 @@ inline void split_scale(float temperature, float* c_hi, float* c_lo) {
     if (!(lo > 0.0f)) lo = 1e-30f;
     *c_hi = hi;
     *c_lo = lo;
+}
+
+// Streaming multiprocessors of the current device, looked up once per device
+// (0 when the query fails).
+inline int device_sms() {
+    static std::atomic<int> sms[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    int n = sms[dev].load(std::memory_order_relaxed);
+    if (n == 0 && cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
+        sms[dev].store(n, std::memory_order_relaxed);
+    return n;
 }
 
 // Launch `kernel` with an optional thread-block cluster of `cluster` CTAs
