@@ -10,6 +10,7 @@ from scipy.special import softmax
 from scipy.stats import chisquare
 
 import oracle
+from paper_2310_07177_gb300 import workloads as W
 
 pytestmark = pytest.mark.gpu
 TIE = 1e-6
@@ -89,6 +90,26 @@ def test_many_rows_at_full_vocabulary(osd):
     ties, differ = _check(osd, z, t, u, 0.5, 1.0)
     print(f"mixed sample 2048 x 32000: near-ties {ties}, of which differ {differ}")
     assert ties < 0.1 * 2048
+
+
+def test_workload_full_size_sampled(osd):
+    """The benchmark's launch: 65536 rows x 32000 bf16 (the distill buffer's rows), beta = 1/2,
+    on the GPU at full size; 64 sampled rows are checked against the oracle."""
+    spec = W.DISTILL[4]
+    d = W.distill_inputs(spec, seed=W.seed_for(4), device="cuda")
+    g = torch.Generator(device="cuda").manual_seed(2310071779)
+    u = torch.rand(spec.N, generator=g, device="cuda")
+    gap = torch.empty(spec.N, device="cuda")
+    tok, _ = osd.osd_mixed_sample(d["draft"], d["target"], u, 0.5, cdf_gap=gap)
+    torch.cuda.synchronize()
+    sel = torch.randperm(spec.N, generator=torch.Generator().manual_seed(1))[:64]
+    z, t = d["draft"][sel.cuda()].cpu(), d["target"][sel.cuda()].cpu()
+    ref, ref_gap = oracle.mixed_sample(z, t, u[sel.cuda()].cpu(), 0.5)
+    got = tok[sel.cuda()].cpu().numpy()
+    ok = ref_gap >= TIE
+    assert np.array_equal(got[ok], ref[ok]), np.nonzero(got[ok] != ref[ok])
+    assert np.all(np.abs(gap[sel.cuda()].cpu().numpy()[ok] - ref_gap[ok]) <= 2e-6)
+    assert bool(((tok >= 0) & (tok < spec.V)).all())
 
 
 def test_strided_and_broadcast_rows(osd):

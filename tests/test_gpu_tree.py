@@ -89,6 +89,14 @@ def test_matches_oracle(osd, tree, B, V, dtype, T):
     _check(osd, inp, T)
 
 
+def test_workload_full_size(osd):
+    """The benchmark's tree workload exactly as it launches it: B=32 sequences over the
+    27-node tree, V=32000 bf16, T=1, every sequence checked against the oracle."""
+    inp = W.tree_inputs(32, W.MEDUSA_TREE, 32000, torch.bfloat16, 1.0, seed=2310071778, target_noise=0.8)
+    ties = _check(osd, inp, 1.0)
+    print(f"tree workload: {ties} of 32 sequences near a tie")
+
+
 def test_acceptance_reaches_every_depth(osd):
     """On draft == target logits every first child passes: the walk follows
     first children to a leaf."""
