@@ -97,6 +97,16 @@ def test_workload_full_size(osd):
     print(f"tree workload: {ties} of 32 sequences near a tie")
 
 
+@pytest.mark.parametrize("extreme", ["zero", "below_one"])
+def test_extreme_uniforms(osd, extreme):
+    """Every uniform at 0, or at the largest float below 1: the tree's draws at the ends
+    of the CDF, against the oracle."""
+    inp = W.tree_inputs(16, W.MEDUSA_TREE, 5000, torch.bfloat16, 1.0, seed=77, target_noise=0.8)
+    val = 0.0 if extreme == "zero" else float(np.nextafter(np.float32(1.0), np.float32(0.0)))
+    inp["uniforms"] = torch.full_like(inp["uniforms"], val)
+    _check(osd, inp, 1.0)
+
+
 def test_acceptance_reaches_every_depth(osd):
     """On draft == target logits every first child passes: the walk follows
     first children to a leaf."""

@@ -187,6 +187,22 @@ def test_gpu_output_distribution_equals_target(osd, T, V, k):
         assert abs(acc / reach - alpha) < 5 * math.sqrt(alpha * (1 - alpha) / reach)
 
 
+@pytest.mark.parametrize("V,dtype", [(1000, torch.float32), (32000, torch.bfloat16), (4099, torch.bfloat16)])
+def test_extreme_uniforms(osd, V, dtype):
+    """The extra-token draw at u = 0 (the first positive weight) and at the largest float
+    below 1 (tau next to W), and accept tests at both ends, against the oracle."""
+    spec = W.VerifySpec(64, 3, V, dtype, 2.0, 0.8, 1.2, 1.0)
+    inp = W.verify_inputs(spec, seed=500 + V)
+    u = inp["uniforms"]
+    below_one = float(np.nextafter(np.float32(1.0), np.float32(0.0)))
+    u[0::2, :] = 0.0
+    u[1::2, -1] = below_one
+    u[1::4, :-1] = below_one
+    res, ref = _run(osd, inp, 1.0)
+    check_verify(res, ref, spec.k, V)
+    check_margins(res, ref)
+
+
 def test_gpu_expected_length_eq1(osd):
     """Eq. 1 on the GPU's own decisions: the same (p, q) at every position gives
     E[a + 1] = (1 - alpha^(k+1)) / (1 - alpha), alpha = sum min(p, q)."""
