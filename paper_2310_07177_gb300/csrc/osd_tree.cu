@@ -8,8 +8,8 @@
 //                      every vocabulary slice of every node's draft and target
 //                      row (the argmax at T = 0): the one pass over all logits.
 //   tree_walk_kernel   one thread-block cluster per sequence walks the tree from
-//                      the root.  At a node it merges the slice statistics of the
-//                      node's two rows, then tests the children in index order
+//                      the root.  It merges every node's slice statistics up
+//                      front; at a node it tests the children in index order
 //                      with the accept rule of Appendix A.1 against the current
 //                      residual.  After j rejections the residual is
 //                      norm(max(0, p - s_j q)) with s_0 = 0 and s_{j+1} = s_j + N_j,
@@ -19,7 +19,8 @@
 //                      moves the walk to the child.  When no child passes, the
 //                      extra token is drawn from max(0, p - s q) by inverse CDF
 //                      from the sub-tile sums of the last pass, as the verifier's
-//                      finalize kernel draws its residual token.
+//                      finalize kernel draws its residual token (masses summed in
+//                      exact 64-bit fixed point).
 #include <algorithm>
 #include <climits>
 #include <cmath>
