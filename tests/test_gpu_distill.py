@@ -231,6 +231,26 @@ def _sampled_full(osd, cfg, kind, beta, n_sample=48):
     return rep
 
 
+@pytest.mark.parametrize("kind", KINDS)
+def test_many_rows_long_spans_sampled(osd, kind):
+    """More rows than SMs at V = 100000 bf16: full-length spans of 12544 entries, which every
+    kind but TVD runs on 256-thread CTAs; 8 sampled rows against the oracle."""
+    N, V = 200, 100000
+    spec = W.DistillSpec(N, V, torch.bfloat16, 2.0, "draft+noise", 1.5, 1.0)
+    inp = W.distill_inputs(spec, seed=4242, device="cuda")
+    z, t = inp["draft"], inp["target"]
+    dl = torch.full((N, V), float("nan"), device="cuda")
+    beta = 0.3 if kind == "jsd" else 0.5
+    loss, g = osd.osd_distill(z, t, None, kind, beta, dlogits=dl, temperature=0.9)
+    torch.cuda.synchronize()
+    idx = torch.tensor(sorted(np.random.default_rng(7).choice(N, 8, replace=False)), device="cuda")
+    zs, ts = z[idx].cpu(), t[idx].cpu()
+    lr, gr = _oracle(zs, ts, None, kind, beta, tau=0.9)
+    skip = _tvd_ambiguous(zs, ts, 0.9) if kind == "tvd" else None
+    check_distill(loss[idx].cpu().numpy(), g[idx].cpu().numpy(), lr, gr, np.ones(8, bool), skip)
+    assert not torch.isnan(g).any()
+
+
 def test_workload_flush_jsd_sampled(osd):
     print(_sampled_full(osd, 3, "jsd", 0.5))
 
