@@ -641,7 +641,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     ap.add_argument("--no-extras", action="store_true",
-                    help="skip the kernels timed outside the step (mixed sampling)")
+                    help="skip the kernels timed outside the step (mixed sampling, tree verification)")
     ap.add_argument("--distill-rows", type=int, default=None,
                     help="override the distill buffer size N (small cases for profiling)")
     args = ap.parse_args()
