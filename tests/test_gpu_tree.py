@@ -151,6 +151,18 @@ def test_gpu_root_token_follows_the_target(osd):
     assert pval > 1e-4, (counts, p * n)
 
 
+def test_empty_batch_and_root_only_tree(osd):
+    dev = torch.device("cuda")
+    e = torch.empty(0, 3, 16, device=dev)
+    res = osd.osd_verify_tree(e, e, [-1, 0, 0], torch.empty(0, 3, dtype=torch.int32, device=dev),
+                              torch.empty(0, 3, device=dev), 1.0)
+    assert res.accepted.numel() == 0 and res.out_tokens.numel() == 0
+    # a tree of the root alone: nothing to test, the extra token is drawn from p at the root
+    inp = W.tree_inputs(24, [-1], 700, torch.float32, 1.0, seed=5)
+    ties = _check(osd, inp, 1.0)
+    assert ties < 24
+
+
 def test_bad_tokens(osd):
     par = [-1, 0, 0, 1]
     inp = W.tree_inputs(3, par, 50, torch.float32, 1.0, seed=1)
