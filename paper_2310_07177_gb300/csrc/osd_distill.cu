@@ -37,6 +37,7 @@ constexpr int kDistMaxCluster = 8;
 constexpr int kDistSpanBytes = 32768;         // target bytes of both rows per CTA
 constexpr int kDistSpanBytesJsd = 49152;      // JSD, bound by its ex2/lg2 work, does best with fewer, longer spans
 constexpr int kDistMaxSmem = 192 * 1024;      // largest staging buffer per CTA
+constexpr float kMinNormal = 1.17549435e-38f;  // smallest normal fp32
 
 struct DistParams {
     const void* draft;
@@ -562,24 +563,14 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
                         b = add2(qj, qq);   // 2q where q >= p, else 0 (exact): into 2 Q+
                         c2 = sub2(qj, qq);  // 2q where q < p, else 0: into 2 Q-
                     } else {
-                        const float2 d = sub2(v, u);
-                        float r[2][2];
-                        const float uu[2] = {u.x, u.y}, vv[2] = {v.x, v.y}, dd[2] = {d.x, d.y};
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            const float ad = fabsf(dd[h]);
-                            const float big = ex2(fmaxf(uu[h], vv[h]));
-                            const float rho = ex2(-ad);  // smaller / larger of p, q
-                            const bool pbig = dd[h] <= 0.f;
-                            const float wbig = pbig ? beta : 1.f - beta;
-                            const float L = lg2(fmaf(1.f - wbig, rho, wbig));  // log2(m / larger)
-                            const float pj = pbig ? big : big * rho;
-                            const float qj = pbig ? big * rho : big;
-                            r[h][0] = -pj * (pbig ? L : L + ad);
-                            r[h][1] = -qj * (pbig ? L + ad : L);
-                        }
-                        a = make_float2(r[0][0], r[1][0]);
-                        b = make_float2(r[0][1], r[1][1]);
+                        // p log2(p/m), q log2(q/m): log2 p, log2 q exact from the logits, log2 m
+                        // by one lg2 (m floored at the smallest normal, where lg2 would flush;
+                        // the entry's p and q are negligible there)
+                        const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
+                        const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
+                        const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
+                        a = mul2(pj, sub2(u, lm));
+                        b = mul2(qj, sub2(v, lm));
                     }
                     if (!two) { a.y = 0.f; b.y = 0.f; c2.y = 0.f; }
                     A2 = add2(A2, a);
@@ -685,19 +676,13 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
                     if (jsd_trivial) {
                         gg = f2(0.f);
                     } else {
-                        const float2 d = sub2(v, fma2(tdiff(e, st.mt), f2(c), cus));  // log2 q - log2 p
-                        const float dd[2] = {d.x, d.y};
-                        float l2mq[2];
-#pragma unroll
-                        for (int h = 0; h < 2; ++h) {
-                            const float ad = fabsf(dd[h]);
-                            const float rho = ex2(-ad);
-                            const bool pbig = dd[h] <= 0.f;
-                            const float wbig = pbig ? beta : 1.f - beta;
-                            const float L = lg2(fmaf(1.f - wbig, rho, wbig));
-                            l2mq[h] = pbig ? L + ad : L;
-                        }
-                        gg = mul2(qj, make_float2(-l2mq[0] - s2.b, -l2mq[1] - s2.b));
+                        // q (log2(q/m) - S), every probability here carrying the gradient's
+                        // factor, which cancels in log2(q/m)
+                        const float2 u = fma2(tdiff(e, st.mt), f2(c), cus);
+                        const float2 pj = make_float2(ex2(u.x), ex2(u.y));
+                        const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
+                        const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
+                        gg = mul2(qj, sub2(sub2(v, lm), f2(s2.b)));
                     }
                 }
                 gr[e] = gg.x;
