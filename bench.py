@@ -236,8 +236,10 @@ def run_ours(args):
         sd = setup["spec_d"]
         dl = torch.empty(sd.N, sd.V, dtype=torch.float32, device=dev)
         loss = torch.empty(sd.N, dtype=torch.float32, device=dev)
-        kinds = ["rkl", "tvd"]
-        dist_pos = 2 * sd.N
+        kinds = args.distill_kinds.split(",")
+        if kinds != ["rkl", "tvd"]:
+            setup["desc"] = setup["desc"].replace("reverse-KL + TVD", " + ".join(k.upper() for k in kinds))
+        dist_pos = len(kinds) * sd.N
         dist_bytes = sd.N * sd.V * (2 * 2 + 4)  # per launch
     else:
         kinds = []
@@ -346,8 +348,9 @@ def run_ours(args):
     achieved = kernels[top]["gbs"]
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                 "frac": round(achieved / peak, 4),
-                "traffic": (_traffic("distill", DISTILL_SOURCES) if top == "distill"
-                            else _traffic("verify", VERIFY_SOURCES)),
+                # the distill counters were taken on the RKL and TVD launches of the default step
+                "traffic": ((_traffic("distill", DISTILL_SOURCES) if kinds == ["rkl", "tvd"] else None)
+                            if top == "distill" else _traffic("verify", VERIFY_SOURCES)),
                 "kernel": "distill_kernel" if top == "distill" else "row_stats_kernel + verify_finalize_kernel",
                 "peak_source": peak_src}
 
@@ -644,7 +647,12 @@ def main():
                     help="skip the kernels timed outside the step (mixed sampling, tree verification)")
     ap.add_argument("--distill-rows", type=int, default=None,
                     help="override the distill buffer size N (small cases for profiling)")
+    ap.add_argument("--distill-kinds", default="rkl,tvd",
+                    help="loss kinds of the timed step's buffer flush, comma-separated (profiling one kind; "
+                         "the e2e and CPU legs keep RKL and TVD)")
     args = ap.parse_args()
+    if any(k not in ("fkl", "rkl", "jsd", "tvd", "ce") for k in args.distill_kinds.split(",")):
+        ap.error("--distill-kinds takes fkl, rkl, jsd, tvd, ce")
     if args.warmup < 3:
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)
     if args.impl == "reference":
