@@ -35,7 +35,7 @@ constexpr int kDistThreadsWide = 256;          // ... and for spans of kDistWide
 constexpr int kDistWideSpan = 12288;           // FKL, RKL, CE and JSD measured 5-10 % faster (V = 128256)
 constexpr int kDistMaxCluster = 8;
 constexpr int kDistSpanBytes = 32768;         // target bytes of both rows per CTA
-constexpr int kDistSpanBytesJsd = 49152;      // JSD, bound by its ex2/lg2 work, does best with fewer, longer spans
+constexpr int kDistSpanBytesJsd = 49152;      // JSD, with the most work per entry, does best with fewer, longer spans
 constexpr int kDistMaxSmem = 192 * 1024;      // largest staging buffer per CTA
 constexpr float kMinNormal = 1.17549435e-38f;  // smallest normal fp32
 
