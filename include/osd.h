@@ -53,7 +53,7 @@ extern "C" {
 typedef enum osd_status {
     OSD_OK = 0,
     OSD_ERR_INVALID_ARG = 1,  /* a null pointer, size, alignment or value out of range */
-    OSD_ERR_UNSUPPORTED = 2,  /* valid arguments beyond this build's limits (e.g. V)   */
+    OSD_ERR_UNSUPPORTED = 2,  /* valid arguments beyond the library's limits (e.g. V) */
     OSD_ERR_CUDA = 3,         /* a CUDA launch or API call failed                        */
     OSD_ERR_TIMEOUT = 4       /* a bounded device-side wait gave up (see osd_distill)    */
 } osd_status;
