@@ -225,12 +225,12 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
     constexpr bool kMoment = kKind == OSD_FKL || kKind == OSD_RKL;
     constexpr bool kNeedEt = kKind != OSD_CE;  // CE needs only the draft normaliser and the label
     constexpr bool kFold = !kClamp;            // exponent arguments by one FMA (see pass 1)
-    // chunk loops unrolled by two where that measured faster: passes 0-2 of TVD, JSD
-    // and CE (+2-3 %; FKL and RKL lose 1 %), and JSD's gradient pass (CE's gains 4 %
-    // without)
+    // chunk loops unrolled by two where that measured faster: pass 0 of every kind (with
+    // the scans below, RKL +2.3 %), passes 1-2 of TVD, JSD and CE (+2-3 %; FKL and RKL
+    // lose 1-2 %), and JSD's gradient pass (the other kinds' lose 1-4 %)
+    constexpr int kUn0 = 2;
     constexpr int kUn = (kKind == OSD_FKL || kKind == OSD_RKL) ? 1 : 2;
     constexpr int kUn3 = (kKind == OSD_JSD) ? 2 : 1;
-    constexpr int kUn0 = 2;  // pass 0 unrolls by two for every kind (with the scans below, RKL +2.3 %)
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ __align__(8) uint64_t bar;
     __shared__ Stats1 s1_mine, s1_all;
