@@ -146,6 +146,29 @@ def test_identical_rows_and_jsd_endpoints(osd):
         assert loss.abs().max().item() == 0.0 and g.abs().max().item() == 0.0
 
 
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+def test_identical_rows_peaked_and_two_mode(osd, dtype):
+    # identical rows where a few entries hold most of the mass: every kind's loss and
+    # gradient stay at the parity floor (the oracle gives exactly 0 here)
+    g0 = torch.Generator().manual_seed(21)
+    z = torch.randn(6, 32000, generator=g0)
+    z[0, 7] = 25.0                       # one entry holds almost all the mass
+    z[1, 3], z[1, 31000] = 20.0, 20.0    # two equal modes
+    z[2, 11], z[2, 12] = 14.0, 13.3      # two unequal modes
+    z[3] *= 6.0                          # broad, large logits
+    z[4, :16000] = float("-inf")         # half the vocabulary impossible
+    z[5] = z[5] * 0.01                   # nearly uniform
+    zd = z.to(dtype).cuda()
+    for kind in ("fkl", "rkl", "jsd", "tvd", "ce"):
+        for beta in ((0.1, 0.5, 0.9) if kind == "jsd" else (0.5,)):
+            loss, g = osd.osd_distill(zd, zd, None, kind, beta)
+            torch.cuda.synchronize()
+            if kind == "ce":  # CE is -log q(argmax t), not a distance: only its gradient's form is checked
+                continue
+            assert loss.abs().max().item() < 1e-6, (kind, beta, loss)
+            assert g.abs().max().item() < 1e-7, (kind, beta, g.abs().max(dim=1).values)
+
+
 def test_extreme_and_neg_inf_logits(osd):
     g0 = torch.Generator().manual_seed(9)
     z = torch.randn(5, 3000, generator=g0) * 3
