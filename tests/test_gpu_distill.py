@@ -169,6 +169,20 @@ def test_identical_rows_peaked_and_two_mode(osd, dtype):
             assert g.abs().max().item() < 1e-7, (kind, beta, g.abs().max(dim=1).values)
 
 
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
+@pytest.mark.parametrize("beta", [0.01, 0.05, 0.95, 0.99])
+def test_jsd_beta_near_the_ends(osd, beta, dtype):
+    # m = beta p + (1 - beta) q is then dominated by one side; log2(p/m) and log2(q/m)
+    # still come out against the oracle within the parity bar
+    spec = W.DistillSpec(4, 32000, dtype, 2.0, "draft+noise", 1.5, 1.0)
+    inp = W.distill_inputs(spec, seed=1234 + int(beta * 100))
+    z, t = inp["draft"], inp["target"]
+    for tau in (1.0, 0.7):
+        lg, gg = _run(osd, z, t, None, "jsd", beta, tau=tau)
+        lr, gr = _oracle(z, t, None, "jsd", beta, tau=tau)
+        check_distill(lg, gg, lr, gr, np.ones(4, bool))
+
+
 def test_extreme_and_neg_inf_logits(osd):
     g0 = torch.Generator().manual_seed(9)
     z = torch.randn(5, 3000, generator=g0) * 3
