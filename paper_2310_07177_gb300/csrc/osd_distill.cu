@@ -572,8 +572,13 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
                         const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
                         const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
                         const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
-                        a = mul2(pj, sub2(u, lm));
-                        b = mul2(qj, sub2(v, lm));
+                        // straight into the sums (the second slot of a one-entry chunk
+                        // carries no mass); JSD has no third sum
+                        const float2 pw = two ? pj : make_float2(pj.x, 0.f);
+                        const float2 qw = two ? qj : make_float2(qj.x, 0.f);
+                        A2 = fma2(pw, sub2(u, lm), A2);
+                        B2 = fma2(qw, sub2(v, lm), B2);
+                        continue;
                     }
                     if (!two) { a.y = 0.f; b.y = 0.f; c2.y = 0.f; }
                     A2 = add2(A2, a);
