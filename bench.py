@@ -14,6 +14,11 @@ The value is positions (verified + distilled) per second for the whole job.
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                     [--workload serving-32k|large-vocab]
 
+With --gpus N > 1 and no torchrun environment, the script starts N ranks
+itself (torch.distributed.run on 127.0.0.1), one per GPU; each rank draws its
+own shard of the workload (weak scaling, no collective on the data path) and
+the job time is the slowest rank's.
+
 `--workload large-vocab` times verify at B=256, k=8, V=128256, T=0.7 followed
 by forward-KL distill of its rejected rows (the 128k-vocabulary serving step).
 `--impl reference` times the CPU oracle (the correctness reference) on a
@@ -338,9 +343,12 @@ def run_ours(args):
         kernels["verify_greedy"] = {"us_per_call": avg_g * 1e3, "alg_bytes": bytes_g,
                                     "gbs": bytes_g / (avg_g / 1e3) / 1e9,
                                     "positions_per_s": sv.B * sv.k / (avg_g / 1e3)}
-    if wl == "serving-32k" and not args.no_extras:
-        kernels["mixed_sample"] = _time_mixed_sample(osd, d, sd, l2_flush, stream, reps=max(3, args.steps // 2))
-        kernels["tree_verify"] = _time_tree_verify(osd, dev, l2_flush, stream, reps=max(3, args.steps // 2))
+    if wl == "serving-32k" and not args.no_extras and rank == 0:
+        reps = max(3, args.steps // 2)
+        kernels["mixed_sample"] = _time_mixed_sample(osd, d, sd, l2_flush, stream, reps=reps)
+        kernels["tree_verify"] = _time_tree_verify(osd, dev, l2_flush, stream, reps=reps)
+        kernels.update(_time_large_vocab(osd, dev, l2_flush, stream, reps=max(5, args.steps)))
+        kernels["distill_jsd_masked"] = _time_jsd_flush(osd, dev, l2_flush, stream, reps=max(5, args.steps))
     for kv in kernels.values():
         kv["frac_of_peak"] = kv["gbs"] / peak
     # the dominant kernel: distill on the default step, verify's row statistics at 128k
@@ -355,7 +363,7 @@ def run_ours(args):
                 "peak_source": peak_src}
 
     e2e = None
-    if not args.no_e2e and (world == 1 or rank == 0):
+    if not args.no_e2e:  # every rank runs it (h2d and d2h are per rank), timed over the job
         e2e = run_e2e(args, osd, setup, dev, stream, positions, wl)
     cpu = cpu_baseline(args, setup) if (rank == 0 and world == 1 and not args.no_cpu_baseline) else None
 
@@ -405,6 +413,76 @@ def _time_mixed_sample(osd, d, sd, l2_flush, stream, reps):
     alg = sd.N * sd.V * 2 * 2 + sd.N * 8  # both bf16 rows, the uniform and the token
     return {"us_per_call": avg * 1e3, "alg_bytes": alg, "gbs": alg / (avg / 1e3) / 1e9,
             "positions_per_s": sd.N / (avg / 1e3), "in_step": False, "beta": 0.5}
+
+
+def _timed(fn, l2_flush, stream, reps, warm=2):
+    """Mean CUDA-event time (ms) of fn() on `stream`, L2 flushed and the device
+    kept busy (so that host enqueue time stays outside the events) before each."""
+    import torch
+    ms = []
+    for i in range(reps + warm):
+        l2_flush.zero_()
+        torch.cuda._sleep(SLEEP_CYCLES)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        b.synchronize()
+        if i >= warm:
+            ms.append(a.elapsed_time(b))
+    return statistics.mean(ms)
+
+
+def _time_large_vocab(osd, dev, l2_flush, stream, reps):
+    """The 128k-vocabulary serving step's two calls, each timed on its own with L2
+    flushed before it: verify at B=256, k=8, V=128256 bf16, T=0.7 (the largest
+    verify workload), then the forward-KL distillation of the rows it rejected,
+    selected and compacted on the device (osd_distill_accepted)."""
+    import torch
+    from paper_2310_07177_gb300 import workloads as W
+    sv = W.VERIFY[5]
+    v = W.verify_inputs(sv, seed=W.seed_for(5), device=dev)
+    ws = torch.empty(osd.osd_verify_workspace_size(sv.B, sv.k, sv.V), dtype=torch.uint8, device=dev)
+    out = osd.osd_verify(v["draft"], v["target"], v["tokens"], v["uniforms"], sv.temperature, workspace=ws)
+    rej = osd.osd_distill_accepted(v["draft"], v["target"], out.accepted, "fkl", 0.5)
+    torch.cuda.synchronize()
+    n_rej = int(rej.count.item())
+    t_v = _timed(lambda: osd.osd_verify(v["draft"], v["target"], v["tokens"], v["uniforms"], sv.temperature,
+                                        workspace=ws, out=out), l2_flush, stream, reps)
+    t_d = _timed(lambda: osd.osd_distill_accepted(v["draft"], v["target"], out.accepted, "fkl", 0.5, out=rej),
+                 l2_flush, stream, reps)
+    bv = _bytes_verify(sv.B, sv.k, sv.V, 2, False)
+    bd = n_rej * sv.V * (2 * 2 + 4) + sv.B * 4
+    res = {
+        "verify_large_vocab": {"us_per_call": t_v * 1e3, "alg_bytes": bv, "gbs": bv / (t_v / 1e3) / 1e9,
+                               "positions_per_s": sv.B * sv.k / (t_v / 1e3), "in_step": False,
+                               "workload": "B=256 k=8 V=128256 bf16 T=0.7"},
+        "distill_rejected_large_vocab": {"us_per_call": t_d * 1e3, "alg_bytes": bd, "rows": n_rej,
+                                         "gbs": bd / (t_d / 1e3) / 1e9, "positions_per_s": n_rej / (t_d / 1e3),
+                                         "in_step": False, "kind": "fkl",
+                                         "workload": "the rows the verify above rejected, V=128256 bf16"},
+    }
+    del v, ws, out, rej
+    return res
+
+
+def _time_jsd_flush(osd, dev, l2_flush, stream, reps):
+    """The 16384 x 32128 buffer flush: generalised JSD (beta = 1/2) loss and
+    gradient under its 40 % mask, timed on its own with L2 flushed before it."""
+    import torch
+    from paper_2310_07177_gb300 import workloads as W
+    spec = W.DISTILL[3]
+    inp = W.distill_inputs(spec, seed=W.seed_for(3), device=dev)
+    loss = torch.empty(spec.N, dtype=torch.float32, device=dev)
+    dl = torch.empty(spec.N, spec.V, dtype=torch.float32, device=dev)
+    n_on = int(inp["mask"].sum().item())
+    t = _timed(lambda: osd.osd_distill(inp["draft"], inp["target"], inp["mask"], "jsd", 0.5, loss=loss,
+                                       dlogits=dl), l2_flush, stream, reps)
+    alg = n_on * spec.V * (2 * 2 + 4)
+    del inp, loss, dl
+    return {"us_per_call": t * 1e3, "alg_bytes": alg, "rows": n_on, "gbs": alg / (t / 1e3) / 1e9,
+            "positions_per_s": n_on / (t / 1e3), "in_step": False,
+            "workload": f"N={spec.N} V={spec.V} bf16, {n_on} rows active (40 % mask), JSD beta=0.5"}
 
 
 def _time_tree_verify(osd, dev, l2_flush, stream, reps):
@@ -475,8 +553,10 @@ def run_e2e(args, osd, setup, dev, stream, positions, wl):
         loss = torch.empty(sd.N, dtype=torch.float32, device=dev)
         dl = torch.empty(sd.N, sd.V, dtype=torch.float32, device=dev)
         h_loss = torch.empty(2, sd.N, dtype=torch.float32).pin_memory()
+        # the greedy pass's results land in pinned buffers of their own, next to the T=1 pass's
+        h_out0 = {key: torch.empty_like(val).pin_memory() for key, val in h_out.items()}
         h2d += sum(t.numel() * t.element_size() for t in hd.values())
-        d2h += h_out["acc"].numel() * 4 + h_out["tok"].numel() * 4 + h_out["mask"].numel() + h_loss.numel() * 4
+        d2h += sum(t.numel() * t.element_size() for t in h_out0.values()) + h_loss.numel() * 4
 
     copy_stream = torch.cuda.Stream(dev)
     copied = [torch.cuda.Event() for _ in range(nbuf)]
@@ -509,9 +589,9 @@ def run_e2e(args, osd, setup, dev, stream, positions, wl):
         h_rej["count"].copy_(rej.count, non_blocking=True)
         if wl == "serving-32k":
             r0 = osd.osd_verify(None, x["target"], x["greedy_tokens"], None, 0.0, workspace=ws)
-            h_out["acc"].copy_(r0.accepted, non_blocking=True)
-            h_out["tok"].copy_(r0.out_tokens, non_blocking=True)
-            h_out["mask"].copy_(r0.mismatch_mask, non_blocking=True)
+            h_out0["acc"].copy_(r0.accepted, non_blocking=True)
+            h_out0["tok"].copy_(r0.out_tokens, non_blocking=True)
+            h_out0["mask"].copy_(r0.mismatch_mask, non_blocking=True)
             for i2, kind in enumerate(("rkl", "tvd")):
                 osd.osd_distill(xd["draft"], xd["target"], None, kind, 0.5, loss=loss, dlogits=dl)
                 h_loss[i2].copy_(loss, non_blocking=True)
@@ -527,13 +607,18 @@ def run_e2e(args, osd, setup, dev, stream, positions, wl):
     steps(max(2, args.warmup))
     torch.cuda.synchronize()
     n = max(3, args.steps // 2)
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if world > 1:
+        torch.distributed.barrier()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(copy_stream)  # before the first upload
     steps(n)
     e1.record(stream)       # after the last step's kernels and read-backs
     e1.synchronize()
-    ms = e0.elapsed_time(e1) / n
-    return {"value": round(positions / (ms / 1e3), 1), "unit": "positions/s", "h2d_bytes_per_step": int(h2d),
+    # whole job: every rank ran its own shard; the slowest rank's time counts
+    ms = job_time_ms(e0.elapsed_time(e1), dev if world > 1 else None) / n
+    return {"value": round(job_throughput(positions, world, ms), 1), "unit": "positions/s",
+            "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(d2h), "ms_per_step": round(ms, 3), "steps": n,
             "pipelined": "step i+1's upload overlaps step i's kernels (two device buffer sets, a copy stream)",
             "note": "dlogits stays on the device, where the draft model's backward pass consumes it"}
@@ -588,14 +673,41 @@ def _oracle_step_time(setup, n_rows, threads):
     return time.perf_counter() - t0, positions
 
 
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the platform)."""
+    import platform
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.split(":")[0].strip() == "Model name":
+                return f"{line.split(':', 1)[1].strip()} ({platform.machine()})"
+    except Exception:
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return f"{line.split(':', 1)[1].strip()} ({platform.machine()})"
+    except Exception:
+        pass
+    return platform.processor() or platform.machine()
+
+
 def cpu_baseline(args, setup):
     threads = os.cpu_count() or 1
     n_rows = args.cpu_rows
     secs, pos = _oracle_step_time(setup, n_rows, threads)
+    # one thread on a smaller sample of the same mix (a few seconds)
+    n1 = max(64, n_rows // 32)
+    secs1, pos1 = _oracle_step_time(setup, n1, 1)
     return {"value": round(pos / secs, 2), "unit": "positions/s", "cores": threads, "kind": "oracle",
             "sample": f"whole verify batch (both passes, with its rejected rows distilled) + {n_rows} "
                       f"distill rows per loss kind, "
-                      f"{secs:.1f} s on {threads} host threads (double-precision C oracle)"}
+                      f"{secs:.1f} s on {threads} host threads (double-precision C oracle)",
+            "single_thread": {"value": round(pos1 / secs1, 2), "unit": "positions/s", "cores": 1,
+                              "sample": f"whole verify batch + {n1} distill rows per loss kind, "
+                                        f"{secs1:.1f} s on one thread"},
+            "cpu_model": cpu_model()}
 
 
 def run_reference(args):
@@ -632,6 +744,44 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+# ----------------------------------------------------------------------------- launcher
+def _free_port() -> int:
+    import socket
+    with socket.socket(socket.AF_INET, socket.SOCK_STREAM) as sock:
+        sock.bind(("127.0.0.1", 0))
+        return sock.getsockname()[1]
+
+
+def launch_ranks(n: int, argv) -> int:
+    """Start this script as n ranks on this node (torch.distributed.run, one
+    process per GPU, rendezvous on 127.0.0.1) and return their exit status."""
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={n}",
+           "--master-addr", "127.0.0.1", f"--master-port={_free_port()}", os.path.abspath(__file__), *argv]
+    return subprocess.call(cmd)
+
+
+def run_launcher_check(args):
+    """CPU-only check of the multi-rank plumbing (gloo, no GPU): every rank
+    times its own stand-in step (rank r sleeps (r + 1) ms), the job time is the
+    slowest rank's, and rank 0 prints the line with the number of ranks."""
+    import torch.distributed as dist
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if world > 1:
+        dist.init_process_group("gloo")
+    local = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        time.sleep(1e-3 * (rank + 1))
+        local.append((time.perf_counter() - t0) * 1e3)
+    ms = job_time_ms(sum(local)) / args.steps
+    if rank == 0:
+        print(json.dumps({"check": "launcher", "n_gpus": world, "steps": args.steps, "ms_per_step": round(ms, 4),
+                          "value": job_throughput(1, world, ms), "scaling": "weak"}), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -650,7 +800,18 @@ def main():
     ap.add_argument("--distill-kinds", default="rkl,tvd",
                     help="loss kinds of the timed step's buffer flush, comma-separated (profiling one kind; "
                          "the e2e and CPU legs keep RKL and TVD)")
+    ap.add_argument("--launcher-check", action="store_true",
+                    help="CPU-only check of the multi-rank launcher (gloo ranks, no GPU work)")
     args = ap.parse_args()
+    if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
+        # not started under torchrun: start the N ranks here, one process per GPU
+        sys.exit(launch_ranks(args.gpus, sys.argv[1:]))
+    if "WORLD_SIZE" in os.environ and int(os.environ["WORLD_SIZE"]) != args.gpus:
+        print(f"warning: --gpus {args.gpus} but WORLD_SIZE={os.environ['WORLD_SIZE']}; the ranks decide",
+              file=sys.stderr)
+    if args.launcher_check:
+        run_launcher_check(args)
+        return
     if any(k not in ("fkl", "rkl", "jsd", "tvd", "ce") for k in args.distill_kinds.split(",")):
         ap.error("--distill-kinds takes fkl, rkl, jsd, tvd, ce")
     if args.warmup < 3:

@@ -150,10 +150,16 @@ osd_status osd_verify(const void *draft_logits, const void *target_logits,
  * nothing: no cudaMalloc, cudaFree or allocating library call.
  *   - The first call on a device looks up that device's copy of the array
  *     (cudaGetSymbolAddress, with the device current); make that first call
- *     before any stream capture.
+ *     before any stream capture.  The address is kept per device together with
+ *     the ID of the context it was found in, and looked up again when the
+ *     current context changes (after cudaDeviceReset, for instance); make the
+ *     first call after such a change before any stream capture too.
  *   - Returns OSD_ERR_UNSUPPORTED when osd_verify_workspace_size(B, k, V)
- *     exceeds 4 MiB (B * (2k+1) * ceil(V / 8192) * 16 bytes), or when the
- *     current device ordinal is 64 or more.
+ *     exceeds 4 MiB, or when the current device ordinal is 64 or more.  That
+ *     size is B * (2k+1) * ceil(V / L) * 16 bytes, rounded up to 256, with
+ *     slices of L = 8192 entries below 512 rows B * (2k+1), 16384 below
+ *     2048 rows and 32768 from 2048 rows on (B = 256, k = 8, V = 128256 needs
+ *     0.28 MB).
  *   - All calls on a device share the one array, which keeps the last call's
  *     contents (every entry is rewritten before it is read, so nothing needs
  *     clearing).  Calls that overlap on the GPU, on different streams or from

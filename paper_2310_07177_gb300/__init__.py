@@ -13,6 +13,7 @@ no CPU path.  If the library has not been built, calls raise immediately.
 """
 from __future__ import annotations
 
+import contextlib
 import ctypes
 import os
 from typing import NamedTuple, Optional
@@ -115,6 +116,15 @@ def _stream(device, stream):
     return ctypes.c_void_p(s.cuda_stream)
 
 
+def _on(dev):
+    """Make ``dev`` the current device for a library call: the C functions work
+    on the current device (its workspace, its streams), which need not be the
+    device the tensors live on."""
+    if dev is None or dev.index is None or torch.cuda.current_device() == dev.index:
+        return contextlib.nullcontext()
+    return torch.cuda.device(dev)
+
+
 def _need_cuda(*ts):
     dev = None
     for t in ts:
@@ -173,10 +183,11 @@ def osd_verify(draft_logits: torch.Tensor, target_logits: torch.Tensor, draft_to
             torch.empty(B, k, dtype=torch.uint8, device=dev),
             torch.empty(B, k, dtype=torch.float32, device=dev) if diagnostics else None,
             torch.empty(B, dtype=torch.float32, device=dev) if diagnostics else None)
-    st = lib.osd_verify(_ptr(draft_logits), _ptr(target_logits), dt, B, k, V, _ptr(draft_tokens),
-                        _ptr(uniforms), float(temperature), _ptr(out.accepted), _ptr(out.out_tokens),
-                        _ptr(out.mismatch_mask), _ptr(out.diag_margin), _ptr(out.diag_cdf_gap),
-                        _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(dev, stream))
+    with _on(dev):
+        st = lib.osd_verify(_ptr(draft_logits), _ptr(target_logits), dt, B, k, V, _ptr(draft_tokens),
+                            _ptr(uniforms), float(temperature), _ptr(out.accepted), _ptr(out.out_tokens),
+                            _ptr(out.mismatch_mask), _ptr(out.diag_margin), _ptr(out.diag_cdf_gap),
+                            _ptr(workspace), workspace.numel() * workspace.element_size(), _stream(dev, stream))
     if st != OSD_OK:
         raise OsdError(st, "osd_verify")
     return out
@@ -191,10 +202,11 @@ def osd_verify_noalloc(draft_logits: torch.Tensor, target_logits: torch.Tensor, 
     lib = load_library()
     B, k1, V = target_logits.shape
     dev = _need_cuda(draft_logits, target_logits, draft_tokens, uniforms, *out)
-    st = lib.osd_verify_noalloc(_ptr(draft_logits), _ptr(target_logits), _dtype_code(target_logits), B, k1 - 1, V,
-                                _ptr(draft_tokens), _ptr(uniforms), float(temperature), _ptr(out.accepted),
-                                _ptr(out.out_tokens), _ptr(out.mismatch_mask), _ptr(out.diag_margin),
-                                _ptr(out.diag_cdf_gap), _stream(dev, stream))
+    with _on(dev):
+        st = lib.osd_verify_noalloc(_ptr(draft_logits), _ptr(target_logits), _dtype_code(target_logits), B, k1 - 1, V,
+                                    _ptr(draft_tokens), _ptr(uniforms), float(temperature), _ptr(out.accepted),
+                                    _ptr(out.out_tokens), _ptr(out.mismatch_mask), _ptr(out.diag_margin),
+                                    _ptr(out.diag_cdf_gap), _stream(dev, stream))
     if st != OSD_OK:
         raise OsdError(st, "osd_verify_noalloc")
     return out
@@ -243,10 +255,11 @@ def osd_distill(draft_logits: torch.Tensor, target_logits: torch.Tensor, mask: O
             or tuple(dlogits.shape) != lead + (V,)):
         raise ValueError("loss / dlogits must be contiguous float32 of the logits' shape")
     kind = LOSS_KINDS[loss_kind] if isinstance(loss_kind, str) else int(loss_kind)
-    st = lib.osd_distill(_ptr(draft_logits), _ptr(target_logits), _dtype_code(draft_logits), G, P, V,
-                         dsg, dsp, tsg, tsp, _ptr(mask), kind, float(beta), float(temperature), _ptr(loss),
-                         _ptr(dlogits),
-                         _ptr(status), _stream(dev, stream))
+    with _on(dev):
+        st = lib.osd_distill(_ptr(draft_logits), _ptr(target_logits), _dtype_code(draft_logits), G, P, V,
+                             dsg, dsp, tsg, tsp, _ptr(mask), kind, float(beta), float(temperature), _ptr(loss),
+                             _ptr(dlogits),
+                             _ptr(status), _stream(dev, stream))
     if st != OSD_OK:
         raise OsdError(st, "osd_distill")
     return loss, dlogits
@@ -287,10 +300,11 @@ def osd_distill_accepted(draft_logits: torch.Tensor, target_logits: torch.Tensor
                                     torch.empty(B, dtype=torch.int32, device=dev),
                                     torch.empty(1, dtype=torch.int32, device=dev))
     kind = LOSS_KINDS[loss_kind] if isinstance(loss_kind, str) else int(loss_kind)
-    st = lib.osd_distill_accepted(_ptr(draft_logits), _ptr(target_logits), _dtype_code(draft_logits), B, k, V,
-                                  _ptr(accepted), kind, float(beta), float(temperature), _ptr(out.loss),
-                                  _ptr(out.dlogits), _ptr(out.seq_of_row), _ptr(out.count), _ptr(status),
-                                  _stream(dev, stream))
+    with _on(dev):
+        st = lib.osd_distill_accepted(_ptr(draft_logits), _ptr(target_logits), _dtype_code(draft_logits), B, k, V,
+                                      _ptr(accepted), kind, float(beta), float(temperature), _ptr(out.loss),
+                                      _ptr(out.dlogits), _ptr(out.seq_of_row), _ptr(out.count), _ptr(status),
+                                      _stream(dev, stream))
     if st != OSD_OK:
         raise OsdError(st, "osd_distill_accepted")
     return out
@@ -323,9 +337,10 @@ def osd_mixed_sample(draft_logits: torch.Tensor, target_logits: torch.Tensor, un
         raise ValueError("uniforms must be contiguous float32 [N]")
     if tokens is None:
         tokens = torch.empty(N, dtype=torch.int32, device=dev)
-    st = lib.osd_mixed_sample(_ptr(draft_logits), _ptr(target_logits), _dtype_code(draft_logits), N, V, ds, tsd,
-                              _ptr(uniforms), float(beta), float(temperature), _ptr(tokens), _ptr(cdf_gap),
-                              _ptr(status), _stream(dev, stream))
+    with _on(dev):
+        st = lib.osd_mixed_sample(_ptr(draft_logits), _ptr(target_logits), _dtype_code(draft_logits), N, V, ds, tsd,
+                                  _ptr(uniforms), float(beta), float(temperature), _ptr(tokens), _ptr(cdf_gap),
+                                  _ptr(status), _stream(dev, stream))
     if st != OSD_OK:
         raise OsdError(st, "osd_mixed_sample")
     return tokens, cdf_gap
@@ -382,11 +397,12 @@ def osd_verify_tree(draft_logits: Optional[torch.Tensor], target_logits: torch.T
                          torch.empty(B, n, dtype=i32, device=dev), torch.empty(B, dtype=i32, device=dev),
                          torch.empty(B, n, dtype=torch.float32, device=dev) if diagnostics else None,
                          torch.empty(B, dtype=torch.float32, device=dev) if diagnostics else None)
-    st = lib.osd_verify_tree(_ptr(draft_logits), _ptr(target_logits), _dtype_code(target_logits), B, n, V, par,
-                             _ptr(tokens), _ptr(uniforms), float(temperature), _ptr(out.accepted), _ptr(out.path),
-                             _ptr(out.out_tokens), _ptr(out.last_node), _ptr(out.diag_margin),
-                             _ptr(out.diag_cdf_gap), _ptr(workspace), workspace.numel() * workspace.element_size(),
-                             _stream(dev, stream))
+    with _on(dev):
+        st = lib.osd_verify_tree(_ptr(draft_logits), _ptr(target_logits), _dtype_code(target_logits), B, n, V, par,
+                                 _ptr(tokens), _ptr(uniforms), float(temperature), _ptr(out.accepted), _ptr(out.path),
+                                 _ptr(out.out_tokens), _ptr(out.last_node), _ptr(out.diag_margin),
+                                 _ptr(out.diag_cdf_gap), _ptr(workspace), workspace.numel() * workspace.element_size(),
+                                 _stream(dev, stream))
     if st != OSD_OK:
         raise OsdError(st, "osd_verify_tree")
     return out
@@ -400,7 +416,8 @@ def osd_check_bounded_wait(limit_us: int, *, device=None, stream: Optional[torch
     dev = torch.device("cuda") if device is None else torch.device(device)
     st = torch.full((1,), -1, dtype=torch.int32, device=dev)
     waited = torch.zeros(1, dtype=torch.int64, device=dev)
-    rc = lib.osd_check_bounded_wait(int(limit_us), _ptr(st), _ptr(waited), _stream(dev, stream))
+    with _on(dev):
+        rc = lib.osd_check_bounded_wait(int(limit_us), _ptr(st), _ptr(waited), _stream(dev, stream))
     if rc != OSD_OK:
         raise OsdError(rc, "osd_check_bounded_wait")
     return int(st.item()), int(waited.item())

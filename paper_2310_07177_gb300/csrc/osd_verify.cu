@@ -26,6 +26,8 @@
 // The log-ratio of the accept test is formed from differences of raw logits and
 // maxima, (t_y - m_t) - (z_y - m_z), and the ratio of the two sums, so no
 // log-sum-exp is rounded on its own.
+#include <cuda.h>
+
 #include <climits>
 #include <cstdint>
 #include <mutex>
@@ -502,9 +504,13 @@ static int verify_slices(int B, int k, int V) {
 
 // CTAs per sequence: up to 8 for few sequences (short spans, low latency); 4 past
 // 128 sequences, where 8 would leave more clusters than fit on the GPU at once and
-// the second wave would wait out the first one's latency phases.
-static void finalize_shape(int B, int V, int* csize, int* span) {
-    const int cmax = (B > 128) ? kFinMaxCluster / 2 : kFinMaxCluster;
+// the second wave would wait out the first one's latency phases.  A span must fit
+// in kFinMaxSub sub-tiles of `sub` entries: the element-wise path (32-entry
+// sub-tiles) takes 8 CTAs at any B once V passes 4 * 8192 * 32 = 2^20.
+static void finalize_shape(int B, int V, int sub, int* csize, int* span) {
+    int cmax = (B > 128) ? kFinMaxCluster / 2 : kFinMaxCluster;
+    const long long per_cta = (long long)kFinMaxSub * sub;
+    if ((long long)cmax * per_cta < V) cmax = kFinMaxCluster;
     int c = (V + 4095) / 4096;
     c = c < 1 ? 1 : (c > cmax ? cmax : c);
     int s = (V + c - 1) / c;
@@ -553,13 +559,13 @@ static osd_status launch_verify(const void* draft, const void* target, int B, in
         const dim3 grid_g(unsigned((B + kGreedyWarps - 1) / kGreedyWarps));
         return from_cuda(launch_ex(true, verify_greedy_kernel, grid_g, dim3(kGreedyWarps * 32), 0, stream, 1, fp));
     }
+    const bool vec = aligned_to(draft, 16) && aligned_to(target, 16) && ((size_t)V * sizeof(In)) % 16 == 0;
+    const int sub = 32 * (vec ? Elem<In>::kVec : 1);
     int csize = 1, span = V;
-    finalize_shape(B, V, &csize, &span);
+    finalize_shape(B, V, sub, &csize, &span);
     fp.csize = csize;
     fp.span = span;
-    const bool vec = aligned_to(draft, 16) && aligned_to(target, 16) && ((size_t)V * sizeof(In)) % 16 == 0;
     const dim3 grid2(unsigned(B) * unsigned(csize));
-    const int sub = 32 * (vec ? Elem<In>::kVec : 1);
     const size_t smem2 = size_t((span + sub - 1) / sub) * sizeof(float);
     if (smem2 > size_t(kFinMaxSub) * sizeof(float)) return OSD_ERR_UNSUPPORTED;
     if (vec)
@@ -628,8 +634,44 @@ namespace {
 constexpr size_t kNoAllocScratchBytes = size_t(4) << 20;  // 4 MiB
 constexpr int kNoAllocMaxDevices = 64;
 __device__ __align__(256) unsigned char g_verify_scratch[kNoAllocScratchBytes];
+
+// The device address of the array, per device, with the ID of the context it
+// was looked up in: a new context (cudaDeviceReset, or a context the caller
+// made current) loads the module again, possibly elsewhere, so the address is
+// looked up again whenever the current context's ID differs.
+struct ScratchSlot {
+    unsigned long long ctx_id;
+    void* addr;
+};
 std::mutex g_scratch_mu;
-void* g_scratch_addr[kNoAllocMaxDevices] = {};
+ScratchSlot g_scratch[kNoAllocMaxDevices] = {};
+
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+// ID of the context current on the calling thread; false when there is none yet
+// (the runtime makes the primary context current on its first device call) or
+// the driver does not provide the query.
+bool current_context_id(unsigned long long* id) {
+    static CtxGetCurrentFn get_current = nullptr;
+    static CtxGetIdFn get_id = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_current = reinterpret_cast<CtxGetCurrentFn>(f);
+        f = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            get_id = reinterpret_cast<CtxGetIdFn>(f);
+    });
+    if (!get_current || !get_id) return false;
+    CUcontext ctx = nullptr;
+    if (get_current(&ctx) != CUDA_SUCCESS || !ctx) return false;
+    return get_id(ctx, id) == CUDA_SUCCESS;
+}
 }  // namespace
 
 extern "C" osd_status osd_verify_noalloc(const void* draft_logits, const void* target_logits,
@@ -647,15 +689,24 @@ extern "C" osd_status osd_verify_noalloc(const void* draft_logits, const void* t
     if (dev < 0 || dev >= kNoAllocMaxDevices) return OSD_ERR_UNSUPPORTED;
     void* scratch = nullptr;
     {
-        // One-time set-up per device, with that device current: the host-side name
-        // of the array is not a device address, so ask the runtime for it.
+        // Set-up once per device and context, with that device current: the
+        // host-side name of the array is not a device address, so ask the runtime.
         std::lock_guard<std::mutex> lock(g_scratch_mu);
-        if (!g_scratch_addr[dev]) {
+        unsigned long long id = 0;
+        const bool have_id = current_context_id(&id);
+        ScratchSlot& slot = g_scratch[dev];
+        if (!have_id || !slot.addr || slot.ctx_id != id) {
             void* addr = nullptr;
             if (cudaGetSymbolAddress(&addr, g_verify_scratch) != cudaSuccess || !addr) return OSD_ERR_CUDA;
-            g_scratch_addr[dev] = addr;
+            // the lookup made a context current if none was: key the address on it;
+            // without a context ID the address is not cached and is looked up every call
+            const bool keyed = have_id || current_context_id(&id);
+            slot.addr = keyed ? addr : nullptr;
+            slot.ctx_id = keyed ? id : 0ull;
+            scratch = addr;
+        } else {
+            scratch = slot.addr;
         }
-        scratch = g_scratch_addr[dev];
     }
     // The statistics pass writes every workspace entry before the finalize pass
     // reads it, so nothing in the shared array needs clearing between calls.

@@ -106,3 +106,22 @@ def test_verify_bytes(B, k, V, s_in):
     assert bench._bytes_verify(B, k, V, s_in, True) == B * (k + 1) * V * s_in
     if (B, k, V, s_in) == (256, 8, 128256, 2):
         assert bench._bytes_verify(B, k, V, s_in, False) == 1116340224
+
+
+def test_gpus_flag_starts_that_many_ranks():
+    """`bench.py --gpus 2` outside torchrun starts two ranks itself; on the
+    CPU-only launcher check (gloo, no GPU work) the line reports both ranks and
+    the slower rank's time (rank r sleeps (r + 1) ms a step)."""
+    import subprocess
+    env = {k: v for k, v in os.environ.items() if k not in ("WORLD_SIZE", "RANK", "LOCAL_RANK")}
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--gpus", "2", "--launcher-check",
+                        "--steps", "4", "--warmup", "0"], capture_output=True, text=True, timeout=300, env=env)
+    assert r.returncode == 0, r.stderr[-2000:]
+    line = json.loads([ln for ln in r.stdout.splitlines() if ln.startswith("{")][-1])
+    assert line["check"] == "launcher" and line["n_gpus"] == 2
+    assert line["ms_per_step"] >= 2.0
+    assert line["value"] == pytest.approx(2 / (line["ms_per_step"] / 1e3), rel=1e-3)
+
+
+def test_cpu_model_names_something():
+    assert isinstance(bench.cpu_model(), str) and bench.cpu_model()

@@ -232,26 +232,25 @@ def test_workload_small_configs_full(osd, cfg):
         np.testing.assert_array_equal(res0.accepted.cpu().numpy(), ref0["accepted"])
 
 
-def test_workload_large_vocab_sampled(osd):
-    """B=256, k=8, V=128256 bf16, T=0.7 at full size on the GPU, exactly as the
-    benchmark launches it; 24 sampled sequences are checked against the oracle."""
-    spec = W.VERIFY[5]
-    inp = W.verify_inputs(spec, seed=W.seed_for(5), device="cuda")
-    res = osd.osd_verify(inp["draft"], inp["target"], inp["tokens"], inp["uniforms"], spec.temperature)
+def test_unaligned_largest_vocabulary_past_128_sequences(osd):
+    """The element-wise finalize (rows off the 16-byte path) at B > 128 and a
+    vocabulary near the limit: its spans need more than four CTAs a sequence."""
+    V = (1 << 21) - 1  # odd: bf16 rows are not 16-byte multiples
+    spec = W.VerifySpec(130, 1, V, torch.bfloat16, 2.0, 1.0, 1.0, 1.0)
+    inp = W.verify_inputs(spec, seed=2121, device="cuda")
+    res = osd.osd_verify(inp["draft"], inp["target"], inp["tokens"], inp["uniforms"], 1.0)
     torch.cuda.synchronize()
-    idx = torch.tensor(sorted(np.random.default_rng(0).choice(spec.B, 24, replace=False)))
+    idx = torch.arange(0, 130, 26)
     ref = oracle.verify(inp["draft"][idx].cpu(), inp["target"][idx].cpu(), inp["tokens"][idx].cpu(),
-                        inp["uniforms"][idx].cpu(), _t32(spec.temperature))
+                        inp["uniforms"][idx].cpu(), 1.0)
 
     class Sub:
         pass
     sub = Sub()
     for f in ("accepted", "out_tokens", "mismatch_mask", "diag_margin", "diag_cdf_gap"):
         setattr(sub, f, getattr(res, f)[idx.to(res.accepted.device)])
-    rep = check_verify(sub, ref, spec.k, spec.V)
-    check_margins(sub, ref)
-    # properties over every sequence
+    check_verify(sub, ref, spec.k, V)
     acc = res.accepted.cpu()
-    assert ((acc >= 0) & (acc <= spec.k)).all()
-    assert (res.mismatch_mask.sum(1).cpu() == (acc < spec.k).to(torch.uint8)).all()
-    print(f"config 5 sampled: {rep}, mean accepted {acc.float().mean():.3f}")
+    assert ((acc >= 0) & (acc <= 1)).all()
+    out = res.out_tokens.cpu()
+    assert ((out[torch.arange(130), acc.long()] >= 0) & (out[torch.arange(130), acc.long()] < V)).all()
