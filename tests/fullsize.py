@@ -5,8 +5,8 @@ inputs and gradients together), more than the oracle should see at once.  The
 rows are therefore brought to the host in chunks; each chunk is split into
 small row blocks that a thread pool hands to the oracle (its C calls release
 the GIL, so the blocks run on every host core), and every block is compared
-with the GPU's rows under the rules of ``tests/parity.py``.  Nothing is
-sampled: the report counts every row.
+with the GPU's rows under the rules of ``tests/parity.py`` (TVD near-tie rows
+included).  Nothing is sampled: the report counts every row.
 """
 from __future__ import annotations
 
@@ -17,14 +17,14 @@ import numpy as np
 import torch
 
 import oracle
-from tests.parity import GRAD_ATOL, GRAD_RTOL, LOSS_ATOL, LOSS_RTOL, TIE, near_tie_rows
+from tests.parity import LOSS_ATOL, LOSS_RTOL, TIE, grad_rows, near_tie_rows, tvd_ties
 
 
 def _threads() -> int:
     return max(1, min(32, os.cpu_count() or 1))
 
 
-def _block_distill(z, t, lg, gg, kind, beta, tau, tvd_skip):
+def _block_distill(z, t, lg, gg, kind, beta, tau):
     """Oracle and comparison for one block of active rows (float32 numpy in)."""
     lr, gr = oracle.distill(z, t, None, kind, beta, temperature=tau)
     lg = lg.astype(np.float64)
@@ -32,21 +32,15 @@ def _block_distill(z, t, lg, gg, kind, beta, tau, tvd_skip):
     lerr = np.abs(lg - lr)
     loss_bad = ~same_inf & ~(lerr <= LOSS_RTOL * np.abs(lr) + LOSS_ATOL)
     fin = np.isfinite(lr)
-    g = gg.astype(np.float64)
-    n_skip = 0
-    if tvd_skip:
-        amb = np.abs(oracle.log_softmax(z, tau) - oracle.log_softmax(t, tau)) < 1e-5
-        n_skip = int(amb[fin].sum())
-        g = np.where(amb, 0.0, g)
-        gr = np.where(amb, 0.0, gr)
-    scale = np.max(np.abs(gr), axis=1)
-    gerr = np.max(np.abs(g - gr), axis=1)
-    grad_bad = fin & ~(gerr <= GRAD_RTOL * scale + GRAD_ATOL)   # NaN errors count as bad
-    rel = np.where(fin, gerr / np.maximum(scale, GRAD_ATOL / GRAD_RTOL), 0.0)
+    ties = tvd_ties(z[fin], t[fin], tau) if kind == "tvd" else None
+    res = grad_rows(gg[fin].astype(np.float64), gr[fin], ties)
     lrel = np.where(~same_inf, lerr / np.maximum(np.abs(lr), 1e-30), 0.0)
-    return {"rows": z.shape[0], "loss_bad": int(loss_bad.sum()), "grad_bad": int(grad_bad.sum()),
-            "inf_rows": int((~fin).sum()), "grad_rel_max": float(np.nanmax(rel)) if rel.size else 0.0,
-            "loss_rel_max": float(np.nanmax(lrel)) if lrel.size else 0.0, "tvd_skipped": n_skip}
+    return {"rows": z.shape[0], "loss_bad": int(loss_bad.sum()), "grad_bad": int((~res["ok"]).sum()),
+            "inf_rows": int((~fin).sum()),
+            "grad_rel_max": float(np.nanmax(res["rel"])) if res["rel"].size else 0.0,
+            "loss_rel_max": float(np.nanmax(lrel)) if lrel.size else 0.0,
+            "tvd_skipped": int(ties.amb.sum()) if ties is not None else 0,
+            "near_tie": int(res["near_tie"].sum()), "near_tie_differ": int(res["near_tie_differ"].sum())}
 
 
 def distill_parity(z: torch.Tensor, t: torch.Tensor, active, loss_g: torch.Tensor, grad_g: torch.Tensor,
@@ -60,7 +54,7 @@ def distill_parity(z: torch.Tensor, t: torch.Tensor, active, loss_g: torch.Tenso
     N, V = z.shape
     act_all = np.ones(N, bool) if active is None else np.asarray(active, bool)
     tot = {"rows": 0, "loss_bad": 0, "grad_bad": 0, "inf_rows": 0, "grad_rel_max": 0.0, "loss_rel_max": 0.0,
-           "tvd_skipped": 0, "inactive_rows": 0}
+           "tvd_skipped": 0, "near_tie": 0, "near_tie_differ": 0, "inactive_rows": 0}
     with cf.ThreadPoolExecutor(max_workers=_threads()) as ex:
         for c0 in range(0, N, chunk):
             c1 = min(N, c0 + chunk)
@@ -81,11 +75,11 @@ def distill_parity(z: torch.Tensor, t: torch.Tensor, active, loss_g: torch.Tenso
             gc = grad_g[torch.as_tensor(rows + c0, device=grad_g.device)].cpu().numpy()
             lc = lg[rows]
             futs = [ex.submit(_block_distill, zc[b:b + block], tc[b:b + block], lc[b:b + block],
-                              gc[b:b + block], kind, beta, tau, kind == "tvd")
+                              gc[b:b + block], kind, beta, tau)
                     for b in range(0, rows.size, block)]
             for f in futs:
                 r = f.result()
-                for key in ("rows", "loss_bad", "grad_bad", "inf_rows", "tvd_skipped"):
+                for key in ("rows", "loss_bad", "grad_bad", "inf_rows", "tvd_skipped", "near_tie", "near_tie_differ"):
                     tot[key] += r[key]
                 tot["grad_rel_max"] = max(tot["grad_rel_max"], r["grad_rel_max"])
                 tot["loss_rel_max"] = max(tot["loss_rel_max"], r["loss_rel_max"])

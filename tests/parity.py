@@ -8,8 +8,13 @@ to |l - l_ref| <= 1e-4 |l_ref| + 1e-6 and gradients, row by row, to
 max|g - g_ref| <= 1e-4 max|g_ref| + 1e-7 (an elementwise relative error is
 meaningless for entries of 1e-9; the 1e-7 floor is fp32 resolution of
 probabilities, reached when p and q nearly coincide and every entry is ~0).
+TVD's gradient is compared as ``grad_rows`` describes: entries where fp32
+cannot order q and p are left out, and rows where their sign choice could
+matter must match the subgradient of the GPU's own choice there.
 """
 from __future__ import annotations
+
+from typing import NamedTuple, Optional
 
 import numpy as np
 
@@ -69,6 +74,74 @@ def check_margins(gpu, ref: dict, tol: float = 2e-6) -> float:
     return worst
 
 
+TVD_TIE = 1e-5  # |ln q - ln p| below this: fp32 cannot tell which of q and p is larger
+
+
+class TvdTies(NamedTuple):
+    """What the TVD comparison needs from the oracle besides its gradient:
+    amb [rows, V] marks entries whose sign(q - p) fp32 cannot decide; q and
+    d = ln q - ln p are the oracle's (float64); tau the temperature."""
+    amb: np.ndarray
+    q: np.ndarray
+    d: np.ndarray
+    tau: float
+
+
+def tvd_ties(z, t, tau: float = 1.0) -> TvdTies:
+    import oracle
+    V = z.shape[-1]
+    lq = oracle.log_softmax(np.asarray(z, np.float64).reshape(-1, V), tau)
+    lp = oracle.log_softmax(np.asarray(t, np.float64).reshape(-1, V), tau)
+    d = lq - lp
+    return TvdTies(np.abs(d) < TVD_TIE, np.exp(lq), d, float(tau))
+
+
+def tvd_subgradient(q: np.ndarray, s: np.ndarray, tau: float) -> np.ndarray:
+    """d/dz of 1/2 sum|p - q| for the sign choice s_j in {-1, 0, 1} of
+    sign(q_j - p_j): q_k (s_k / 2 - sum_j q_j s_j / 2) / tau (reading 9)."""
+    return q * (0.5 * s - 0.5 * np.sum(q * s, axis=1, keepdims=True)) / tau
+
+
+def grad_rows(gg: np.ndarray, gr: np.ndarray, tvd: Optional[TvdTies] = None) -> dict:
+    """Row-by-row gradient comparison (float64 [rows, V]).
+
+    TVD is not differentiable where q_j = p_j: any value in [-1/2, 1/2] of the
+    sign there gives a valid subgradient (reading 9).  Entries whose order fp32
+    cannot decide (|ln q - ln p| < 1e-5) are left out of the comparison, and
+    their sign also enters every other entry through sum_j q_j s_j / 2: a flip
+    moves entry k by up to q_k (sum of q over those entries) / tau.  Rows where
+    that can exceed half the tolerance are near-tie rows: there the GPU's
+    gradient must equal the exact subgradient for the signs it chose at those
+    entries (read off its own gradient), with the oracle's q and its signs
+    everywhere else.  Returns ok, rel [rows] and the near_tie, near_tie_differ
+    masks."""
+    rows = gg.shape[0]
+    near = np.zeros(rows, bool)
+    differ = np.zeros(rows, bool)
+    g, r = gg, gr
+    if tvd is not None:
+        g = np.where(tvd.amb, 0.0, gg)
+        r = np.where(tvd.amb, 0.0, gr)
+    scale = np.max(np.abs(r), axis=1)
+    lim = GRAD_RTOL * scale + GRAD_ATOL
+    err = np.max(np.abs(g - r), axis=1)
+    ok = err <= lim
+    rel = err / np.maximum(scale, GRAD_ATOL / GRAD_RTOL)
+    if tvd is not None:
+        qmax = np.max(np.where(tvd.amb, 0.0, tvd.q), axis=1)
+        shift = qmax * np.sum(np.where(tvd.amb, tvd.q, 0.0), axis=1) / tvd.tau
+        near = shift > 0.5 * lim
+        for i in np.nonzero(near & ~ok)[0]:
+            s = np.where(tvd.amb[i], np.sign(gg[i]), np.sign(tvd.d[i]))[None, :]
+            alt = tvd_subgradient(tvd.q[i][None, :], s, tvd.tau)[0]
+            e2 = np.max(np.abs(gg[i] - alt))
+            if e2 <= lim[i]:
+                ok[i] = True
+                differ[i] = True
+                rel[i] = e2 / max(scale[i], GRAD_ATOL / GRAD_RTOL)
+    return {"ok": ok, "rel": rel, "near_tie": near, "near_tie_differ": differ}
+
+
 def check_distill(loss_g, grad_g, loss_r, grad_r, active: np.ndarray, skip_elems=None) -> dict:
     """Loss / gradient parity on active rows; inactive rows keep their sentinel."""
     lg = np.asarray(loss_g, np.float64)
@@ -88,17 +161,15 @@ def check_distill(loss_g, grad_g, loss_r, grad_r, active: np.ndarray, skip_elems
     # defined gradient on either side: only the loss is compared there
     fin = np.isfinite(lra)
     ga, gra = gg[act][fin], gr[act][fin]
-    if skip_elems is not None:
-        sk = np.asarray(skip_elems, bool)[act][fin]
-        ga = np.where(sk, 0.0, ga)
-        gra = np.where(sk, 0.0, gra)
-    scale = np.max(np.abs(gra), axis=1)
-    gerr = np.max(np.abs(ga - gra), axis=1)
-    assert np.all(np.isfinite(gerr)), "non-finite gradients"
-    ok = gerr <= GRAD_RTOL * scale + GRAD_ATOL
-    rel = gerr / np.maximum(scale, GRAD_ATOL / GRAD_RTOL)
-    worst = float(rel.max()) if rel.size else 0.0
-    assert np.all(ok), f"gradient mismatch: worst row-relative error {worst:.3g}"
+    tvd = None
+    if skip_elems is not None:  # a TvdTies for the same rows as the logits
+        sel = np.nonzero(act)[0][fin]
+        tvd = TvdTies(skip_elems.amb[sel], skip_elems.q[sel], skip_elems.d[sel], skip_elems.tau)
+    assert np.all(np.isfinite(ga)), "non-finite gradients"
+    res = grad_rows(ga, gra, tvd)
+    worst = float(res["rel"].max()) if res["rel"].size else 0.0
+    assert np.all(res["ok"]), f"gradient mismatch: worst row-relative error {worst:.3g}"
     lrel = err[~same_inf] / np.maximum(np.abs(lra[~same_inf]), 1e-30)
     return {"rows": int(act.sum()), "infinite_loss_rows": int((~fin).sum()), "grad_rel_max": worst,
-            "loss_rel_max": float(lrel.max()) if lrel.size else 0.0}
+            "loss_rel_max": float(lrel.max()) if lrel.size else 0.0,
+            "near_tie": int(res["near_tie"].sum()), "near_tie_differ": int(res["near_tie_differ"].sum())}
