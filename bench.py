@@ -664,7 +664,8 @@ def _oracle_step_time(setup, n_rows, threads):
         zd = d["draft"][:n_rows].cpu()
         td = d["target"][:n_rows].cpu()
         for kind in ("rkl", "tvd"):
-            for (a, b) in chunks(n_rows, threads):
+            # blocks of at most 256 rows: the oracle holds each block in double precision
+            for (a, b) in chunks(n_rows, max(threads, (n_rows + 255) // 256)):
                 jobs.append(lambda a=a, b=b, kind=kind: (oracle.distill(zd[a:b], td[a:b], None, kind, 0.5),
                                                          b - a)[1])
     t0 = time.perf_counter()
@@ -722,15 +723,15 @@ def run_reference(args):
              else _setup_large_vocab(dev))
     threads = os.cpu_count() or 1
     for _ in range(args.warmup):
-        _oracle_step_time(setup, max(16, args.cpu_rows // 8), threads)
+        _oracle_step_time(setup, max(16, args.ref_rows // 8), threads)
     times, pos = [], 0
     for _ in range(args.steps):
-        s, pos = _oracle_step_time(setup, args.cpu_rows, threads)
+        s, pos = _oracle_step_time(setup, args.ref_rows, threads)
         times.append(s)
     ms = 1e3 * sum(times) / len(times)
     value = pos / (ms / 1e3)
     sample = (f"per step: whole verify batch (both passes, with its rejected rows distilled) + "
-              f"{args.cpu_rows} distill rows per loss kind "
+              f"{args.ref_rows} distill rows per loss kind "
               f"of the same workload, {threads} host threads")
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 2), "unit": "positions/s",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3),
@@ -789,8 +790,12 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", choices=["serving-32k", "large-vocab"], default="serving-32k")
-    ap.add_argument("--cpu-rows", type=int, default=16384,
-                    help="distill rows per loss kind in the oracle sample (about 20 s of CPU time on 16 cores)")
+    ap.add_argument("--cpu-rows", type=int, default=65536,
+                    help="distill rows per loss kind in the cpu_baseline oracle sample (65536: the whole step, "
+                         "about 7 s on 16 Neoverse-V2 cores)")
+    ap.add_argument("--ref-rows", type=int, default=16384,
+                    help="distill rows per loss kind in each step of --impl reference (about 2 s a step on "
+                         "16 Neoverse-V2 cores)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     ap.add_argument("--no-extras", action="store_true",

@@ -130,52 +130,49 @@ __global__ void __launch_bounds__(kGreedyWarps * 32) verify_greedy_kernel(FinPar
     }
 }
 
-template <typename In, bool kVecPath>
-__global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams p) {
+// Shared memory of one sequence's decision: the merged statistics of its 2k+1
+// rows (local row r <= k is target row r, r > k is draft row r-k-1), the draft
+// tokens, the two logits each accept test needs, the uniforms, and a.
+struct SeqSmem {
+    float m[2 * OSD_VERIFY_MAX_K + 1];
+    float s[2 * OSD_VERIFY_MAX_K + 1];
+    float zy[OSD_VERIFY_MAX_K], ty[OSD_VERIFY_MAX_K];
+    int y[OSD_VERIFY_MAX_K];
+    float u[OSD_VERIFY_MAX_K + 1];
+    int a;
+};
+
+// Prologue of sequence b's decision, run by every thread of a CTA of kThreads:
+// every independent global load goes out in one round (the last warp fetches
+// the draft tokens and gathers the two logits each accept test needs, the warp
+// before it the uniforms); then, once the row statistics are complete, the
+// warps merge each row's slice statistics, loading up to four rows per lane
+// before reducing.  Returns non-zero, for every thread, when a draft token
+// lies outside [0, V).
+template <typename In, int kThreads>
+__device__ __forceinline__ int seq_prologue(const FinParams& p, int b, SeqSmem& sh) {
     using E = Elem<In>;
-    constexpr int kW = kVecPath ? E::kVec : 1;  // entries per lane per sub-tile
-    constexpr int kSub = 32 * kW;
-    constexpr int kWarps = kFinThreads / 32;
-
-    __shared__ float s_m[2 * OSD_VERIFY_MAX_K + 1];
-    __shared__ float s_s[2 * OSD_VERIFY_MAX_K + 1];
-    __shared__ float s_zy[OSD_VERIFY_MAX_K], s_ty[OSD_VERIFY_MAX_K];
-    __shared__ int s_y[OSD_VERIFY_MAX_K];
-    __shared__ float s_u[OSD_VERIFY_MAX_K + 1];
-    __shared__ int s_a, s_owner, s_mode, s_tile;
-    extern __shared__ float s_sub[];  // one residual sum per sub-tile of this CTA's span
-    // residual masses in exact 64-bit fixed point (fix_of): a dependent fp64 add is slow here
-    __shared__ unsigned long long s_span_total;  // read by the other CTAs of the cluster
-    __shared__ unsigned long long s_tau, s_W, s_base;
-
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int rank = (p.csize > 1) ? static_cast<int>(cluster_rank()) : 0;
-    const int b = blockIdx.x / p.csize;
+    constexpr int kWarps = kThreads / 32;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int k = p.k, V = p.V;
     const int32_t* y = p.tokens + size_t(b) * k;
     const In* draft = static_cast<const In*>(p.draft);
     const In* target = static_cast<const In*>(p.target);
-
-    // Prologue: every independent global load goes out in one round.  The last
-    // warp fetches the draft tokens and gathers the two logits each accept test
-    // needs; the warp before it fetches the uniforms; all warps merge the slice
-    // statistics of the 2k+1 rows (local row r <= k is target row r, r > k is
-    // draft row r-k-1), loading up to four rows per lane before reducing.
     int bad = 0;
     if (warp == kWarps - 1) {
         for (int i = lane; i < k; i += 32) {
             const int t = y[i];
-            s_y[i] = t;
+            sh.y[i] = t;
             if (t < 0 || t >= V) {
                 bad = 1;
             } else {
-                s_zy[i] = E::load(draft + (size_t(b) * k + i) * V + t);
-                s_ty[i] = E::load(target + (size_t(b) * (k + 1) + i) * V + t);
+                sh.zy[i] = E::load(draft + (size_t(b) * k + i) * V + t);
+                sh.ty[i] = E::load(target + (size_t(b) * (k + 1) + i) * V + t);
             }
         }
     }
     if (warp == kWarps - 2)
-        for (int i = lane; i <= k; i += 32) s_u[i] = p.uniforms[size_t(b) * (k + 1) + i];
+        for (int i = lane; i <= k; i += 32) sh.u[i] = p.uniforms[size_t(b) * (k + 1) + i];
     grid_dependency_wait();  // the row statistics are complete from here on
     const int nrows = 2 * k + 1;
     const float ch0 = p.c_hi, cl0 = p.c_lo;
@@ -201,26 +198,31 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
             if (have[q]) acc = MaxSum{part[q][0].m, part[q][0].s};
             for (int sl = lane + 32; sl < p.n_slices; sl += 32) acc = merge(acc, MaxSum{st[sl].m, st[sl].s});
             acc = warp_reduce(acc, merge);
-            if (lane == 0) { s_m[r] = acc.m; s_s[r] = acc.s; }
+            if (lane == 0) { sh.m[r] = acc.m; sh.s[r] = acc.s; }
         }
     }
-    bad = __syncthreads_or(bad);
+    return __syncthreads_or(bad);
+}
 
+// Outputs of a sequence with a bad draft token (one CTA of kThreads writes them).
+template <int kThreads>
+__device__ __forceinline__ void seq_write_bad(const FinParams& p, int b) {
+    const int tid = threadIdx.x, k = p.k;
     int32_t* out = p.out_tokens + size_t(b) * (k + 1);
-    if (bad) {  // uniform over the cluster, before any distributed shared memory access
-        if (rank == 0) {
-            if (tid == 0) { p.accepted[b] = -1; if (p.diag_gap) p.diag_gap[b] = __int_as_float(0x7fc00000); }
-            for (int i = tid; i <= k; i += kFinThreads) out[i] = -1;
-            for (int i = tid; i < k; i += kFinThreads) {
-                p.mask[size_t(b) * k + i] = 0;
-                if (p.diag_margin) p.diag_margin[size_t(b) * k + i] = __int_as_float(0x7fc00000);
-            }
-        }
-        return;
+    if (tid == 0) { p.accepted[b] = -1; if (p.diag_gap) p.diag_gap[b] = __int_as_float(0x7fc00000); }
+    for (int i = tid; i <= k; i += kThreads) out[i] = -1;
+    for (int i = tid; i < k; i += kThreads) {
+        p.mask[size_t(b) * k + i] = 0;
+        if (p.diag_margin) p.diag_margin[size_t(b) * k + i] = __int_as_float(0x7fc00000);
     }
+}
 
-    // ---- accept tests: warp 0 runs them all at once, one position per lane, and
-    // the first failing position is a (the tests after it are not decided)
+// The k accept tests: warp 0 runs them all at once, one position per lane, and
+// the first failing position is a (the tests after it are not decided).  Sets
+// sh.a, writes the margins of the decided positions when `margins` is set, and
+// ends on a block barrier.
+__device__ __forceinline__ void seq_accept(const FinParams& p, int b, SeqSmem& sh, bool margins) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, k = p.k;
     if (warp == 0) {
         int a = k;
         float r_all[(OSD_VERIFY_MAX_K + 31) / 32];
@@ -230,44 +232,81 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
             bool fail = false;
             r_all[c] = 0.f;
             if (i < k) {
-                const float mt = s_m[i], st = s_s[i];
-                const float mz = s_m[k + 1 + i], sz = s_s[k + 1 + i];
-                const float D = (s_ty[i] - mt) - (s_zy[i] - mz);
+                const float mt = sh.m[i], st = sh.s[i];
+                const float mz = sh.m[k + 1 + i], sz = sh.s[k + 1 + i];
+                const float D = (sh.ty[i] - mt) - (sh.zy[i] - mz);
                 r_all[c] = expf(__fdiv_rn(D, p.T)) * __fdiv_rn(sz, st);
-                fail = !(s_u[i] < r_all[c]);
+                fail = !(sh.u[i] < r_all[c]);
             }
             const unsigned f = __ballot_sync(0xffffffffu, fail);
             if (f && a == k) a = c * 32 + __ffs(f) - 1;
         }
-        if (rank == 0 && p.diag_margin) {
+        if (margins) {
 #pragma unroll
             for (int c = 0; c < (OSD_VERIFY_MAX_K + 31) / 32; ++c) {
                 const int i = c * 32 + lane;
-                if (i < k && i <= a) p.diag_margin[size_t(b) * k + i] = fabsf(s_u[i] - r_all[c]);
+                if (i < k && i <= a) p.diag_margin[size_t(b) * k + i] = fabsf(sh.u[i] - r_all[c]);
             }
         }
-        if (lane == 0) s_a = a;
+        if (lane == 0) sh.a = a;
     }
     __syncthreads();
-    const int a = s_a;
-    if (rank == 0) {
-        if (tid == 0) p.accepted[b] = a;
-        for (int i = tid; i <= k; i += kFinThreads)
-            if (i < a) out[i] = s_y[i];
-            else if (i > a) out[i] = -1;
-        for (int i = tid; i < k; i += kFinThreads) {
-            p.mask[size_t(b) * k + i] = (i == a) ? 1 : 0;
-            if (p.diag_margin && i > a) p.diag_margin[size_t(b) * k + i] = __int_as_float(0x7fc00000);
-        }
+}
+
+// accepted, the accepted tokens and the -1 padding after a, the mask, and the
+// margins past the decision (one CTA of kThreads); the token at a is the draw's.
+template <int kThreads>
+__device__ __forceinline__ void seq_write_outputs(const FinParams& p, int b, const SeqSmem& sh, int a) {
+    const int tid = threadIdx.x, k = p.k;
+    int32_t* out = p.out_tokens + size_t(b) * (k + 1);
+    if (tid == 0) p.accepted[b] = a;
+    for (int i = tid; i <= k; i += kThreads)
+        if (i < a) out[i] = sh.y[i];
+        else if (i > a) out[i] = -1;
+    for (int i = tid; i < k; i += kThreads) {
+        p.mask[size_t(b) * k + i] = (i == a) ? 1 : 0;
+        if (p.diag_margin && i > a) p.diag_margin[size_t(b) * k + i] = __int_as_float(0x7fc00000);
     }
+}
+
+template <typename In, bool kVecPath>
+__global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams p) {
+    using E = Elem<In>;
+    constexpr int kW = kVecPath ? E::kVec : 1;  // entries per lane per sub-tile
+    constexpr int kSub = 32 * kW;
+    constexpr int kWarps = kFinThreads / 32;
+
+    __shared__ SeqSmem sh;
+    __shared__ int s_owner, s_mode, s_tile;
+    extern __shared__ float s_sub[];  // one residual sum per sub-tile of this CTA's span
+    // residual masses in exact 64-bit fixed point (fix_of): a dependent fp64 add is slow here
+    __shared__ unsigned long long s_span_total;  // read by the other CTAs of the cluster
+    __shared__ unsigned long long s_tau, s_W, s_base;
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int rank = (p.csize > 1) ? static_cast<int>(cluster_rank()) : 0;
+    const int b = blockIdx.x / p.csize;
+    const int k = p.k, V = p.V;
+    const In* draft = static_cast<const In*>(p.draft);
+    const In* target = static_cast<const In*>(p.target);
+
+    const int bad = seq_prologue<In, kFinThreads>(p, b, sh);
+    int32_t* out = p.out_tokens + size_t(b) * (k + 1);
+    if (bad) {  // uniform over the cluster, before any distributed shared memory access
+        if (rank == 0) seq_write_bad<kFinThreads>(p, b);
+        return;
+    }
+    seq_accept(p, b, sh, rank == 0 && p.diag_margin);
+    const int a = sh.a;
+    if (rank == 0) seq_write_outputs<kFinThreads>(p, b, sh, a);
 
     // ---- extra token: inverse CDF of w = max(0, p_a - q_a) (a < k) or p_k (a == k)
     const bool bonus = (a == k);
     const In* trow = target + (size_t(b) * (k + 1) + a) * V;
     const In* zrow = draft + (size_t(b) * k + (bonus ? 0 : a)) * V;
-    const float mt = s_m[a], inv_st = 1.0f / s_s[a];
-    const float mz = bonus ? 0.f : s_m[k + 1 + a];
-    const float inv_sz = bonus ? 0.f : 1.0f / s_s[k + 1 + a];
+    const float mt = sh.m[a], inv_st = 1.0f / sh.s[a];
+    const float mz = bonus ? 0.f : sh.m[k + 1 + a];
+    const float inv_sz = bonus ? 0.f : 1.0f / sh.s[k + 1 + a];
     const float ch = p.c_hi, cl = p.c_lo;
     auto weight = [&](float t, float z) -> float {
         const float pj = ex2(mul_c(t - mt, ch, cl)) * inv_st;
@@ -361,7 +400,7 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
     // warp 0 of every CTA derives W, tau = floor(u W) and the owning CTA identically:
     // lane r holds CTA r's total, a warp scan gives the prefix in rank order
     if (warp == 0) {
-        const float u = s_u[k];
+        const float u = sh.u[k];
         unsigned long long tot = 0ull;
         if (lane < p.csize) tot = (lane == rank) ? s_span_total : ld_dsmem_u64(map_rank(&s_span_total, lane));
         const unsigned long long incl = warp_incl_scan_u64(tot);
@@ -502,6 +541,8 @@ static int verify_slices(int B, int k, int V) {
     return (V + len - 1) / len;
 }
 
+static size_t round256(size_t x) { return (x + 255) / 256 * 256; }
+
 // CTAs per sequence: up to 8 for few sequences (short spans, low latency); 4 past
 // 128 sequences, where 8 would leave more clusters than fit on the GPU at once and
 // the second wave would wait out the first one's latency phases.  A span must fit
@@ -583,8 +624,7 @@ extern "C" osd_status osd_verify_workspace_size(int B, int k, int V, size_t* byt
     if (!bytes || B < 0 || k < 1 || V < 1) return OSD_ERR_INVALID_ARG;
     if (k > OSD_VERIFY_MAX_K || V > OSD_VERIFY_MAX_V) return OSD_ERR_UNSUPPORTED;
     const size_t rows = size_t(B) * size_t(2 * k + 1);
-    size_t need = rows * size_t(osd::verify_slices(B, k, V)) * sizeof(RowStat);
-    need = (need + 255) / 256 * 256;
+    const size_t need = osd::round256(rows * size_t(osd::verify_slices(B, k, V)) * sizeof(RowStat));
     *bytes = need < 256 ? 256 : need;
     return OSD_OK;
 }
@@ -613,13 +653,13 @@ extern "C" osd_status osd_verify(const void* draft_logits, const void* target_lo
         return OSD_ERR_INVALID_ARG;
     if (workspace_bytes < need) return OSD_ERR_INVALID_ARG;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    RowStat* stats = static_cast<RowStat*>(workspace);
     if (dtype == OSD_BF16)
         return osd::launch_verify<__nv_bfloat16>(draft_logits, target_logits, B, k, V, draft_tokens, uniforms,
                                                  temperature, accepted, out_tokens, mismatch_mask, diag_margin,
-                                                 diag_cdf_gap, stats, s);
+                                                 diag_cdf_gap, static_cast<RowStat*>(workspace), s);
     return osd::launch_verify<float>(draft_logits, target_logits, B, k, V, draft_tokens, uniforms, temperature,
-                                     accepted, out_tokens, mismatch_mask, diag_margin, diag_cdf_gap, stats, s);
+                                     accepted, out_tokens, mismatch_mask, diag_margin, diag_cdf_gap,
+                                     static_cast<RowStat*>(workspace), s);
 }
 
 // ------------------------------------------------------------------ no-allocation variant

@@ -56,6 +56,12 @@ CASES = [  # (B, k, V, dtype, T)
     (160, 2, 20000, torch.bfloat16, 1.0),    # past 128 sequences: 4 finalize CTAs per sequence
     (130, 3, 40961, torch.float32, 0.7),     # the same, element-wise path
     (2, 3, 1 << 21, torch.bfloat16, 1.0),    # the largest vocabulary
+    # past 128 sequences the finalize takes clusters of at most 4 CTAs
+    (129, 1, 4096, torch.float32, 1.0),
+    (200, 3, 8264, torch.bfloat16, 1.0),
+    (300, 2, 16384, torch.float32, 0.7),     # exactly one slice
+    (150, 4, 49160, torch.bfloat16, 1.3),    # a ragged last slice
+    (140, 2, 16392, torch.bfloat16, 0.7),    # a last slice of one 8-entry vector
 ]
 
 
@@ -89,13 +95,14 @@ def test_greedy_matches_oracle(osd, B, k, V, dtype):
     assert torch.equal(res2.out_tokens, res.out_tokens)
 
 
-def test_identical_logits_accept_all(osd):
-    spec = W.VerifySpec(16, 5, 5000, torch.bfloat16, 2.0, 1.0, 0.0, 1.0)
+@pytest.mark.parametrize("B,V", [(16, 5000), (160, 8192)])
+def test_identical_logits_accept_all(osd, B, V):
+    spec = W.VerifySpec(B, 5, V, torch.bfloat16, 2.0, 1.0, 0.0, 1.0)
     inp = W.verify_inputs(spec, seed=5)
     inp["target"] = torch.cat([inp["draft"], inp["target"][:, -1:]], dim=1).contiguous()
     res, ref = _run(osd, inp, 1.0)
     assert (res.accepted.cpu() == 5).all()
-    check_verify(res, ref, 5, 5000)
+    check_verify(res, ref, 5, V)
 
 
 def test_extreme_and_neg_inf_logits(osd):
@@ -187,11 +194,40 @@ def test_gpu_output_distribution_equals_target(osd, T, V, k):
         assert abs(acc / reach - alpha) < 5 * math.sqrt(alpha * (1 - alpha) / reach)
 
 
-@pytest.mark.parametrize("V,dtype", [(1000, torch.float32), (32000, torch.bfloat16), (4099, torch.bfloat16)])
-def test_extreme_uniforms(osd, V, dtype):
+def test_gpu_output_distribution_large_batch(osd):
+    """Section 3 at a large batch: 2 x 10^5 sequences at V = 4096, k = 1; the
+    first emitted token follows p_0.  The vocabulary is binned into 8 hot
+    entries and 16 ranges of the rest."""
+    rng = np.random.default_rng(4321)
+    V, k, n = 4096, 1, 200_000
+    z1 = rng.normal(0, 1.0, (k, V))
+    t1 = rng.normal(0, 1.0, (k + 1, V))
+    hot = rng.choice(V, 8, replace=False)
+    t1[0, hot] += 5.0
+    z1[0, hot[:4]] += 5.5      # the draft favours half of them, the residual the other half
+    a, out = _mc(osd, z1, t1, 1.0, n, seed=4322)
+    p0 = softmax(t1[0])
+    bins = np.full(V, -1)
+    bins[hot] = np.arange(8)
+    rest = np.setdiff1d(np.arange(V), hot)
+    bins[rest] = 8 + np.arange(rest.size) * 16 // rest.size
+    obs = np.bincount(bins[out[:, 0]], minlength=24)
+    exp = np.bincount(bins, weights=p0, minlength=24) * n
+    assert chisquare(obs, exp).pvalue > 1e-3
+    # the acceptance rate at position 0 is sum min(p, q)
+    q0 = softmax(z1[0])
+    alpha = np.minimum(p0, q0).sum()
+    acc = (a >= 1).mean()
+    assert abs(acc - alpha) < 5 * math.sqrt(alpha * (1 - alpha) / n), (acc, alpha)
+
+
+@pytest.mark.parametrize("B,V,dtype", [(64, 1000, torch.float32), (64, 32000, torch.bfloat16),
+                                       (64, 4099, torch.bfloat16), (160, 32000, torch.bfloat16),
+                                       (136, 20000, torch.float32)])
+def test_extreme_uniforms(osd, B, V, dtype):
     """The extra-token draw at u = 0 (the first positive weight) and at the largest float
     below 1 (tau next to W), and accept tests at both ends, against the oracle."""
-    spec = W.VerifySpec(64, 3, V, dtype, 2.0, 0.8, 1.2, 1.0)
+    spec = W.VerifySpec(B, 3, V, dtype, 2.0, 0.8, 1.2, 1.0)
     inp = W.verify_inputs(spec, seed=500 + V)
     u = inp["uniforms"]
     below_one = float(np.nextafter(np.float32(1.0), np.float32(0.0)))
