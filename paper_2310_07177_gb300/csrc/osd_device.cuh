@@ -353,6 +353,53 @@ __device__ __forceinline__ int ld_dsmem_s32(uint32_t addr) {
     return v;
 }
 
+// ---------------------------------------------------------------- tensor memory (tcgen05)
+// Tensor memory: 128 lanes x 512 columns of 32-bit cells per SM.  A CTA allocates
+// a power-of-two number of columns (32..512) with one warp; warp w of a CTA may
+// access lanes 32 (w % 4) .. 32 (w % 4) + 31, each thread its own lane.  An
+// address is (lane << 16) | column.
+__device__ __forceinline__ void tm_alloc(uint32_t* dst_smem, uint32_t ncols) {  // one whole warp
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;"
+                 :: "r"(smem_addr(dst_smem)), "r"(ncols) : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tm_dealloc(uint32_t taddr, uint32_t ncols) {  // one whole warp
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" :: "r"(taddr), "r"(ncols) : "memory");
+}
+// Order tensor-memory accesses around a thread barrier (alloc -> use -> dealloc).
+__device__ __forceinline__ void tm_fence_before_sync() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tm_fence_after_sync() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// Eight consecutive columns of this thread's lane (warp-collective, uniform address).
+__device__ __forceinline__ void tm_ld8(uint32_t taddr, uint4& a, uint4& b) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(a.x), "=r"(a.y), "=r"(a.z), "=r"(a.w), "=r"(b.x), "=r"(b.y), "=r"(b.z), "=r"(b.w)
+                 : "r"(taddr) : "memory");
+}
+__device__ __forceinline__ void tm_ld4(uint32_t taddr, uint4& a) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(a.x), "=r"(a.y), "=r"(a.z), "=r"(a.w) : "r"(taddr) : "memory");
+}
+__device__ __forceinline__ void tm_st8(uint32_t taddr, const uint4& a, const uint4& b) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};"
+                 :: "r"(taddr), "r"(a.x), "r"(a.y), "r"(a.z), "r"(a.w), "r"(b.x), "r"(b.y), "r"(b.z), "r"(b.w)
+                 : "memory");
+}
+__device__ __forceinline__ void tm_st4(uint32_t taddr, const uint4& a) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x4.b32 [%0], {%1,%2,%3,%4};"
+                 :: "r"(taddr), "r"(a.x), "r"(a.y), "r"(a.z), "r"(a.w) : "memory");
+}
+__device__ __forceinline__ void tm_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tm_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+// Generic-proxy accesses of shared memory before this point are ordered before
+// later async-proxy (bulk copy) writes to it.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // Sentinel for vector slots past the end of a row or slice: -inf never
 // raises a maximum and adds 0 to a sum.
 template <typename In> struct NegInfRaw;
