@@ -737,11 +737,12 @@ struct TmShape {
 // This thread's chunks of a span held in tensor memory: slot s is chunk
 // v = tid + kTmThreads s (entries v kVec ..), its draft words in columns
 // 4s .. 4s+3 and its target words in t_off + 4s ..; then the ragged tail of
-// fewer than kVec entries, kept in shared memory.  f is `sweep`'s callback,
-// with the chunk's packed words by reference: kStore writes them back.
+// fewer than kVec entries, one per thread tid < tail, kept in that thread's
+// registers (tz, tt).  f is `sweep`'s callback, with the chunk's packed words by
+// reference: kStore writes them back.
 template <typename In, bool kClampZ, bool kClampT, bool kMax, bool kMin, bool kStore, typename F>
-__device__ __forceinline__ void sweep_tm(uint32_t tw, const TmShape& sh, int nv, int tail, float* tail_z,
-                                         float* tail_t, F&& f) {
+__device__ __forceinline__ void sweep_tm(uint32_t tw, const TmShape& sh, int nv, int tail, float& tz, float& tt,
+                                         F&& f) {
     using E = Elem<In>;
     constexpr int kVec = E::kVec;
     const int tid = threadIdx.x;
@@ -771,12 +772,12 @@ __device__ __forceinline__ void sweep_tm(uint32_t tw, const TmShape& sh, int nv,
     }
     if constexpr (kStore) tm_wait_st();
     if (tid < tail) {
-        float z = tail_z[tid], t = tail_t[tid];
+        float z = tz, t = tt;
         if (kClampZ) z = E::clamp1(z);
         if (kClampT) t = E::clamp1(t);
         uint4 dz{}, dt{};
         f(&z, &t, std::integral_constant<int, 1>{}, nv * kVec + tid, z, t, fminf(z, t) == kNegInf, dz, dt);
-        if constexpr (kStore) { tail_z[tid] = z; tail_t[tid] = t; }
+        if constexpr (kStore) { tz = z; tt = t; }
     }
 }
 
@@ -831,8 +832,7 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
     __shared__ float3 red_s[kT / 32];
     __shared__ int s_err;
     __shared__ float s_cu, s_cv, s_loss, s_K, s_tp;
-    __shared__ Label red_l[kT / 32];
-    __shared__ float tail_z[kVec], tail_t[kVec], tail_q[kVec];
+    __shared__ Label red_l[kKind == OSD_CE ? kT / 32 : 1];
 
     const int tid = threadIdx.x, warp = tid >> 5;
     const int csize = p.csize;
@@ -860,7 +860,8 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
     tm_fence_after_sync();
     const uint32_t tw = s_taddr + (static_cast<uint32_t>(32 * warp) << 16);
 
-    float nz = 0.f, nt = 0.f;  // the ragged tail of the row in flight
+    float nz = 0.f, nt = 0.f;  // the ragged tail entry (tid < tail) of the row in flight ...
+    float tz = 0.f, tt = 0.f, tq = 0.f;  // ... and of this row (TVD: tq = q sign(q - p) there)
     auto issue = [&](long long row) {
         const long long g = row / p.P, pp = row - g * p.P;
         const In* zsrc = static_cast<const In*>(p.draft) + g * p.dsg + pp * p.dsp + e0;
@@ -914,10 +915,8 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
             tm_st8(tw + tsh.t_off + 4 * s0, tr[0], tr[1]);
         }
         tm_wait_st();
-        if (tid < tail) {
-            tail_z[tid] = nz;
-            tail_t[tid] = nt;
-        }
+        tz = nz;
+        tt = nt;
         __syncthreads();  // the staging buffer is free; s_err is final for this row
         const int err_local = s_err;
         // a copy that gave up may still land: it stays in flight, and the exit waits for it
@@ -936,7 +935,7 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
         bool have_tp = false;
         Label lab{kNegInf, INT_MAX, 0.f};
         if (!err_local) {
-            sweep_tm<In, kClamp, kClamp, true, false, kClamp>(tw, tsh, nv, tail, tail_z, tail_t,
+            sweep_tm<In, kClamp, kClamp, true, false, kClamp>(tw, tsh, nv, tail, tz, tt,
                 [&](const float* z, const float* t, auto tag, int j0, float cz, float ct, bool, uint4&, uint4&) {
                     [[maybe_unused]] constexpr int kCnt = decltype(tag)::value;
                     if (cz > mz) {
@@ -986,7 +985,7 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
         if (!err_local) {
             const float2 gz2 = f2(gzb), gt2 = f2(gtb), tp2 = f2(tpv);
             const float2 nMz2 = f2(-Mz), nMt2 = f2(-Mt);
-            sweep_tm<In, false, false, false, kMoment, false>(tw, tsh, nv, tail, tail_z, tail_t,
+            sweep_tm<In, false, false, false, kMoment, false>(tw, tsh, nv, tail, tz, tt,
                 [&](const float* z, const float* t, auto tag, int, float, float, bool ninf, uint4&, uint4&) {
                     constexpr int kCnt = decltype(tag)::value;
                     row_ninf |= ninf;
@@ -1132,7 +1131,7 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
             // ---- pass 2: divergence terms with the global normalisers
             float2 A2 = f2(0.f), B2 = f2(0.f), C2 = f2(0.f);
             if (!row_err && !jsd_trivial) {
-                sweep_tm<In, false, false, false, false, kKind == OSD_TVD>(tw, tsh, nv, tail, tail_z, tail_t,
+                sweep_tm<In, false, false, false, false, kKind == OSD_TVD>(tw, tsh, nv, tail, tz, tt,
                     [&](const float* z, const float* t, auto tag, int j0, float, float, bool, uint4& zr, uint4& tr) {
                         constexpr int kCnt = decltype(tag)::value;
                         constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && kKind == OSD_TVD;
@@ -1175,7 +1174,7 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
                             C2 = add2(C2, c2);
                         }
                         if constexpr (kKind == OSD_TVD) {
-                            if constexpr (kCnt == 1) tail_q[j0 - tail0] = qs[0];
+                            if constexpr (kCnt == 1) tq = qs[0];
                             else pack_q<In>(qs, zr, tr);  // written back to tensor memory by the sweep
                         }
                     });
@@ -1230,7 +1229,7 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
                 const uint32_t neg = static_cast<uint32_t>(__float_as_int(q) >> 31);
                 return __uint_as_float(fpos ^ (neg & fdiff));
             };
-            sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, 0, tail_z, tail_t,
+            sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, 0, tz, tt,
                 [&](const float*, const float*, auto tag, int j0, float, float, bool, uint4& zr, uint4& tr) {
                     constexpr int kCnt = decltype(tag)::value;
                     if constexpr (kCnt == kVec) {
@@ -1246,15 +1245,12 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
                         for (int e = 0; e < kVec; e += 4) stg_v4(orow + j0 + e, gr[e], gr[e + 1], gr[e + 2], gr[e + 3]);
                     }
                 });
-            if (tid < tail) {
-                const float q = tail_q[tid];
-                orow[tail0 + tid] = q * (__float_as_int(q) < 0 ? gneg : gpos);
-            }
+            if (tid < tail) orow[tail0 + tid] = tq * (__float_as_int(tq) < 0 ? gneg : gpos);
         } else if (kKind != OSD_TVD && !row_err) {
             const float K = s_K, tpg = s_tp;
             const float2 cvs = f2(cv + p.lg_scale), cus = f2(cu + p.lg_scale);
             const int label = st.idx;
-            sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, tail, tail_z, tail_t,
+            sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, tail, tz, tt,
                 [&](const float* z, const float* t, auto tag, int j0, float, float, bool, uint4& zr, uint4& tr) {
                     constexpr int kCnt = decltype(tag)::value;
                     constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && (kKind == OSD_FKL || kKind == OSD_RKL);
@@ -1487,7 +1483,10 @@ static osd_status distill_run(const void* draft_logits, const void* target_logit
     const bool tm_path = aligned && !accepted && (kind == OSD_TVD || kind == OSD_JSD);
     int csize = 1, span = V;
     // JSD, with the most work per entry, stages best in longer spans on the per-row
-    // kernel; the TMEM-staged runs take 32 KB spans for every kind
+    // kernel; the TMEM-staged runs take the 32 KB spans for every kind.  (At
+    // V = 32000 a span of 8000 bf16 entries leaves room for seven CTAs an SM; spans
+    // cut in 16-byte steps to seven CTAs at V = 32128, five CTAs a row instead of
+    // four, measured 8 % slower for JSD than four spans of 8064 at six CTAs.)
     size_t span_bytes = (kind == OSD_JSD && !tm_path) ? kDistSpanBytesJsd : kDistSpanBytes;
     // no more rows than SMs: half-length spans put twice the CTAs to work on them
     // (measured 6-12 % less latency at 4 and 128 rows of 32000)
