@@ -269,41 +269,41 @@ __device__ __forceinline__ void seq_write_outputs(const FinParams& p, int b, con
     }
 }
 
-template <typename In, bool kVecPath>
-__global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams p) {
+// Shared memory of the extra token's draw (span_total is read by the other CTAs
+// of the cluster).
+struct DrawSmem {
+    unsigned long long span_total;
+    unsigned long long tau, W, base;
+    int owner, mode, tile;
+};
+
+// The extra token of sequence b (Appendix A.1; reading 4 and 4b for the
+// convention and the arithmetic): inverse CDF of w = max(0, p_a - q_a) when
+// a < k, of p_k when a = k.  This CTA, rank `rank` of a cluster of p.csize,
+// owns entries [e0, e0 + n) of the vocabulary: it sums their weights per
+// sub-tile (fp32 in a warp, exact 64-bit fixed point beyond), the CTAs' span
+// totals meet through distributed shared memory, and the CTA whose span holds
+// tau = floor(u W) rescans that one sub-tile exactly.  Entry j of the target and
+// draft rows at position a is trow[j - off], zrow[j - off], in shared memory when
+// kSmem (a staged span) and global memory otherwise; trow_g is the whole target
+// row in global memory, for the case W = 0 (argmax of p_a).  s_sub holds at least
+// n / (32 kW) floats.  Every thread calls it; it ends having arrived (relaxed) at
+// the cluster barrier, and the caller waits there before it exits.
+template <typename In, bool kVecPath, int kThreads, bool kSmem>
+__device__ __forceinline__ void residual_draw(const FinParams& p, int b, int a, const SeqSmem& sh, int rank,
+                                              int e0, int n, const In* trow, const In* zrow, int off,
+                                              const In* trow_g, float* s_sub, DrawSmem& ds) {
     using E = Elem<In>;
     constexpr int kW = kVecPath ? E::kVec : 1;  // entries per lane per sub-tile
     constexpr int kSub = 32 * kW;
-    constexpr int kWarps = kFinThreads / 32;
-
-    __shared__ SeqSmem sh;
-    __shared__ int s_owner, s_mode, s_tile;
-    extern __shared__ float s_sub[];  // one residual sum per sub-tile of this CTA's span
-    // residual masses in exact 64-bit fixed point (fix_of): a dependent fp64 add is slow here
-    __shared__ unsigned long long s_span_total;  // read by the other CTAs of the cluster
-    __shared__ unsigned long long s_tau, s_W, s_base;
-
+    constexpr int kWarps = kThreads / 32;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int rank = (p.csize > 1) ? static_cast<int>(cluster_rank()) : 0;
-    const int b = blockIdx.x / p.csize;
     const int k = p.k, V = p.V;
-    const In* draft = static_cast<const In*>(p.draft);
-    const In* target = static_cast<const In*>(p.target);
-
-    const int bad = seq_prologue<In, kFinThreads>(p, b, sh);
-    int32_t* out = p.out_tokens + size_t(b) * (k + 1);
-    if (bad) {  // uniform over the cluster, before any distributed shared memory access
-        if (rank == 0) seq_write_bad<kFinThreads>(p, b);
-        return;
-    }
-    seq_accept(p, b, sh, rank == 0 && p.diag_margin);
-    const int a = sh.a;
-    if (rank == 0) seq_write_outputs<kFinThreads>(p, b, sh, a);
-
-    // ---- extra token: inverse CDF of w = max(0, p_a - q_a) (a < k) or p_k (a == k)
     const bool bonus = (a == k);
-    const In* trow = target + (size_t(b) * (k + 1) + a) * V;
-    const In* zrow = draft + (size_t(b) * k + (bonus ? 0 : a)) * V;
+    int32_t* out = p.out_tokens + size_t(b) * (k + 1);
+    // entry j of the two rows: trow[j - off], zrow[j - off], from shared memory when kSmem
+    auto ldv = [&](const In* q) { return kSmem ? lds_v4(q) : ldg_stream(q); };
+    auto ld1 = [&](const In* q) { return kSmem ? E::lds(q) : E::load(q); };
     const float mt = sh.m[a], inv_st = 1.0f / sh.s[a];
     const float mz = bonus ? 0.f : sh.m[k + 1 + a];
     const float inv_sz = bonus ? 0.f : 1.0f / sh.s[k + 1 + a];
@@ -314,8 +314,6 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
         const float qj = ex2(mul_c(z - mz, ch, cl)) * inv_sz;
         return fmaxf(pj - qj, 0.f);
     };
-    const int e0 = rank * p.span;
-    const int n = max(0, min(p.span, V - e0));
     const int nsub = (n + kSub - 1) / kSub;  // sub-tiles: one warp step of 32 x kW entries
     // raw entries of this lane in sub-tile s (slots past the span read as -inf: weight 0)
     struct Raw {
@@ -325,14 +323,14 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
         const int j0 = e0 + s * kSub + lane * kW;
         const int cnt = min(kW, e0 + n - j0);
         if (kVecPath && cnt == kW) {
-            r.t = ldg_stream(trow + j0);
-            r.z = bonus ? r.t : ldg_stream(zrow + j0);
+            r.t = ldv(trow + (j0 - off));
+            r.z = bonus ? r.t : ldv(zrow + (j0 - off));
         } else {
             float tv[kW], zv[kW];
 #pragma unroll
             for (int e = 0; e < kW; ++e) {
-                tv[e] = (e < cnt) ? E::load(trow + j0 + e) : kNegInf;
-                zv[e] = (e < cnt && !bonus) ? E::load(zrow + j0 + e) : kNegInf;
+                tv[e] = (e < cnt) ? ld1(trow + (j0 - off) + e) : kNegInf;
+                zv[e] = (e < cnt && !bonus) ? ld1(zrow + (j0 - off) + e) : kNegInf;
             }
             r.t = pack_raw<In, kW>(tv);
             r.z = pack_raw<In, kW>(zv);
@@ -393,7 +391,7 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
         unsigned long long part = 0ull;
         for (int s2 = lane; s2 < nsub; s2 += 32) part += fix_of(s_sub[s2]);
         part = warp_sum_u64(part);
-        if (lane == 0) s_span_total = part;
+        if (lane == 0) ds.span_total = part;
     }
     if (p.csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
 
@@ -402,7 +400,7 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
     if (warp == 0) {
         const float u = sh.u[k];
         unsigned long long tot = 0ull;
-        if (lane < p.csize) tot = (lane == rank) ? s_span_total : ld_dsmem_u64(map_rank(&s_span_total, lane));
+        if (lane < p.csize) tot = (lane == rank) ? ds.span_total : ld_dsmem_u64(map_rank(&ds.span_total, lane));
         const unsigned long long incl = warp_incl_scan_u64(tot);
         const unsigned long long W = __shfl_sync(0xffffffffu, incl, 31);
         const unsigned long long tau = fix_scale(u, W);
@@ -457,14 +455,14 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
                 tile = last;
             }
         }
-        if (lane == 0) { s_owner = owner; s_mode = mode; s_tau = tau; s_W = W; s_base = base; s_tile = tile; }
+        if (lane == 0) { ds.owner = owner; ds.mode = mode; ds.tau = tau; ds.W = W; ds.base = base; ds.tile = tile; }
     }
     __syncthreads();
     if (p.csize > 1) cluster_arrive_relaxed();  // done reading the other CTAs' shared memory
 
-    if (rank == s_owner && warp == 0) {
-        const unsigned long long tau = s_tau, W = s_W;
-        const int mode = s_mode, s = s_tile;
+    if (rank == ds.owner && warp == 0) {
+        const unsigned long long tau = ds.tau, W = ds.W;
+        const int mode = ds.mode, s = ds.tile;
         if (mode == 0 || mode == 1) {
             float w[kW];
             {
@@ -480,7 +478,7 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
                 unsigned long long mine = 0ull;
 #pragma unroll
                 for (int e = 0; e < kW; ++e) mine += fix_of(w[e]);
-                const unsigned long long excl = s_base + warp_incl_scan_u64(mine) - mine;
+                const unsigned long long excl = ds.base + warp_incl_scan_u64(mine) - mine;
                 const bool hit = excl <= tau && excl + mine > tau;
                 if (hit) {
                     unsigned long long C = excl;
@@ -520,7 +518,7 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
             // no residual mass at all: argmax of p_a over the whole row
             MaxIdx acc{kNegInf, INT_MAX};
             for (int j = lane; j < V; j += 32) {
-                const float t = E::load(trow + j);
+                const float t = E::load(trow_g + j);
                 if (t > acc.m) { acc.m = t; acc.i = j; }
             }
             acc = warp_reduce(acc, [](MaxIdx x, MaxIdx y) { return merge_mi(x, y); });
@@ -530,7 +528,208 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
             }
         }
     }
+}
+
+template <typename In, bool kVecPath>
+__global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams p) {
+    __shared__ SeqSmem sh;
+    extern __shared__ float s_sub[];  // one residual sum per sub-tile of this CTA's span
+    // residual masses in exact 64-bit fixed point (fix_of): a dependent fp64 add is slow here
+    __shared__ DrawSmem ds;
+
+    const int rank = (p.csize > 1) ? static_cast<int>(cluster_rank()) : 0;
+    const int b = blockIdx.x / p.csize;
+    const int k = p.k, V = p.V;
+    const In* draft = static_cast<const In*>(p.draft);
+    const In* target = static_cast<const In*>(p.target);
+
+    const int bad = seq_prologue<In, kFinThreads>(p, b, sh);
+    if (bad) {  // uniform over the cluster, before any distributed shared memory access
+        if (rank == 0) seq_write_bad<kFinThreads>(p, b);
+        return;
+    }
+    seq_accept(p, b, sh, rank == 0 && p.diag_margin);
+    const int a = sh.a;
+    if (rank == 0) seq_write_outputs<kFinThreads>(p, b, sh, a);
+
+    // ---- extra token: inverse CDF of w = max(0, p_a - q_a) (a < k) or p_k (a == k)
+    {
+        const bool bonus = (a == k);
+        const In* trow = target + (size_t(b) * (k + 1) + a) * V;
+        const In* zrow = draft + (size_t(b) * k + (bonus ? 0 : a)) * V;
+        const int e0 = rank * p.span;
+        const int n = max(0, min(p.span, V - e0));
+        residual_draw<In, kVecPath, kFinThreads, false>(p, b, a, sh, rank, e0, n, trow, zrow, 0, trow, s_sub, ds);
+    }
     if (p.csize > 1) cluster_wait();  // keep this CTA's shared memory alive for its peers
+}
+
+// ------------------------------------------------------------------ one launch for small batches
+// At serving batch sizes the two launches above cost more in latency than in
+// bytes.  One thread-block cluster per sequence does both passes (T > 0): each
+// CTA bulk-copies its vocabulary span of all 2k+1 rows into shared memory,
+// computes the span's statistics of every row from there, merges them across
+// the cluster, runs the accept tests, and draws the extra token from the staged
+// rows (residual_draw) without reading them again.  At B = 32, k = 5, V = 32000
+// it measured 23.9 us against 27.1 us for the two launches (512 threads; 256
+// threads 26.7 us; 16-CTA clusters 38 us).  The greedy pass (T = 0) keeps its
+// two launches: one launch over the k+1 target rows measured 11.2 against 10.3 us.
+constexpr int kFuseThreads = 512;
+constexpr int kFuseCluster = 8;          // CTAs per sequence (above 8 needs the non-portable opt-in)
+constexpr int kFuseParts = 4;           // warp items per row for the span statistics
+constexpr int kFuseMaxB = 64;           // sequences up to which osd_verify takes one launch
+constexpr size_t kFuseMaxSmem = 200 * 1024;  // staged rows + sub-tile sums per CTA
+constexpr uint64_t kFuseWaitNs = 1000000000ull;  // bound on the wait for the staged rows
+
+// Rows of sequence b staged by this CTA: local row r <= k is target row r, r > k
+// draft row r-k-1; each holds entries [e0, e0 + n) at r * span.
+template <typename In>
+__device__ __forceinline__ const In* fused_src(const FinParams& p, int b, int r, int e0) {
+    const In* draft = static_cast<const In*>(p.draft);
+    const In* target = static_cast<const In*>(p.target);
+    return (r <= p.k) ? target + (size_t(b) * (p.k + 1) + r) * p.V + e0
+                      : draft + (size_t(b) * p.k + (r - p.k - 1)) * p.V + e0;
+}
+
+template <typename In>
+__global__ void __launch_bounds__(kFuseThreads) verify_fused_kernel(FinParams p) {
+    using E = Elem<In>;
+    constexpr int kVec = E::kVec;
+    constexpr int kWarps = kFuseThreads / 32;
+    constexpr int kMaxRows = 2 * OSD_VERIFY_MAX_K + 1;
+    extern __shared__ __align__(128) unsigned char fsm[];
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ SeqSmem sh;
+    __shared__ DrawSmem ds;
+    __shared__ MaxSum part_ms[kMaxRows * kFuseParts];
+    __shared__ MaxSum cta_ms[kMaxRows];  // this CTA's span statistics per row (read by the peers)
+    __shared__ int s_tmo, s_any_tmo;  // a staging copy gave up: this CTA's, any of the cluster's
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int csize = p.csize;
+    const int rank = (csize > 1) ? static_cast<int>(cluster_rank()) : 0;
+    const int b = blockIdx.x / csize;
+    const int k = p.k, V = p.V;
+    const int nrows = 2 * k + 1;
+    const int e0 = rank * p.span;
+    const int n = min(p.span, V - e0);
+    In* rows = reinterpret_cast<In*>(fsm);
+    float* s_sub = reinterpret_cast<float*>(fsm + size_t(nrows) * p.span * sizeof(In));
+    const uint32_t bytes = static_cast<uint32_t>(n * sizeof(In));  // a multiple of 16 on this path
+
+    // ---- stage every row's span (one barrier, all the copies in flight at once)
+    if (tid == 0) {
+        mbar_init(&bar, 1);
+        mbar_arrive_expect_tx(&bar, bytes * static_cast<uint32_t>(nrows));
+        for (int r = 0; r < nrows; ++r) bulk_g2s(rows + size_t(r) * p.span, fused_src<In>(p, b, r, e0), bytes, &bar);
+    }
+    // meanwhile the draft tokens, the two logits each accept test needs, and the uniforms
+    int bad = 0;
+    const int32_t* y = p.tokens + size_t(b) * k;
+    if (warp == kWarps - 1) {
+        for (int i = lane; i < k; i += 32) {
+            const int t = y[i];
+            sh.y[i] = t;
+            if (t < 0 || t >= V) {
+                bad = 1;
+            } else {
+                sh.zy[i] = E::load(static_cast<const In*>(p.draft) + (size_t(b) * k + i) * V + t);
+                sh.ty[i] = E::load(static_cast<const In*>(p.target) + (size_t(b) * (k + 1) + i) * V + t);
+            }
+        }
+    }
+    if (warp == kWarps - 2)
+        for (int i = lane; i <= k; i += 32) sh.u[i] = p.uniforms[size_t(b) * (k + 1) + i];
+    __syncthreads();  // the barrier is initialised before anyone waits on it
+    const int timed_out = mbar_wait_bounded(&bar, 0, kFuseWaitNs) ? 0 : 1;
+    bad = __syncthreads_or(bad);
+    const int tmo = __syncthreads_or(timed_out);
+    if (tmo) mbar_wait_bounded(&bar, 0, kFuseWaitNs);  // a copy that gave up gets a last chance to land
+    if (tid == 0) s_tmo = tmo;
+    if (bad) {  // uniform over the cluster, before any distributed shared memory access
+        if (rank == 0) seq_write_bad<kFuseThreads>(p, b);
+        return;
+    }
+
+    // ---- span statistics of every row: warp items (row, part), then per row over the parts
+    const int nch = n / kVec;
+    const float ch = p.c_hi, cl = p.c_lo;
+    for (int it = warp; it < nrows * kFuseParts; it += kWarps) {
+        const int r = it / kFuseParts, part = it - r * kFuseParts;
+        const In* row = rows + size_t(r) * p.span;
+        const int c0 = nch * part / kFuseParts, c1 = nch * (part + 1) / kFuseParts;
+        float m = kNegInf;
+        float2 s2 = f2(0.f);
+        for (int c = c0 + lane; c < c1; c += 32) {
+            const uint4 w = lds_v4(row + c * kVec);
+            const float cm = E::max_raw(w);
+            if (cm > m) {
+                s2 = (m == kNegInf) ? f2(0.f) : mul2(s2, f2(ex2(mul_c(m - cm, ch, cl))));
+                m = cm;
+            }
+            if (m != kNegInf) {
+                float x[kVec];
+                E::unpack(w, x);
+#pragma unroll
+                for (int e = 0; e < kVec; e += 2) {
+                    const float2 d = sub2(make_float2(x[e], x[e + 1]), f2(m));
+                    const float2 g = fma2(d, f2(ch), mul2(d, f2(cl)));
+                    s2 = add2(s2, make_float2(ex2(g.x), ex2(g.y)));
+                }
+            }
+        }
+        MaxSum acc{m, s2.x + s2.y};
+        acc = warp_reduce(acc, [ch, cl](MaxSum x, MaxSum z) { return merge_ms(x, z, ch, cl); });
+        if (lane == 0) part_ms[it] = acc;
+    }
+    __syncthreads();
+    if (tid < nrows) {
+        MaxSum acc = part_ms[tid * kFuseParts];
+        for (int q = 1; q < kFuseParts; ++q) acc = merge_ms(acc, part_ms[tid * kFuseParts + q], ch, cl);
+        cta_ms[tid] = acc;
+    }
+    // ---- the cluster's spans: every CTA merges all of them in rank order (lane c <- CTA c)
+    if (csize > 1) cluster_sync_publish(tid < nrows || tid == 0); else __syncthreads();
+    if (warp == 0) {  // did any CTA of the cluster miss its rows?
+        int f = 0;
+        if (lane < csize) f = (lane == rank) ? s_tmo : ld_dsmem_s32(map_rank(&s_tmo, lane));
+        f = __any_sync(0xffffffffu, f != 0);
+        if (lane == 0) s_any_tmo = f;
+    }
+    for (int r = warp; r < nrows; r += kWarps) {
+        MaxSum o{kNegInf, 0.f};
+        if (lane < csize) {
+            if (lane == rank) {
+                o = cta_ms[r];
+            } else {
+                const uint32_t base = map_rank(&cta_ms[r], lane);
+                o.m = ld_dsmem_f32(base + offsetof(MaxSum, m));
+                o.s = ld_dsmem_f32(base + offsetof(MaxSum, s));
+            }
+        }
+        o = warp_reduce(o, [ch, cl](MaxSum x, MaxSum z) { return merge_ms(x, z, ch, cl); });
+        if (lane == 0) { sh.m[r] = o.m; sh.s[r] = o.s; }
+    }
+    __syncthreads();
+    if (s_any_tmo) {  // the GPU did not deliver a row in time: the sequence is reported as bad
+        if (rank == 0) seq_write_bad<kFuseThreads>(p, b);
+        if (csize > 1) {
+            cluster_arrive_relaxed();
+            cluster_wait();
+        }
+        return;
+    }
+
+    seq_accept(p, b, sh, rank == 0 && p.diag_margin);
+    const int a = sh.a;
+    if (rank == 0) seq_write_outputs<kFuseThreads>(p, b, sh, a);
+    // ---- extra token from the staged rows at position a
+    const bool bonus = (a == k);
+    const In* trow_s = rows + size_t(a) * p.span;
+    const In* zrow_s = bonus ? trow_s : rows + size_t(k + 1 + a) * p.span;
+    const In* trow_g = static_cast<const In*>(p.target) + (size_t(b) * (k + 1) + a) * V;
+    residual_draw<In, true, kFuseThreads, true>(p, b, a, sh, rank, e0, n, trow_s, zrow_s, e0, trow_g, s_sub, ds);
+    if (csize > 1) cluster_wait();  // keep this CTA's shared memory alive for its peers
 }
 
 // ------------------------------------------------------------------ host
@@ -561,6 +760,52 @@ static void finalize_shape(int B, int V, int sub, int* csize, int* span) {
     *span = s;
 }
 
+// One launch for small batches: the cluster shape and shared memory, or false
+// when the rows are not 16-byte aligned, the batch is large, or the staged rows
+// do not fit (the two-launch path then runs).
+template <typename In>
+static bool fused_shape(int B, int k, int V, bool greedy, const void* draft, const void* target, int* csize,
+                        int* span, size_t* smem) {
+    if (greedy || B > kFuseMaxB) return false;
+    if (!aligned_to(target, 16) || !aligned_to(draft, 16) || ((size_t)V * sizeof(In)) % 16 != 0) return false;
+    int c = kFuseCluster;
+    int s = (V + c - 1) / c;
+    s = (s + 63) / 64 * 64;
+    c = (V + s - 1) / s;
+    const int nrows = 2 * k + 1;
+    const size_t bytes = size_t(nrows) * s * sizeof(In) + size_t(s / 128 + 1) * sizeof(float);
+    if (bytes > kFuseMaxSmem) return false;
+    *csize = c;
+    *span = s;
+    *smem = bytes;
+    return true;
+}
+template <typename In>
+static cudaError_t launch_fused(const FinParams& fp, size_t smem, cudaStream_t stream) {
+    auto kern = verify_fused_kernel<In>;
+    {
+        // dynamic plus static shared memory passes 48 KB from a few rows on: opt in.  The
+        // opt-in only grows, once per device, so later calls (and captures) make no attribute call
+        static std::mutex mu;
+        static size_t allowed[64] = {};
+        int dev = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e != cudaSuccess) return e;
+        if (dev < 0 || dev >= 64) return cudaErrorInvalidValue;
+        std::lock_guard<std::mutex> lock(mu);
+        if (allowed[dev] < smem) {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+            if (e != cudaSuccess) return e;
+            if (kFuseCluster > 8) {
+                e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+                if (e != cudaSuccess) return e;
+            }
+            allowed[dev] = smem;
+        }
+    }
+    return launch(kern, dim3(unsigned(fp.B) * unsigned(fp.csize)), dim3(kFuseThreads), smem, stream, fp.csize, fp);
+}
+
 template <typename In>
 static osd_status launch_verify(const void* draft, const void* target, int B, int k, int V,
                                 const int32_t* tokens, const float* uniforms, float T,
@@ -568,6 +813,21 @@ static osd_status launch_verify(const void* draft, const void* target, int B, in
                                 float* diag_margin, float* diag_gap, RowStat* stats,
                                 cudaStream_t stream) {
     const bool greedy = (T == 0.f);
+    {
+        int fc = 1, fspan = V;
+        size_t fsmem = 0;
+        if (fused_shape<In>(B, k, V, greedy, draft, target, &fc, &fspan, &fsmem)) {
+            FinParams fp = {};
+            fp.draft = draft; fp.target = target; fp.B = B; fp.k = k; fp.V = V;
+            fp.tokens = tokens; fp.uniforms = uniforms; fp.T = T;
+            split_scale(T, &fp.c_hi, &fp.c_lo);
+            fp.accepted = accepted; fp.out_tokens = out_tokens; fp.mask = mask;
+            fp.diag_margin = diag_margin; fp.diag_gap = diag_gap;
+            fp.csize = fc;
+            fp.span = fspan;
+            return from_cuda(launch_fused<In>(fp, fsmem, stream));
+        }
+    }
     const int slice_len = verify_slice_len(B, k);
     const int n_slices = verify_slices(B, k, V);
     const long long n_draft_rows = greedy ? 0 : (long long)B * k;
