@@ -256,3 +256,21 @@ def test_many_rows_long_spans_sampled(osd, kind):
     skip = _tvd_ambiguous(zs, ts, 0.9) if kind == "tvd" else None
     check_distill(loss[idx].cpu().numpy(), g[idx].cpu().numpy(), lr, gr, np.ones(8, bool), skip)
     assert not torch.isnan(g).any()
+
+
+@pytest.mark.parametrize("kind", ["tvd", "jsd"])
+@pytest.mark.parametrize("V", [8196, 32004, 100, 12])
+def test_single_row_ragged_tail(osd, kind, V):
+    """One bf16 row with V = 4 (mod 8): the row is on the 16-byte path, and its last span ends
+    in a tail of 4 entries shorter than a 16-byte chunk (the TMEM-staged kernel keeps those in
+    registers; TVD keeps q sign(q - p) there for its gradient)."""
+    g0 = torch.Generator().manual_seed(V)
+    z = (torch.randn(1, V, generator=g0) * 2).to(torch.bfloat16)
+    t = (z.float() + torch.randn(1, V, generator=g0)).to(torch.bfloat16)
+    t[0, V - 1] = 9.0   # mass in the tail itself
+    z[0, V - 2] = 7.0
+    for tau in (1.0, 0.8):
+        lg, gg = _run(osd, z, t, None, kind, 0.4, tau=tau)
+        lr, gr = _oracle(z, t, None, kind, 0.4, tau=tau)
+        skip = _tvd_ambiguous(z, t, tau) if kind == "tvd" else None
+        check_distill(lg, gg, lr, gr, np.ones(1, bool), skip)
