@@ -711,8 +711,8 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
 }
 
 // ------------------------------------------------------------------ TMEM-staged runs of rows
-// The same passes over the same spans, but each cluster walks a run of
-// kTmRows consecutive rows.  A row's span lands in shared memory by bulk copy
+// The same passes over the same spans, but each cluster walks a run of up to
+// kTmRows consecutive rows (the last runs shorter, see launch_distill_tm).  A row's span lands in shared memory by bulk copy
 // as above, is moved at once into tensor memory (each thread owns one
 // tensor-memory lane and keeps its 16-byte chunks in that lane's columns), and
 // the next active row's bulk copy then goes into the freed shared memory while
@@ -732,6 +732,10 @@ struct TmShape {
     int slots;       // 16-byte chunks of each row per thread
     int t_off;       // first column of the target words (z words from column 0)
     uint32_t ncols;  // tensor-memory columns per CTA
+    // runs, longest first: rows [0, end8) in runs of kTmRows, [end8, end2) in runs
+    // of 2, then runs of one row; n8 and n2 runs of the first two kinds
+    long long end8, end2;
+    int n8, n2;
 };
 
 // This thread's chunks of a span held in tensor memory: slot s is chunk
@@ -878,8 +882,17 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
         }
     };
     // this cluster's run of rows; masked-out rows get loss 0 and are skipped
-    const long long r0 = static_cast<long long>(cid) * kTmRows;
-    const long long r1 = min(rows, r0 + kTmRows);
+    long long r0, r1;
+    if (cid < tsh.n8) {
+        r0 = static_cast<long long>(cid) * kTmRows;
+        r1 = min(tsh.end8, r0 + kTmRows);
+    } else if (cid < tsh.n8 + tsh.n2) {
+        r0 = tsh.end8 + 2ll * (cid - tsh.n8);
+        r1 = min(tsh.end2, r0 + 2);
+    } else {
+        r0 = tsh.end2 + (cid - tsh.n8 - tsh.n2);
+        r1 = min(rows, r0 + 1);
+    }
     auto active = [&](long long r) { return !p.mask || p.mask[r] != 0; };
     if (p.mask && rank == 0 && tid == 0)
         for (long long r = r0; r < r1; ++r)
@@ -1378,6 +1391,7 @@ static cudaError_t launch_distill_dtype(osd_loss kind, const DistParams& dp, lon
 struct TmLaunch {
     TmShape shape;
     size_t smem;
+    int occ;  // resident CTAs an SM
 };
 template <typename In, int kKind>
 static cudaError_t tm_launch_shape(int span, TmLaunch* out) {
@@ -1392,6 +1406,7 @@ static cudaError_t tm_launch_shape(int span, TmLaunch* out) {
     struct Entry {
         int dev, span;
         size_t smem;
+        int occ;
     };
     static std::mutex mu;
     static Entry cache[64];
@@ -1403,8 +1418,9 @@ static cudaError_t tm_launch_shape(int span, TmLaunch* out) {
         std::lock_guard<std::mutex> lock(mu);
         for (int i = 0; i < n_cache; ++i)
             if (cache[i].dev == dev && cache[i].span == span) {
-                out->shape = TmShape{slots, t_off, ncols};
+                out->shape = TmShape{slots, t_off, ncols, 0, 0, 0, 0};
                 out->smem = cache[i].smem;
+                out->occ = cache[i].occ;
                 return cudaSuccess;
             }
     }
@@ -1436,10 +1452,11 @@ static cudaError_t tm_launch_shape(int span, TmLaunch* out) {
     if (occ < 1 || occ * static_cast<int>(ncols) > 512) return cudaErrorInvalidValue;
     {
         std::lock_guard<std::mutex> lock(mu);
-        if (n_cache < 64) cache[n_cache++] = Entry{dev, span, smem};
+        if (n_cache < 64) cache[n_cache++] = Entry{dev, span, smem, occ};
     }
-    out->shape = TmShape{slots, t_off, ncols};
+    out->shape = TmShape{slots, t_off, ncols, 0, 0, 0, 0};
     out->smem = smem;
+    out->occ = occ;
     return cudaSuccess;
 }
 template <typename In, int kKind>
@@ -1447,9 +1464,22 @@ static cudaError_t launch_distill_tm(const DistParams& dp, long long rows, cudaS
     TmLaunch tl;
     const cudaError_t e = tm_launch_shape<In, kKind>(dp.span, &tl);
     if (e != cudaSuccess) return e;
-    const long long runs = (rows + kTmRows - 1) / kTmRows;
+    // Longest runs first: the hardware hands out clusters in about index order, so
+    // the last rows, in runs of 2 and then of 1, even out the clusters' finishing
+    // times (K = the clusters resident at once: the last K rows singly, the 2K
+    // before them in pairs).  With runs of 8 throughout, 6554 rows over about 228
+    // resident clusters left some clusters 32 rows and others 24.
+    const long long K = std::max<long long>(1, static_cast<long long>(device_sms()) * tl.occ / dp.csize);
+    const long long ones = std::min(rows, K);
+    const long long twos = std::min(rows - ones, 2 * K);
+    TmShape sh = tl.shape;
+    sh.end2 = rows - ones;
+    sh.end8 = sh.end2 - twos;
+    sh.n8 = static_cast<int>((sh.end8 + kTmRows - 1) / kTmRows);
+    sh.n2 = static_cast<int>((twos + 1) / 2);
+    const long long runs = sh.n8 + sh.n2 + ones;
     return launch(distill_tm_kernel<In, kKind>, dim3(static_cast<unsigned>(runs * dp.csize)), dim3(kTmThreads),
-                  tl.smem, s, dp.csize, dp, tl.shape);
+                  tl.smem, s, dp.csize, dp, sh);
 }
 template <typename In>
 static cudaError_t launch_distill_tm_kind(osd_loss kind, const DistParams& dp, long long rows, cudaStream_t s) {
