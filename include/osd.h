@@ -113,8 +113,8 @@ osd_status osd_verify_workspace_size(int B, int k, int V, size_t *bytes);
  * uniforms       [B, k+1]     fp32 in [0, 1) (not read when T == 0)
  * temperature    >= 0 and finite, else OSD_ERR_INVALID_ARG
  * accepted       [B]          out: a in 0..k; -1 if any draft token of the
- *                             sequence lies outside [0, V), or (batches of up
- *                             to 64 sequences at T > 0, staged by bulk copy) if
+ *                             sequence lies outside [0, V), or (small batches
+ *                             at T > 0, whose rows are staged by bulk copy) if
  *                             the GPU did not deliver the sequence's rows within
  *                             a one-second bound
  * out_tokens     [B, k+1]     out: y_0..y_{a-1}, the sampled token at a, then -1

@@ -28,6 +28,7 @@
 // log-sum-exp is rounded on its own.
 #include <cuda.h>
 
+#include <atomic>
 #include <climits>
 #include <cstdint>
 #include <mutex>
@@ -570,14 +571,15 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
 // CTA bulk-copies its vocabulary span of all 2k+1 rows into shared memory,
 // computes the span's statistics of every row from there, merges them across
 // the cluster, runs the accept tests, and draws the extra token from the staged
-// rows (residual_draw) without reading them again.  At B = 32, k = 5, V = 32000
-// it measured 23.9 us against 27.1 us for the two launches (512 threads; 256
-// threads 26.7 us; 16-CTA clusters 38 us).  The greedy pass (T = 0) keeps its
-// two launches: one launch over the k+1 target rows measured 11.2 against 10.3 us.
+// rows (residual_draw) without reading them again.  It runs only when its grid
+// fits in one wave (fused_shape).  At B = 32, k = 5, V = 32000 it measured 23.9 us
+// in the bench step against 27.1 us for the two launches (512 threads; 256 threads
+// 26.7 us; 16-CTA clusters 38 us).  The greedy pass (T = 0) keeps its two
+// launches: one launch over the k+1 target rows measured 11.2 against 10.3 us.
 constexpr int kFuseThreads = 512;
 constexpr int kFuseCluster = 8;          // CTAs per sequence (above 8 needs the non-portable opt-in)
 constexpr int kFuseParts = 4;           // warp items per row for the span statistics
-constexpr int kFuseMaxB = 64;           // sequences up to which osd_verify takes one launch
+constexpr int kFuseMaxB = 64;           // at most this many sequences, and the grid in one wave
 constexpr size_t kFuseMaxSmem = 200 * 1024;  // staged rows + sub-tile sums per CTA
 constexpr uint64_t kFuseWaitNs = 1000000000ull;  // bound on the wait for the staged rows
 
@@ -760,9 +762,37 @@ static void finalize_shape(int B, int V, int sub, int* csize, int* span) {
     *span = s;
 }
 
+// Resident CTAs an SM of the one-launch kernel with `smem` bytes of dynamic shared
+// memory, or 0 when a query fails.  The opt-in for that much shared memory is set
+// here first; both are kept per device for the last size asked, so repeated calls
+// (and calls under stream capture) make no runtime query.
+template <typename In>
+static int fused_ctas_per_sm(size_t smem) {
+    auto kern = verify_fused_kernel<In>;
+    static std::mutex mu;
+    static size_t allowed[64] = {};
+    static size_t last_smem[64] = {};
+    static int last_occ[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    std::lock_guard<std::mutex> lock(mu);
+    if (last_smem[dev] == smem && last_occ[dev] > 0) return last_occ[dev];
+    if (allowed[dev] < smem) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
+            cudaSuccess)
+            return 0;
+        allowed[dev] = smem;
+    }
+    int occ = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kFuseThreads, smem) != cudaSuccess) return 0;
+    last_smem[dev] = smem;
+    last_occ[dev] = occ;
+    return occ;
+}
+
 // One launch for small batches: the cluster shape and shared memory, or false
-// when the rows are not 16-byte aligned, the batch is large, or the staged rows
-// do not fit (the two-launch path then runs).
+// when the rows are not 16-byte aligned, the staged rows do not fit, or the
+// grid would not fit in one wave (the two-launch path then runs).
 template <typename In>
 static bool fused_shape(int B, int k, int V, bool greedy, const void* draft, const void* target, int* csize,
                         int* span, size_t* smem) {
@@ -775,32 +805,29 @@ static bool fused_shape(int B, int k, int V, bool greedy, const void* draft, con
     const int nrows = 2 * k + 1;
     const size_t bytes = size_t(nrows) * s * sizeof(In) + size_t(s / 128 + 1) * sizeof(float);
     if (bytes > kFuseMaxSmem) return false;
+    // only in one wave: at B = 32, k = 5, V = 32000 (two CTAs an SM) one launch took
+    // 22.2 us against 23.2 us for two; from B = 48 on, past one wave, 34 against 26 us
+    const long long ctas = (long long)B * c;
+    if (ctas > (long long)device_sms() * fused_ctas_per_sm<In>(bytes)) return false;
     *csize = c;
     *span = s;
     *smem = bytes;
     return true;
 }
+// The one-launch kernel (fused_shape has set its shared-memory opt-in).
 template <typename In>
 static cudaError_t launch_fused(const FinParams& fp, size_t smem, cudaStream_t stream) {
     auto kern = verify_fused_kernel<In>;
-    {
-        // dynamic plus static shared memory passes 48 KB from a few rows on: opt in.  The
-        // opt-in only grows, once per device, so later calls (and captures) make no attribute call
-        static std::mutex mu;
-        static size_t allowed[64] = {};
+    if (kFuseCluster > 8) {
+        static std::atomic<int> nonportable[64];
         int dev = 0;
         cudaError_t e = cudaGetDevice(&dev);
         if (e != cudaSuccess) return e;
         if (dev < 0 || dev >= 64) return cudaErrorInvalidValue;
-        std::lock_guard<std::mutex> lock(mu);
-        if (allowed[dev] < smem) {
-            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+        if (!nonportable[dev].load(std::memory_order_relaxed)) {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
             if (e != cudaSuccess) return e;
-            if (kFuseCluster > 8) {
-                e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-                if (e != cudaSuccess) return e;
-            }
-            allowed[dev] = smem;
+            nonportable[dev].store(1, std::memory_order_relaxed);
         }
     }
     return launch(kern, dim3(unsigned(fp.B) * unsigned(fp.csize)), dim3(kFuseThreads), smem, stream, fp.csize, fp);
