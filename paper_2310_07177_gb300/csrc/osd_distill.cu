@@ -720,9 +720,11 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
 // of row i, with the shared-memory footprint of one staged span per CTA.  The
 // hardware schedules the runs like any grid (no assumption on how many
 // clusters are resident), and masked-out rows of a run cost one mask read.
-// 16-byte-aligned rows.  The kernel handles every loss kind (all five passed the
-// parity tests on it); the launcher uses it for TVD and JSD, the kinds with a
-// second pass, where it measured faster than the per-row kernel.
+// 16-byte-aligned rows; TVD and JSD, the kinds with a second pass over the
+// normalised distributions (FKL, RKL and CE measured slower on an earlier form of
+// these runs than on the per-row kernel).  A row costs two cluster barriers and
+// one CTA barrier: pass 0 and pass 1 fold into one sweep with running maxima, and
+// each warp publishes its own partials, which every warp then merges.
 constexpr int kTmThreads = 128;  // one warp per tensor-memory lane quarter
 constexpr int kTmG = 2;          // chunk slots per round of tensor-memory loads
 constexpr int kTmRows = 8;       // rows per cluster run
@@ -819,26 +821,64 @@ __device__ __forceinline__ void unpack_q(const uint4& zr, const uint4& tr, float
     }
 }
 
-template <typename In, int kKind>
-__global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, TmShape tsh) {
-    constexpr int kT = kTmThreads;
-    constexpr int kVec = Elem<In>::kVec;
-    constexpr bool kClamp = kKind == OSD_JSD;
-    constexpr bool kMoment = kKind == OSD_FKL || kKind == OSD_RKL;
-    constexpr bool kNeedEt = kKind != OSD_CE;
-    constexpr bool kFold = !kClamp;
-    extern __shared__ __align__(128) unsigned char dsm[];
-    __shared__ __align__(8) uint64_t bar;
-    __shared__ uint32_t s_taddr;
-    __shared__ Stats1 s1_mine, s1_all;
-    __shared__ Stats2 s2_mine, s2_all;
-    __shared__ float2 red_m[kT / 32];
-    __shared__ float3 red_s[kT / 32];
-    __shared__ int s_err;
-    __shared__ float s_cu, s_cv, s_loss, s_K, s_tp;
-    __shared__ Label red_l[kKind == OSD_CE ? kT / 32 : 1];
+// A row's statistics travel without cluster barriers: each warp reduces its
+// partial and leaves it in a slot of its CTA (arriving on named barrier 1, where
+// warp 0 waits); warp 0 merges the slots into the CTA's partial and pushes it
+// with st.async into slot `rank` of every CTA's receive buffer, where it
+// completes 16 bytes on that CTA's barrier for the pass; warp 0 of each CTA then
+// merges the csize partials, in rank order, and hands the result to the other
+// warps through named barrier 2 (they wait, it arrives).  Every
+// CTA sees the same partials in the same order, so all reach the same bits.  The
+// two passes use two receive buffers and barriers: a CTA pushes its next partial
+// for a pass only after every CTA's partial of the pass in between has reached
+// it, and that one comes from each peer only once the peer has read the buffer.
+__device__ __forceinline__ float warp_max(float x) {
+    for (int off = 16; off > 0; off >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, off));
+    return x;
+}
+__device__ __forceinline__ float warp_sum(float x) {
+    // the butterfly leaves the same bits in every lane (each step adds the same two values)
+    for (int off = 16; off > 0; off >>= 1) x += __shfl_xor_sync(0xffffffffu, x, off);
+    return x;
+}
+// log2 of a sum of exponentials that is at least 1 (the term of the maximum):
+// the exponent plus lg2.approx of the mantissa in [1, 2), absolute error about
+// 2^-22 there; anything else (0, inf, NaN) through log2f
+__device__ __forceinline__ float log2_sum(float x) {
+    if (!(x >= 1.f && x <= 3.0e38f)) return log2f(x);
+    const uint32_t b = __float_as_uint(x);
+    return static_cast<float>(static_cast<int>(b >> 23) - 127) + lg2(__uint_as_float((b & 0x007fffffu) | 0x3f800000u));
+}
+constexpr bool kTmOnlineJsd = false;
+constexpr uint64_t kTmPartWaitNs = 3000000000ull;  // partials: peers may first wait out their copies
+// Named barriers 1 and 2 of the CTA (0 is __syncthreads): `arrive` marks the
+// warp's arrival without waiting (release), `sync` waits for all kTmThreads (acquire).
+__device__ __forceinline__ void named_arrive(int id) {
+    asm volatile("bar.arrive %0, %1;" :: "r"(id), "n"(kTmThreads) : "memory");
+}
+__device__ __forceinline__ void named_sync(int id) {
+    asm volatile("bar.sync %0, %1;" :: "r"(id), "n"(kTmThreads) : "memory");
+}
 
-    const int tid = threadIdx.x, warp = tid >> 5;
+template <typename In, int kKind>
+__global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p, TmShape tsh) {
+    static_assert(kKind == OSD_TVD || kKind == OSD_JSD, "the TMEM-staged runs serve TVD and JSD");
+    constexpr int kT = kTmThreads, kW = kT / 32;
+    constexpr int kVec = Elem<In>::kVec;
+    constexpr bool kJsd = kKind == OSD_JSD;
+    // TVD: exponent arguments x c - m c as one fma; JSD: logits clamped to -1e30, (x - m) c
+    constexpr bool kFold = !kJsd;
+    // pass 0 and pass 1 as one sweep with running maxima (TVD), or as two sweeps
+    // with the warp's maxima in between (JSD)
+    constexpr bool kOnline = kTmOnlineJsd || !kJsd;
+    extern __shared__ __align__(128) unsigned char dsm[];
+    __shared__ __align__(8) uint64_t bar, pbar1, pbar2;
+    __shared__ uint32_t s_taddr;
+    __shared__ float4 s_slot[kW];  // the warps' partials of the pass in progress
+    __shared__ float4 s_res;       // warp 0's merged result of the pass in progress ...
+    __shared__ int s_rerr;         // ... and whether the row failed
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int csize = p.csize;
     const float c = p.c, inv_tau = p.inv_tau;
     const int rank = (csize > 1) ? static_cast<int>(cluster_rank()) : 0;
@@ -851,26 +891,36 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
     const uint32_t bytes = static_cast<uint32_t>(tail0 * sizeof(In));
     In* zs = reinterpret_cast<In*>(dsm);
     In* ts = zs + p.span;
+    float4* recv1 = reinterpret_cast<float4*>(ts + p.span);  // [csize] CTA partials of pass 0+1
+    float4* recv2 = recv1 + csize;                          // [csize] CTA partials of pass 2
 
     // tensor memory for this CTA (the launch keeps resident CTAs x columns <= 512,
-    // so the allocation never waits), and the staging barrier
+    // so the allocation never waits), and the barriers
     if (warp == 0) tm_alloc(&s_taddr, tsh.ncols);
     if (tid == 0) {
         mbar_init(&bar, 1);
-        s_err = 0;
+        mbar_init(&pbar1, 1);
+        mbar_init(&pbar2, 1);
     }
     tm_fence_before_sync();
-    __syncthreads();
+    if (csize > 1) {  // every CTA's barriers are initialised before any peer pushes to them
+        __syncwarp();
+        asm volatile("barrier.cluster.arrive.release.aligned;\n"
+                     "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+    } else {
+        __syncthreads();
+    }
     tm_fence_after_sync();
     const uint32_t tw = s_taddr + (static_cast<uint32_t>(32 * warp) << 16);
 
     float nz = 0.f, nt = 0.f;  // the ragged tail entry (tid < tail) of the row in flight ...
     float tz = 0.f, tt = 0.f, tq = 0.f;  // ... and of this row (TVD: tq = q sign(q - p) there)
-    auto issue = [&](long long row) {
+    // the bulk copies of a row's span (tid 0, when `copy`) and its tail entries
+    auto issue = [&](long long row, bool copy) {
         const long long g = row / p.P, pp = row - g * p.P;
         const In* zsrc = static_cast<const In*>(p.draft) + g * p.dsg + pp * p.dsp + e0;
         const In* tsrc = static_cast<const In*>(p.target) + g * p.tsg + pp * p.tsp + e0;
-        if (tid == 0 && bytes) {
+        if (tid == 0 && bytes && copy) {
             fence_proxy_async_smem();  // this CTA's reads of the staging buffer come first
             mbar_arrive_expect_tx(&bar, 2 * bytes);
             bulk_g2s(zs, zsrc, bytes, &bar);
@@ -899,23 +949,33 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
             if (!p.mask[r]) p.loss[r] = 0.f;
     long long row = r0;
     while (row < r1 && !active(row)) ++row;
-    bool inflight = false;
-    uint32_t infl_phase = 0;  // the barrier phase the copy in flight completes
+    // tid 0: a copy issued and not yet seen landed, and the barrier phase it completes
+    bool pending = false;
+    uint32_t pend_phase = 0;
     if (row < r1) {
-        issue(row);
-        inflight = true;
+        issue(row, true);
+        pending = true;
     }
-    uint32_t phase = 0;
+    auto to_ref = [c](float m, float g) {  // 2^((m - g) c), rounded as the terms are
+        if (m == kNegInf) return 0.f;
+        return kFold ? ex2(__fmul_rn(m, c) - __fmul_rn(g, c)) : ex2((m - g) * c);
+    };
+    const float beta = p.beta;
+    const bool jsd_trivial = kJsd && (beta == 0.f || beta == 1.f);
+    uint32_t phase = 0;  // the staging barrier's phase for this row
+    uint32_t pph = 0;    // pbar1 and pbar2: one phase per row
+    bool gave_up = false;  // warp 0: a wait for the peers' partials ran out
     bool stop = false;
     for (long long next; row < r1; row = next, phase ^= 1u) {
         next = row + 1;
         while (next < r1 && !active(next)) ++next;
-        if (stop) {  // a copy gave up earlier: the rest of this run reports NaN
+        if (stop) {  // a wait gave up earlier: the rest of this run reports NaN
             if (rank == 0 && tid == 0) p.loss[row] = __int_as_float(0x7fc00000);
             continue;
         }
         // ---- this row's span: shared memory (bounded wait) -> tensor memory
-        if (bytes && !mbar_wait_bounded(&bar, phase, kStageWaitNs)) atomicOr(&s_err, 1);
+        const bool landed = !bytes || mbar_wait_bounded(&bar, phase, kStageWaitNs);
+        if (tid == 0 && landed) pending = false;
         for (int s0 = 0; s0 < tsh.slots; s0 += kTmG) {
             uint4 zr[kTmG], tr[kTmG];
 #pragma unroll
@@ -930,318 +990,263 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
         tm_wait_st();
         tz = nz;
         tt = nt;
-        __syncthreads();  // the staging buffer is free; s_err is final for this row
-        const int err_local = s_err;
-        // a copy that gave up may still land: it stays in flight, and the exit waits for it
-        inflight = err_local != 0;
-        infl_phase = phase;
-        // ---- the next active row's copy goes in flight while this row is processed
-        if (next < r1 && !err_local) {
-            issue(next);
-            inflight = true;
-            infl_phase = phase ^ 1u;
+        __syncthreads();  // the staging buffer is free
+        // ---- the next active row's copy goes in flight while this row is
+        // processed; after a copy that gave up (which may still land) none does
+        if (next < r1) {
+            issue(next, landed);
+            if (tid == 0 && landed) {
+                pending = true;
+                pend_phase = phase ^ 1u;
+            }
         }
 
-        // ---- pass 0: this thread's maxima (RKL: the target logit at the draft
-        // maximum; CE: the first target maximum and the draft logit there)
-        float mz = kNegInf, mt = kNegInf, tp = 0.f;
-        bool have_tp = false;
-        Label lab{kNegInf, INT_MAX, 0.f};
-        if (!err_local) {
-            sweep_tm<In, kClamp, kClamp, true, false, kClamp>(tw, tsh, nv, tail, tz, tt,
-                [&](const float* z, const float* t, auto tag, int j0, float cz, float ct, bool, uint4&, uint4&) {
-                    [[maybe_unused]] constexpr int kCnt = decltype(tag)::value;
-                    if (cz > mz) {
-                        mz = cz;
-                        if constexpr (kKind == OSD_RKL) {
-#pragma unroll
-                            for (int e = kCnt - 1; e >= 0; --e)
-                                if (z[e] == cz) tp = t[e];
-                            have_tp = true;
-                        }
-                    }
-                    if (ct > mt) {
-                        mt = ct;
-                        if constexpr (kKind == OSD_CE) {
-                            int ei = 0;
-                            float zl = z[0];
-#pragma unroll
-                            for (int e = kCnt - 1; e >= 0; --e)
-                                if (t[e] == ct) { ei = e; zl = z[e]; }
-                            lab = Label{ct, e0 + j0 + ei, zl};
-                        }
-                    }
+        float mz = kNegInf, mt = kNegInf;
+        float2 Ez2 = f2(0.f), Et2 = f2(0.f);
+        if constexpr (!kOnline) {
+            // ---- pass 0: this warp's maxima (JSD: clamped logits kept), then pass 1:
+            // sums of 2^((x - m) c) against them
+            sweep_tm<In, kJsd, kJsd, true, false, kJsd>(tw, tsh, nv, tail, tz, tt,
+                [&](const float*, const float*, auto, int, float cz, float ct, bool, uint4&, uint4&) {
+                    mz = fmaxf(mz, cz);
+                    mt = fmaxf(mt, ct);
                 });
-        }
-        if (kKind == OSD_RKL && (!have_tp || tp == kNegInf)) tp = 0.f;
-        float gzb, gtb, tpv = 0.f;
-        Label bl{kNegInf, INT_MAX, 0.f};
-        if constexpr (kKind == OSD_RKL) {
-            const float3 r = block_max_pivot<kT>(mz, tp, mt, red_s);
-            gzb = r.x;
-            tpv = r.y;
-            gtb = r.z;
-        } else {
-            const float2 bm = block_max2<true, kT>(mz, mt, red_m);
-            gzb = bm.x;
-            gtb = bm.y;
-            if constexpr (kKind == OSD_CE)
-                bl = block_reduce<kT>(lab, [](Label a, Label b) { return merge_label(a, b); }, red_l);
-        }
-
-        // ---- pass 1: sums of 2^((x - m) c) against the block maxima (+ the FKL/RKL moment)
-        bool row_ninf = false, rkl_inf = false;
-        float2 Ez2 = f2(0.f), Et2 = f2(0.f), X2 = f2(0.f);
-        const bool zok = kClamp || gzb != kNegInf;
-        const bool tok = kNeedEt && (kClamp || gtb != kNegInf);
-        const float Mz = zok ? __fmul_rn(gzb, c) : 0.f, Mt = tok ? __fmul_rn(gtb, c) : 0.f;
-        if (!err_local) {
-            const float2 gz2 = f2(gzb), gt2 = f2(gtb), tp2 = f2(tpv);
-            const float2 nMz2 = f2(-Mz), nMt2 = f2(-Mt);
-            sweep_tm<In, false, false, false, kMoment, false>(tw, tsh, nv, tail, tz, tt,
-                [&](const float* z, const float* t, auto tag, int, float, float, bool ninf, uint4&, uint4&) {
+            mz = warp_max(mz);
+            mt = warp_max(mt);
+            const float Mz = __fmul_rn(mz, c), Mt = __fmul_rn(mt, c);
+            sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, tail, tz, tt,
+                [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4&, uint4&) {
                     constexpr int kCnt = decltype(tag)::value;
-                    row_ninf |= ninf;
-                    if (kCnt == 1 || ninf) {
-#pragma unroll
-                        for (int e = 0; e < kCnt; ++e) {
-                            if (zok) {
-                                const float ez = kFold ? ex2(fmaf(z[e], c, -Mz)) : ex2((z[e] - gzb) * c);
-                                Ez2.x += ez;
-                                if (kKind == OSD_RKL && z[e] != kNegInf) {
-                                    if (t[e] == kNegInf) rkl_inf = true;
-                                    else X2.x = fmaf(ez, (z[e] - gzb) - (t[e] - tpv), X2.x);
-                                }
-                            }
-                            if (tok) {
-                                const float et = kFold ? ex2(fmaf(t[e], c, -Mt)) : ex2((t[e] - gtb) * c);
-                                Et2.x += et;
-                                if (kKind == OSD_FKL && et > 0.f) X2.x = fmaf(et, t[e] - z[e], X2.x);
-                            }
-                        }
+                    if constexpr (kCnt == 1) {
+                        if (mz != kNegInf) Ez2.x += kFold ? ex2(fmaf(z[0], c, -Mz)) : ex2((z[0] - mz) * c);
+                        if (mt != kNegInf) Et2.x += kFold ? ex2(fmaf(t[0], c, -Mt)) : ex2((t[0] - mt) * c);
                     } else {
 #pragma unroll
                         for (int e = 0; e < kCnt; e += 2) {
-                            const float2 zz = make_float2(z[e], z[e + 1]);
-                            float2 a;
-                            if constexpr (kFold) a = fma2(zz, f2(c), nMz2);
-                            else a = mul2(sub2(zz, gz2), f2(c));
-                            const float2 ez = make_float2(ex2(a.x), ex2(a.y));
-                            Ez2 = add2(Ez2, ez);
-                            if (kKind == OSD_RKL)
-                                X2 = fma2(ez, sub2(sub2(zz, gz2), sub2(make_float2(t[e], t[e + 1]), tp2)), X2);
+                            const float2 zz = make_float2(z[e], z[e + 1]), tt2 = make_float2(t[e], t[e + 1]);
+                            const float2 a = kFold ? fma2(zz, f2(c), f2(-Mz)) : mul2(sub2(zz, f2(mz)), f2(c));
+                            const float2 b = kFold ? fma2(tt2, f2(c), f2(-Mt)) : mul2(sub2(tt2, f2(mt)), f2(c));
+                            Ez2 = add2(Ez2, make_float2(ex2(a.x), ex2(a.y)));
+                            Et2 = add2(Et2, make_float2(ex2(b.x), ex2(b.y)));
                         }
-                        if constexpr (kNeedEt) {
+                    }
+                });
+        } else {
+        // ---- pass 0+1: this thread's running maxima and sums of 2^((x - m) c),
+        // rescaled whenever a chunk raises the maximum (JSD: clamped logits kept)
+        sweep_tm<In, kJsd, kJsd, true, false, kJsd>(tw, tsh, nv, tail, tz, tt,
+            [&](const float* z, const float* t, auto tag, int, float cz, float ct, bool, uint4&, uint4&) {
+                constexpr int kCnt = decltype(tag)::value;
+                if (cz > mz) {
+                    Ez2 = mul2(Ez2, f2(to_ref(mz, cz)));
+                    mz = cz;
+                }
+                if (ct > mt) {
+                    Et2 = mul2(Et2, f2(to_ref(mt, ct)));
+                    mt = ct;
+                }
+                const float Mz = __fmul_rn(mz, c), Mt = __fmul_rn(mt, c);
+                if constexpr (kCnt == 1) {
+                    if (mz != kNegInf) Ez2.x += kFold ? ex2(fmaf(z[0], c, -Mz)) : ex2((z[0] - mz) * c);
+                    if (mt != kNegInf) Et2.x += kFold ? ex2(fmaf(t[0], c, -Mt)) : ex2((t[0] - mt) * c);
+                } else {
+                    if (mz != kNegInf) {
 #pragma unroll
-                            for (int e = 0; e < kCnt; e += 2) {
-                                const float2 tt = make_float2(t[e], t[e + 1]);
-                                float2 a;
-                                if constexpr (kFold) a = fma2(tt, f2(c), nMt2);
-                                else a = mul2(sub2(tt, gt2), f2(c));
-                                const float2 et = make_float2(ex2(a.x), ex2(a.y));
-                                Et2 = add2(Et2, et);
-                                if (kKind == OSD_FKL) X2 = fma2(et, sub2(tt, make_float2(z[e], z[e + 1])), X2);
-                            }
+                        for (int e = 0; e < kCnt; e += 2) {
+                            const float2 zz = make_float2(z[e], z[e + 1]);
+                            const float2 a = kFold ? fma2(zz, f2(c), f2(-Mz)) : mul2(sub2(zz, f2(mz)), f2(c));
+                            Ez2 = add2(Ez2, make_float2(ex2(a.x), ex2(a.y)));
                         }
+                    }
+                    if (mt != kNegInf) {
+#pragma unroll
+                        for (int e = 0; e < kCnt; e += 2) {
+                            const float2 tt2 = make_float2(t[e], t[e + 1]);
+                            const float2 a = kFold ? fma2(tt2, f2(c), f2(-Mt)) : mul2(sub2(tt2, f2(mt)), f2(c));
+                            Et2 = add2(Et2, make_float2(ex2(a.x), ex2(a.y)));
+                        }
+                    }
+                }
+            });
+        }
+        {
+            const float wz = warp_max(mz), wt = warp_max(mt);
+            const float ez = warp_sum((Ez2.x + Ez2.y) * to_ref(mz, wz));
+            const float et = warp_sum((Et2.x + Et2.y) * to_ref(mt, wt));
+            const bool werr = __any_sync(0xffffffffu, !landed);
+            if (lane == 0) {
+                s_slot[warp] = make_float4(wz, werr ? -1.f : ez, wt, et);  // a negative sum flags a failed copy
+            }
+            if (warp != 0) named_arrive(1);
+        }
+        float gz, gt, cu, cv;
+        bool row_err;
+        if (warp == 0) {
+            named_sync(1);
+            float4 s = lane < kW ? s_slot[lane] : make_float4(kNegInf, 0.f, kNegInf, 0.f);
+            bool err = s.y < 0.f;
+            s.y = fmaxf(s.y, 0.f);
+            const float cz = warp_max(s.x), ct = warp_max(s.z);
+            float4 part = make_float4(cz, warp_sum(s.y * to_ref(s.x, cz)), ct, warp_sum(s.w * to_ref(s.z, ct)));
+            if (__any_sync(0xffffffffu, err)) part.y = -1.f;
+            float4 o = make_float4(kNegInf, 0.f, kNegInf, 0.f);
+            if (csize > 1) {
+                if (lane < csize)  // to slot `rank` of CTA `lane`
+                    st_async_v4(map_rank(&recv1[rank], lane), part, map_rank(&pbar1, lane));
+                if (lane == 0) mbar_arrive_expect_tx(&pbar1, static_cast<uint32_t>(csize) * 16u);
+                if (!mbar_wait_cluster_bounded(&pbar1, pph, kTmPartWaitNs)) {
+                    err = true;
+                    gave_up = true;
+                }
+                if (lane < csize) o = recv1[lane];
+            } else if (lane == 0) {
+                o = part;
+            }
+            err |= o.y < 0.f;
+            o.y = fmaxf(o.y, 0.f);
+            gz = warp_max(o.x);
+            gt = warp_max(o.z);
+            const float Ez = warp_sum(o.y * to_ref(o.x, gz)), Et = warp_sum(o.w * to_ref(o.z, gt));
+            float dz = 0.f, dt = 0.f;  // TVD: the rounding of m c in the terms' exponents
+            if (kFold) {
+                if (gz != kNegInf) dz = fmaf(gz, c, -__fmul_rn(gz, c));
+                if (gt != kNegInf) dt = fmaf(gt, c, -__fmul_rn(gt, c));
+            }
+            cu = -log2_sum(Et) + dt;
+            cv = -log2_sum(Ez) + dz;
+            row_err = __any_sync(0xffffffffu, err);
+            if (lane == 0) {
+                s_res = make_float4(gz, gt, cu, cv);
+                s_rerr = row_err;
+            }
+            named_arrive(2);
+        } else {
+            named_sync(2);
+            const float4 r = s_res;
+            gz = r.x;
+            gt = r.y;
+            cu = r.z;
+            cv = r.w;
+            row_err = s_rerr != 0;
+        }
+        if (row_err) {  // the row and the rest of the run report NaN
+            if (rank == 0 && tid == 0) {
+                p.loss[row] = __int_as_float(0x7fc00000);
+                if (p.status) atomicExch(p.status, static_cast<int32_t>(OSD_ERR_TIMEOUT));
+            }
+            stop = true;
+            continue;
+        }
+
+        // ---- pass 2: divergence terms with the global normalisers.  TVD: A = sum
+        // |q - p|, S = sum q' with q' = q sign(q - p) (kept in tensor memory in
+        // place of the chunk's logits) and Q = sum q; JSD: KL(p||m) and KL(q||m) in bits
+        float2 A2 = f2(0.f), B2 = f2(0.f), C2 = f2(0.f);
+        if (!jsd_trivial) {
+            sweep_tm<In, false, false, false, false, !kJsd>(tw, tsh, nv, tail, tz, tt,
+                [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4& zr, uint4& tr) {
+                    constexpr int kCnt = decltype(tag)::value;
+                    constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && !kJsd;
+                    const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw4[4] = {tr.x, tr.y, tr.z, tr.w};
+                    [[maybe_unused]] float qs[kCnt];
+#pragma unroll
+                    for (int e = 0; e < kCnt; e += 2) {
+                        const bool two = (e + 1 < kCnt);
+                        float2 u, v;
+                        if constexpr (kRaw) {
+                            u = fma2(bf16x2_minus(tw4[e / 2], gt), f2(c), f2(cu));
+                            v = fma2(bf16x2_minus(zw[e / 2], gz), f2(c), f2(cv));
+                        } else {
+                            u = fma2(sub2(make_float2(t[e], two ? t[e + 1] : t[e]), f2(gt)), f2(c), f2(cu));
+                            v = fma2(sub2(make_float2(z[e], two ? z[e + 1] : z[e]), f2(gz)), f2(c), f2(cv));
+                        }
+                        const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
+                        if constexpr (kJsd) {
+                            const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
+                            const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
+                            const float2 pw = two ? pj : make_float2(pj.x, 0.f);
+                            const float2 qw = two ? qj : make_float2(qj.x, 0.f);
+                            A2 = fma2(pw, sub2(u, lm), A2);
+                            B2 = fma2(qw, sub2(v, lm), B2);
+                        } else {
+                            const float2 df = sub2(qj, pj);
+                            const float2 qq = make_float2(copysignf(qj.x, df.x), copysignf(qj.y, df.y));
+                            qs[e] = qq.x;
+                            if (two) qs[e + 1] = qq.y;
+                            A2.x += fabsf(df.x);
+                            if (two) A2.y += fabsf(df.y);
+                            B2 = add2(B2, two ? qq : make_float2(qq.x, 0.f));
+                            C2 = add2(C2, two ? qj : make_float2(qj.x, 0.f));
+                        }
+                    }
+                    if constexpr (!kJsd) {
+                        if constexpr (kCnt == 1) tq = qs[0];
+                        else pack_q<In>(qs, zr, tr);  // written back to tensor memory by the sweep
                     }
                 });
         }
         {
-            const float3 bs = block_sum3<true, kT>(Ez2.x + Ez2.y, Et2.x + Et2.y, X2.x + X2.y, red_s);
-            const int any_ninf = kMoment ? __syncthreads_or(row_ninf ? 1 : 0) : 0;
-            const int any_inf = (kKind == OSD_RKL) ? __syncthreads_or(rkl_inf ? 1 : 0) : 0;
-            if (tid == 0)
-                s1_mine = Stats1{gzb, bs.x, (kKind == OSD_CE) ? bl.m : gtb, bs.y, bs.z,
-                                 err_local | (any_ninf << 1) | (any_inf << 2), bl.i,
-                                 (kKind == OSD_RKL) ? tpv : bl.z};
+            const float wa = warp_sum(A2.x + A2.y), wb = warp_sum(B2.x + B2.y);
+            const float wc = kJsd ? 0.f : warp_sum(C2.x + C2.y);
+            if (lane == 0) {
+                s_slot[warp] = make_float4(wa, wb, wc, 0.f);
+            }
+            if (warp != 0) named_arrive(1);
         }
-        if (csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
-        if (tid < 32) {
-            Stats1 o{kNegInf, 0.f, kNegInf, 0.f, 0.f, 0, INT_MAX, 0.f};
-            if (tid < csize) {
-                if (tid == rank) {
-                    o = s1_mine;
-                } else {
-                    const uint32_t base = map_rank(&s1_mine, tid);
-                    o.mz = ld_dsmem_f32(base + offsetof(Stats1, mz));
-                    o.Ez = ld_dsmem_f32(base + offsetof(Stats1, Ez));
-                    o.mt = ld_dsmem_f32(base + offsetof(Stats1, mt));
-                    o.Et = ld_dsmem_f32(base + offsetof(Stats1, Et));
-                    o.X = ld_dsmem_f32(base + offsetof(Stats1, X));
-                    o.err = ld_dsmem_s32(base + offsetof(Stats1, err));
-                    if (kKind == OSD_CE) o.idx = ld_dsmem_s32(base + offsetof(Stats1, idx));
-                    if (kKind == OSD_CE || kKind == OSD_RKL) o.zy = ld_dsmem_f32(base + offsetof(Stats1, zy));
+        float sa, sb, sc;
+        if (warp == 0) {
+            named_sync(1);
+            bool err = false;
+            const float4 s = lane < kW ? s_slot[lane] : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float4 part = make_float4(warp_sum(s.x), warp_sum(s.y), kJsd ? 0.f : warp_sum(s.z), 0.f);
+            float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (csize > 1) {
+                if (lane < csize) st_async_v4(map_rank(&recv2[rank], lane), part, map_rank(&pbar2, lane));
+                if (lane == 0) mbar_arrive_expect_tx(&pbar2, static_cast<uint32_t>(csize) * 16u);
+                if (!mbar_wait_cluster_bounded(&pbar2, pph, kTmPartWaitNs)) {
+                    err = true;
+                    gave_up = true;
                 }
+                if (lane < csize) o = recv2[lane];
+            } else if (lane == 0) {
+                o = part;
             }
-            Label L{o.mt, o.idx, o.zy};
-            if constexpr (kKind == OSD_CE) {
-                for (int off = 16; off > 0; off >>= 1) {
-                    const Label w{__shfl_xor_sync(0xffffffffu, L.m, off), __shfl_xor_sync(0xffffffffu, L.i, off),
-                                  __shfl_xor_sync(0xffffffffu, L.z, off)};
-                    L = merge_label(L, w);
-                }
+            sa = warp_sum(o.x);
+            sb = warp_sum(o.y);
+            sc = kJsd ? 0.f : warp_sum(o.z);
+            row_err = __any_sync(0xffffffffu, err);
+            if (lane == 0) {
+                s_res = make_float4(sa, sb, sc, 0.f);
+                s_rerr = row_err;
             }
-            float gz = o.mz, gt = o.mt;
-            int err = o.err;
-            for (int off = 16; off > 0; off >>= 1) {
-                gz = fmaxf(gz, __shfl_xor_sync(0xffffffffu, gz, off));
-                gt = fmaxf(gt, __shfl_xor_sync(0xffffffffu, gt, off));
-                err |= __shfl_xor_sync(0xffffffffu, err, off);
-            }
-            auto to_row = [c](float m, float g) {
-                if (m == kNegInf) return 0.f;
-                return kFold ? ex2(__fmul_rn(m, c) - __fmul_rn(g, c)) : ex2((m - g) * c);
-            };
-            const float sz = to_row(o.mz, gz), st = to_row(o.mt, gt);
-            float tg = 0.f;
-            if constexpr (kKind == OSD_RKL) {
-                tg = (o.mz == gz && o.mz != kNegInf) ? o.zy : kNegInf;
-                for (int off = 16; off > 0; off >>= 1) tg = fmaxf(tg, __shfl_xor_sync(0xffffffffu, tg, off));
-                if (tg == kNegInf) tg = 0.f;
-            }
-            float Ez = o.Ez * sz, Et = o.Et * st, X;
-            if constexpr (kKind == OSD_RKL)
-                X = (o.mz == kNegInf) ? 0.f : fmaf(o.Ez, (o.mz - gz) - (o.zy - tg), o.X) * sz;
-            else
-                X = o.X * st;
-            for (int off = 16; off > 0; off >>= 1) {
-                Ez += __shfl_xor_sync(0xffffffffu, Ez, off);
-                Et += __shfl_xor_sync(0xffffffffu, Et, off);
-                X += __shfl_xor_sync(0xffffffffu, X, off);
-            }
-            if (tid == 0) {
-                s1_all = Stats1{gz, Ez, gt, Et, X, err, L.i, L.z};
-                float dz = 0.f, dt = 0.f;
-                if (kFold) {
-                    if (gz != kNegInf) dz = fmaf(gz, c, -__fmul_rn(gz, c));
-                    if (gt != kNegInf) dt = fmaf(gt, c, -__fmul_rn(gt, c));
-                }
-                s_cu = -log2f(Et) + dt;
-                s_cv = -log2f(Ez) + dz;
-                const float lr = logf(Ez / Et) - kLn2 * (dz - dt);
-                float l = 0.f;
-                if (kKind == OSD_FKL) l = (X / Et - (gt - gz)) * inv_tau + lr;
-                if (kKind == OSD_RKL) l = (err & 4) ? __builtin_huge_valf() : (X / Ez + (gt - tg)) * inv_tau - lr;
-                if (kKind == OSD_CE) l = (gz - L.z) * inv_tau + (logf(Ez) - kLn2 * dz);
-                s_loss = l;
-                s_K = X / Ez * inv_tau;
-                s_tp = tg;
-            }
+            named_arrive(2);
+        } else {
+            named_sync(2);
+            const float4 r = s_res;
+            sa = r.x;
+            sb = r.y;
+            sc = r.z;
+            row_err = s_rerr != 0;
         }
-        __syncthreads();
-        const Stats1 st = s1_all;
-        const bool row_err = (st.err & 1) != 0;  // uniform over the cluster
-        const bool has_ninf = (st.err & 2) != 0;
-        const float cu = s_cu, cv = s_cv;
-        const float2 mt2 = f2(st.mt), mz2 = f2(st.mz);
-        auto log2p = [&](float2 x) { return fma2(sub2(x, mt2), f2(c), f2(cu)); };
-        auto log2q = [&](float2 x) { return fma2(sub2(x, mz2), f2(c), f2(cv)); };
-        float loss = s_loss;
-        const float beta = p.beta;
-        const bool jsd_trivial = (kKind == OSD_JSD) && (beta == 0.f || beta == 1.f);
-        Stats2 s2 = {0.f, 0.f, 0.f};
-        if constexpr (kKind == OSD_JSD || kKind == OSD_TVD) {
-            // ---- pass 2: divergence terms with the global normalisers
-            float2 A2 = f2(0.f), B2 = f2(0.f), C2 = f2(0.f);
-            if (!row_err && !jsd_trivial) {
-                sweep_tm<In, false, false, false, false, kKind == OSD_TVD>(tw, tsh, nv, tail, tz, tt,
-                    [&](const float* z, const float* t, auto tag, int j0, float, float, bool, uint4& zr, uint4& tr) {
-                        constexpr int kCnt = decltype(tag)::value;
-                        constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && kKind == OSD_TVD;
-                        const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw4[4] = {tr.x, tr.y, tr.z, tr.w};
-                        float qs[kCnt];
-#pragma unroll
-                        for (int e = 0; e < kCnt; e += 2) {
-                            const bool two = (e + 1 < kCnt);
-                            float2 u, v;
-                            if constexpr (kRaw) {
-                                u = fma2(bf16x2_minus(tw4[e / 2], st.mt), f2(c), f2(cu));
-                                v = fma2(bf16x2_minus(zw[e / 2], st.mz), f2(c), f2(cv));
-                            } else {
-                                u = log2p(make_float2(t[e], two ? t[e + 1] : t[e]));
-                                v = log2q(make_float2(z[e], two ? z[e + 1] : z[e]));
-                            }
-                            float2 a, b, c2 = f2(0.f);
-                            if (kKind == OSD_TVD) {
-                                const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
-                                const float2 df = sub2(qj, pj);
-                                a = make_float2(fabsf(df.x), fabsf(df.y));
-                                const float2 qq = make_float2(copysignf(qj.x, df.x), copysignf(qj.y, df.y));
-                                qs[e] = qq.x;
-                                if (e + 1 < kCnt) qs[e + 1] = qq.y;
-                                b = add2(qj, qq);
-                                c2 = sub2(qj, qq);
-                            } else {
-                                const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
-                                const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
-                                const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
-                                const float2 pw = two ? pj : make_float2(pj.x, 0.f);
-                                const float2 qw = two ? qj : make_float2(qj.x, 0.f);
-                                A2 = fma2(pw, sub2(u, lm), A2);
-                                B2 = fma2(qw, sub2(v, lm), B2);
-                                continue;
-                            }
-                            if (!two) { a.y = 0.f; b.y = 0.f; c2.y = 0.f; }
-                            A2 = add2(A2, a);
-                            B2 = add2(B2, b);
-                            C2 = add2(C2, c2);
-                        }
-                        if constexpr (kKind == OSD_TVD) {
-                            if constexpr (kCnt == 1) tq = qs[0];
-                            else pack_q<In>(qs, zr, tr);  // written back to tensor memory by the sweep
-                        }
-                    });
-            }
-            const float3 bs = block_sum3<true, kT>(A2.x + A2.y, B2.x + B2.y, C2.x + C2.y, red_s);
-            if (tid == 0) s2_mine = Stats2{bs.x, bs.y, bs.z};
-            if (csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
-            if (tid < 32) {
-                float a = 0.f, b = 0.f, cc = 0.f;
-                if (tid < csize) {
-                    if (tid == rank) {
-                        a = s2_mine.a;
-                        b = s2_mine.b;
-                        cc = s2_mine.c;
-                    } else {
-                        const uint32_t base = map_rank(&s2_mine, tid);
-                        a = ld_dsmem_f32(base + offsetof(Stats2, a));
-                        b = ld_dsmem_f32(base + offsetof(Stats2, b));
-                        if (kKind == OSD_TVD) cc = ld_dsmem_f32(base + offsetof(Stats2, c));
-                    }
-                }
-                for (int off = 16; off > 0; off >>= 1) {
-                    a += __shfl_xor_sync(0xffffffffu, a, off);
-                    b += __shfl_xor_sync(0xffffffffu, b, off);
-                    if (kKind == OSD_TVD) cc += __shfl_xor_sync(0xffffffffu, cc, off);
-                }
-                if (tid == 0) s2_all = Stats2{a, b, cc};
-            }
-            __syncthreads();
-            s2 = s2_all;
-            if (kKind == OSD_TVD) {
-                loss = 0.5f * s2.a;
-                s2.b *= 0.5f;
-                s2.c *= 0.5f;
-            } else {
-                loss = jsd_trivial ? 0.f : kLn2 * (beta * s2.a + (1.f - beta) * s2.b);
-            }
-        }
-        if (csize > 1) cluster_arrive_relaxed();  // finished reading the other CTAs' shared memory
 
         if (rank == 0 && tid == 0) {
+            const float loss = kJsd ? (jsd_trivial ? 0.f : kLn2 * (beta * sa + (1.f - beta) * sb)) : 0.5f * sa;
             p.loss[row] = row_err ? __int_as_float(0x7fc00000) : loss;
             if (row_err && p.status) atomicExch(p.status, static_cast<int32_t>(OSD_ERR_TIMEOUT));
         }
+        if (row_err) {
+            stop = true;
+            continue;
+        }
+        pph ^= 1u;
 
         // ---- pass 3: d loss / d draft logits of the span
         float* orow = p.dlogits + row * V + e0;
-        if (kKind == OSD_TVD && !row_err) {
-            const float gpos = s2.c * inv_tau, gneg = s2.b * inv_tau;
-            const uint32_t fpos = __float_as_uint(gpos), fdiff = fpos ^ __float_as_uint(gneg);
-            auto factor = [fpos, fdiff](float q) {
-                const uint32_t neg = static_cast<uint32_t>(__float_as_int(q) >> 31);
-                return __uint_as_float(fpos ^ (neg & fdiff));
-            };
+        if constexpr (!kJsd) {
+            // d TVD / d z = q (s Q - S) / (2 tau) with s = sign(q - p), S = sum q s
+            // and Q = sum q (1 up to rounding; summed, it cancels S exactly where
+            // every s is the same): k1 q' + k2 |q'| with k1 = Q / (2 tau), k2 = -S / (2 tau)
+            const float k1 = 0.5f * sc * inv_tau, k2 = -0.5f * sb * inv_tau;
             sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, 0, tz, tt,
                 [&](const float*, const float*, auto tag, int j0, float, float, bool, uint4& zr, uint4& tr) {
                     constexpr int kCnt = decltype(tag)::value;
@@ -1249,64 +1254,32 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
                         float q[kVec], gr[kVec];
                         unpack_q<In>(zr, tr, q);
 #pragma unroll
-                        for (int e = 0; e < kVec; e += 2) {
-                            const float2 r = mul2(make_float2(q[e], q[e + 1]), make_float2(factor(q[e]), factor(q[e + 1])));
-                            gr[e] = r.x;
-                            gr[e + 1] = r.y;
-                        }
+                        for (int e = 0; e < kVec; ++e) gr[e] = fmaf(k2, fabsf(q[e]), k1 * q[e]);
 #pragma unroll
                         for (int e = 0; e < kVec; e += 4) stg_v4(orow + j0 + e, gr[e], gr[e + 1], gr[e + 2], gr[e + 3]);
                     }
                 });
-            if (tid < tail) orow[tail0 + tid] = tq * (__float_as_int(tq) < 0 ? gneg : gpos);
-        } else if (kKind != OSD_TVD && !row_err) {
-            const float K = s_K, tpg = s_tp;
+            if (tid < tail) orow[tail0 + tid] = fmaf(k2, fabsf(tq), k1 * tq);
+        } else {
             const float2 cvs = f2(cv + p.lg_scale), cus = f2(cu + p.lg_scale);
-            const int label = st.idx;
             sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, tail, tz, tt,
-                [&](const float* z, const float* t, auto tag, int j0, float, float, bool, uint4& zr, uint4& tr) {
+                [&](const float* z, const float* t, auto tag, int j0, float, float, bool, uint4&, uint4&) {
                     constexpr int kCnt = decltype(tag)::value;
-                    constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && (kKind == OSD_FKL || kKind == OSD_RKL);
-                    const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw4[4] = {tr.x, tr.y, tr.z, tr.w};
-                    auto zdiff = [&](int e, float m) {
-                        if constexpr (kRaw) return bf16x2_minus(zw[e / 2], m);
-                        else return sub2(make_float2(z[e], (e + 1 < kCnt) ? z[e + 1] : z[e]), f2(m));
-                    };
-                    auto tdiff = [&](int e, float m) {
-                        if constexpr (kRaw) return bf16x2_minus(tw4[e / 2], m);
-                        else return sub2(make_float2(t[e], (e + 1 < kCnt) ? t[e + 1] : t[e]), f2(m));
-                    };
                     float gr[kCnt];
 #pragma unroll
                     for (int e = 0; e < kCnt; e += 2) {
                         const bool two = (e + 1 < kCnt);
-                        const float2 zd = zdiff(e, st.mz);
-                        const float2 v = fma2(zd, f2(c), cvs);
-                        const float2 qj = make_float2(ex2(v.x), ex2(v.y));
                         float2 gg;
-                        if (kKind == OSD_FKL) {
-                            const float2 u = fma2(tdiff(e, st.mt), f2(c), cus);
-                            gg = sub2(qj, make_float2(ex2(u.x), ex2(u.y)));
-                        } else if (kKind == OSD_CE) {
-                            const int j = e0 + j0 + e;
-                            gg = sub2(qj, make_float2(j == label ? inv_tau : 0.f, j + 1 == label ? inv_tau : 0.f));
-                        } else if (kKind == OSD_RKL) {
-                            const float2 dd = sub2(zd, tdiff(e, tpg));
-                            gg = mul2(qj, fma2(dd, f2(inv_tau), f2(-K)));
-                            if (has_ninf) {
-                                if (!(qj.x > 0.f)) gg.x = 0.f;
-                                if (!(qj.y > 0.f)) gg.y = 0.f;
-                            }
+                        if (jsd_trivial) {
+                            gg = f2(0.f);
                         } else {
-                            if (jsd_trivial) {
-                                gg = f2(0.f);
-                            } else {
-                                const float2 u = fma2(tdiff(e, st.mt), f2(c), cus);
-                                const float2 pj = make_float2(ex2(u.x), ex2(u.y));
-                                const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
-                                const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
-                                gg = mul2(qj, sub2(sub2(v, lm), f2(s2.b)));
-                            }
+                            const float2 v = fma2(sub2(make_float2(z[e], two ? z[e + 1] : z[e]), f2(gz)), f2(c), cvs);
+                            const float2 u = fma2(sub2(make_float2(t[e], two ? t[e + 1] : t[e]), f2(gt)), f2(c), cus);
+                            const float2 qj = make_float2(ex2(v.x), ex2(v.y));
+                            const float2 pj = make_float2(ex2(u.x), ex2(u.y));
+                            const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
+                            const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
+                            gg = mul2(qj, sub2(sub2(v, lm), f2(sb)));
                         }
                         gr[e] = gg.x;
                         if (two) gr[e + 1] = gg.y;
@@ -1320,12 +1293,19 @@ __global__ void __launch_bounds__(kTmThreads) distill_tm_kernel(DistParams p, Tm
                     }
                 });
         }
-        if (tid == 0) s_err = 0;  // read by every thread of the CTA before the barriers above
-        // the peers are done with this row's partials before the next row overwrites them
-        if (csize > 1) cluster_wait(); else __syncthreads();
-        if (row_err) stop = true;
     }
-    if (inflight && bytes) mbar_wait_bounded(&bar, infl_phase, kStageWaitNs);  // a copy still in flight lands first
+    if (tid == 0 && pending && bytes) mbar_wait_bounded(&bar, pend_phase, kStageWaitNs);  // a copy still in flight lands first
+    if (csize > 1) {
+        // every peer has made all its pushes (in the normal course this CTA has
+        // received them all); after a wait that gave up, the partial it waited
+        // for gets a short while longer to land before the CTA exits
+        cluster_arrive_relaxed();
+        cluster_wait();
+        if (gave_up) {
+            mbar_wait_cluster_bounded(&pbar1, pph, 10000000ull);
+            mbar_wait_cluster_bounded(&pbar2, pph, 10000000ull);
+        }
+    }
     tm_fence_before_sync();
     __syncthreads();
     tm_fence_after_sync();
@@ -1394,7 +1374,7 @@ struct TmLaunch {
     int occ;  // resident CTAs an SM
 };
 template <typename In, int kKind>
-static cudaError_t tm_launch_shape(int span, TmLaunch* out) {
+static cudaError_t tm_launch_shape(int span, int csize, TmLaunch* out) {
     constexpr int kVec = Elem<In>::kVec;
     const int nv = span / kVec;
     const int slots = (nv + kTmThreads - 1) / kTmThreads;
@@ -1404,7 +1384,7 @@ static cudaError_t tm_launch_shape(int span, TmLaunch* out) {
     if (ncols > 512) return cudaErrorInvalidValue;
     auto kern = distill_tm_kernel<In, kKind>;
     struct Entry {
-        int dev, span;
+        int dev, span, csize;
         size_t smem;
         int occ;
     };
@@ -1417,7 +1397,7 @@ static cudaError_t tm_launch_shape(int span, TmLaunch* out) {
     {
         std::lock_guard<std::mutex> lock(mu);
         for (int i = 0; i < n_cache; ++i)
-            if (cache[i].dev == dev && cache[i].span == span) {
+            if (cache[i].dev == dev && cache[i].span == span && cache[i].csize == csize) {
                 out->shape = TmShape{slots, t_off, ncols, 0, 0, 0, 0};
                 out->smem = cache[i].smem;
                 out->occ = cache[i].occ;
@@ -1433,7 +1413,8 @@ static cudaError_t tm_launch_shape(int span, TmLaunch* out) {
     e = cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
     if (e != cudaSuccess) return e;
     const size_t per_col = (size_t(smem_sm) + 511) / 512;
-    size_t smem = std::max(2 * size_t(span) * sizeof(In), size_t(ncols) * per_col);
+    // the staged span, then the two receive buffers of csize 16-byte partials
+    size_t smem = std::max(2 * size_t(span) * sizeof(In) + 2 * size_t(csize) * 16, size_t(ncols) * per_col);
     if (smem > size_t(kDistMaxSmem)) return cudaErrorInvalidValue;
     {
         // the opt-in only ever grows, so that a cached larger launch stays valid
@@ -1452,7 +1433,7 @@ static cudaError_t tm_launch_shape(int span, TmLaunch* out) {
     if (occ < 1 || occ * static_cast<int>(ncols) > 512) return cudaErrorInvalidValue;
     {
         std::lock_guard<std::mutex> lock(mu);
-        if (n_cache < 64) cache[n_cache++] = Entry{dev, span, smem, occ};
+        if (n_cache < 64) cache[n_cache++] = Entry{dev, span, csize, smem, occ};
     }
     out->shape = TmShape{slots, t_off, ncols, 0, 0, 0, 0};
     out->smem = smem;
@@ -1462,7 +1443,7 @@ static cudaError_t tm_launch_shape(int span, TmLaunch* out) {
 template <typename In, int kKind>
 static cudaError_t launch_distill_tm(const DistParams& dp, long long rows, cudaStream_t s) {
     TmLaunch tl;
-    const cudaError_t e = tm_launch_shape<In, kKind>(dp.span, &tl);
+    const cudaError_t e = tm_launch_shape<In, kKind>(dp.span, dp.csize, &tl);
     if (e != cudaSuccess) return e;
     // Longest runs first: the hardware hands out clusters in about index order, so
     // the last rows, in runs of 2 and then of 1, even out the clusters' finishing
@@ -1507,9 +1488,9 @@ static osd_status distill_run(const void* draft_logits, const void* target_logit
                          row_ok(d_stride_g, G) && row_ok(d_stride_p, p_rows) && row_ok(t_stride_g, G) &&
                          row_ok(t_stride_p, p_rows);
     // the TMEM-staged runs (if the span fits) for the kinds with a second pass, where
-    // they measured faster: TVD 72.5 % against 70.1 % of the HBM peak, JSD 68.0 %
+    // they measured faster: TVD 85.1 % against 70.1 % of the HBM peak, JSD 70.1 %
     // against 63.0 % (65536 x 32000 bf16); FKL, RKL and CE, near the bandwidth roof on
-    // the per-row kernel, measured 1-13 points slower on them
+    // the per-row kernel, measured 1-13 points slower on an earlier form of them
     const bool tm_path = aligned && !accepted && (kind == OSD_TVD || kind == OSD_JSD);
     int csize = 1, span = V;
     // JSD, with the most work per entry, stages best in longer spans on the per-row
