@@ -722,12 +722,12 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
 // clusters are resident), and masked-out rows of a run cost one mask read.
 // 16-byte-aligned rows; TVD and JSD, the kinds with a second pass over the
 // normalised distributions (FKL, RKL and CE measured slower on an earlier form of
-// these runs than on the per-row kernel).  A row costs two cluster barriers and
-// one CTA barrier: pass 0 and pass 1 fold into one sweep with running maxima, and
-// each warp publishes its own partials, which every warp then merges.
+// these runs than on the per-row kernel).  A row costs one CTA barrier (the
+// staging buffer is free) and two exchanges of partials within the cluster.
 constexpr int kTmThreads = 128;  // one warp per tensor-memory lane quarter
 constexpr int kTmG = 2;          // chunk slots per round of tensor-memory loads
 constexpr int kTmRows = 8;       // rows per cluster run
+constexpr int kTmJsdG = 1;       // JSD's passes 2 and 3: one chunk slot per round (no spills at 72 registers)
 constexpr int kTmMaxChunks = 4096;  // 16-byte chunks per span (<= 256 columns; longer spans stage as above)
 
 struct TmShape {
@@ -746,19 +746,25 @@ struct TmShape {
 // fewer than kVec entries, one per thread tid < tail, kept in that thread's
 // registers (tz, tt).  f is `sweep`'s callback, with the chunk's packed words by
 // reference: kStore writes them back.
-template <typename In, bool kClampZ, bool kClampT, bool kMax, bool kMin, bool kStore, typename F>
+template <typename In, bool kClampZ, bool kClampT, bool kMax, bool kMin, bool kStore, int kG = kTmG, typename F>
 __device__ __forceinline__ void sweep_tm(uint32_t tw, const TmShape& sh, int nv, int tail, float& tz, float& tt,
                                          F&& f) {
+    static_assert(kG == 1 || kG == kTmG, "one or kTmG chunk slots per round");
     using E = Elem<In>;
     constexpr int kVec = E::kVec;
     const int tid = threadIdx.x;
-    for (int s0 = 0; s0 < sh.slots; s0 += kTmG) {
-        uint4 zr[kTmG], tr[kTmG];
-        tm_ld8(tw + 4 * s0, zr[0], zr[1]);
-        tm_ld8(tw + sh.t_off + 4 * s0, tr[0], tr[1]);
+    for (int s0 = 0; s0 < sh.slots; s0 += kG) {
+        uint4 zr[kG], tr[kG];
+        if constexpr (kG == 1) {
+            tm_ld4(tw + 4 * s0, zr[0]);
+            tm_ld4(tw + sh.t_off + 4 * s0, tr[0]);
+        } else {
+            tm_ld8(tw + 4 * s0, zr[0], zr[1]);
+            tm_ld8(tw + sh.t_off + 4 * s0, tr[0], tr[1]);
+        }
         tm_wait_ld();
 #pragma unroll
-        for (int g = 0; g < kTmG; ++g) {
+        for (int g = 0; g < kG; ++g) {
             const int v = tid + kTmThreads * (s0 + g);
             if (v < nv) {
                 if (kClampZ) E::clamp_raw(zr[g]);
@@ -771,7 +777,10 @@ __device__ __forceinline__ void sweep_tm(uint32_t tw, const TmShape& sh, int nv,
                 f(z, t, std::integral_constant<int, kVec>{}, v * kVec, cz, ct, ninf, zr[g], tr[g]);
             }
         }
-        if constexpr (kStore) {
+        if constexpr (kStore && kG == 1) {
+            tm_st4(tw + 4 * s0, zr[0]);
+            tm_st4(tw + sh.t_off + 4 * s0, tr[0]);
+        } else if constexpr (kStore) {
             tm_st8(tw + 4 * s0, zr[0], zr[1]);
             tm_st8(tw + sh.t_off + 4 * s0, tr[0], tr[1]);
         }
@@ -849,7 +858,6 @@ __device__ __forceinline__ float log2_sum(float x) {
     const uint32_t b = __float_as_uint(x);
     return static_cast<float>(static_cast<int>(b >> 23) - 127) + lg2(__uint_as_float((b & 0x007fffffu) | 0x3f800000u));
 }
-constexpr bool kTmOnlineJsd = false;
 constexpr uint64_t kTmPartWaitNs = 3000000000ull;  // partials: peers may first wait out their copies
 // Named barriers 1 and 2 of the CTA (0 is __syncthreads): `arrive` marks the
 // warp's arrival without waiting (release), `sync` waits for all kTmThreads (acquire).
@@ -868,9 +876,6 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
     constexpr bool kJsd = kKind == OSD_JSD;
     // TVD: exponent arguments x c - m c as one fma; JSD: logits clamped to -1e30, (x - m) c
     constexpr bool kFold = !kJsd;
-    // pass 0 and pass 1 as one sweep with running maxima (TVD), or as two sweeps
-    // with the warp's maxima in between (JSD)
-    constexpr bool kOnline = kTmOnlineJsd || !kJsd;
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ __align__(8) uint64_t bar, pbar1, pbar2;
     __shared__ uint32_t s_taddr;
@@ -1003,79 +1008,39 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
 
         float mz = kNegInf, mt = kNegInf;
         float2 Ez2 = f2(0.f), Et2 = f2(0.f);
-        if constexpr (!kOnline) {
-            // ---- pass 0: this warp's maxima (JSD: clamped logits kept), then pass 1:
-            // sums of 2^((x - m) c) against them
-            sweep_tm<In, kJsd, kJsd, true, false, kJsd>(tw, tsh, nv, tail, tz, tt,
-                [&](const float*, const float*, auto, int, float cz, float ct, bool, uint4&, uint4&) {
-                    mz = fmaxf(mz, cz);
-                    mt = fmaxf(mt, ct);
-                });
-            mz = warp_max(mz);
-            mt = warp_max(mt);
-            const float Mz = __fmul_rn(mz, c), Mt = __fmul_rn(mt, c);
-            sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, tail, tz, tt,
-                [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4&, uint4&) {
-                    constexpr int kCnt = decltype(tag)::value;
-                    if constexpr (kCnt == 1) {
-                        if (mz != kNegInf) Ez2.x += kFold ? ex2(fmaf(z[0], c, -Mz)) : ex2((z[0] - mz) * c);
-                        if (mt != kNegInf) Et2.x += kFold ? ex2(fmaf(t[0], c, -Mt)) : ex2((t[0] - mt) * c);
-                    } else {
-#pragma unroll
-                        for (int e = 0; e < kCnt; e += 2) {
-                            const float2 zz = make_float2(z[e], z[e + 1]), tt2 = make_float2(t[e], t[e + 1]);
-                            const float2 a = kFold ? fma2(zz, f2(c), f2(-Mz)) : mul2(sub2(zz, f2(mz)), f2(c));
-                            const float2 b = kFold ? fma2(tt2, f2(c), f2(-Mt)) : mul2(sub2(tt2, f2(mt)), f2(c));
-                            Ez2 = add2(Ez2, make_float2(ex2(a.x), ex2(a.y)));
-                            Et2 = add2(Et2, make_float2(ex2(b.x), ex2(b.y)));
-                        }
-                    }
-                });
-        } else {
-        // ---- pass 0+1: this thread's running maxima and sums of 2^((x - m) c),
-        // rescaled whenever a chunk raises the maximum (JSD: clamped logits kept)
+        // ---- pass 0: this warp's maxima (JSD: clamped logits kept), then pass 1:
+        // sums of 2^((x - m) c) against them
         sweep_tm<In, kJsd, kJsd, true, false, kJsd>(tw, tsh, nv, tail, tz, tt,
-            [&](const float* z, const float* t, auto tag, int, float cz, float ct, bool, uint4&, uint4&) {
+            [&](const float*, const float*, auto, int, float cz, float ct, bool, uint4&, uint4&) {
+                mz = fmaxf(mz, cz);
+                mt = fmaxf(mt, ct);
+            });
+        mz = warp_max(mz);
+        mt = warp_max(mt);
+        // (TVD: a warp whose entries are all -inf takes m c = 0, and its terms 2^-inf = 0)
+        const float Mz = mz == kNegInf ? 0.f : __fmul_rn(mz, c), Mt = mt == kNegInf ? 0.f : __fmul_rn(mt, c);
+        sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, tail, tz, tt,
+            [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4&, uint4&) {
                 constexpr int kCnt = decltype(tag)::value;
-                if (cz > mz) {
-                    Ez2 = mul2(Ez2, f2(to_ref(mz, cz)));
-                    mz = cz;
-                }
-                if (ct > mt) {
-                    Et2 = mul2(Et2, f2(to_ref(mt, ct)));
-                    mt = ct;
-                }
-                const float Mz = __fmul_rn(mz, c), Mt = __fmul_rn(mt, c);
                 if constexpr (kCnt == 1) {
-                    if (mz != kNegInf) Ez2.x += kFold ? ex2(fmaf(z[0], c, -Mz)) : ex2((z[0] - mz) * c);
-                    if (mt != kNegInf) Et2.x += kFold ? ex2(fmaf(t[0], c, -Mt)) : ex2((t[0] - mt) * c);
+                    Ez2.x += kFold ? ex2(fmaf(z[0], c, -Mz)) : ex2((z[0] - mz) * c);
+                    Et2.x += kFold ? ex2(fmaf(t[0], c, -Mt)) : ex2((t[0] - mt) * c);
                 } else {
-                    if (mz != kNegInf) {
 #pragma unroll
-                        for (int e = 0; e < kCnt; e += 2) {
-                            const float2 zz = make_float2(z[e], z[e + 1]);
-                            const float2 a = kFold ? fma2(zz, f2(c), f2(-Mz)) : mul2(sub2(zz, f2(mz)), f2(c));
-                            Ez2 = add2(Ez2, make_float2(ex2(a.x), ex2(a.y)));
-                        }
-                    }
-                    if (mt != kNegInf) {
-#pragma unroll
-                        for (int e = 0; e < kCnt; e += 2) {
-                            const float2 tt2 = make_float2(t[e], t[e + 1]);
-                            const float2 a = kFold ? fma2(tt2, f2(c), f2(-Mt)) : mul2(sub2(tt2, f2(mt)), f2(c));
-                            Et2 = add2(Et2, make_float2(ex2(a.x), ex2(a.y)));
-                        }
+                    for (int e = 0; e < kCnt; e += 2) {
+                        const float2 zz = make_float2(z[e], z[e + 1]), tt2 = make_float2(t[e], t[e + 1]);
+                        const float2 a = kFold ? fma2(zz, f2(c), f2(-Mz)) : mul2(sub2(zz, f2(mz)), f2(c));
+                        const float2 b = kFold ? fma2(tt2, f2(c), f2(-Mt)) : mul2(sub2(tt2, f2(mt)), f2(c));
+                        Ez2 = add2(Ez2, make_float2(ex2(a.x), ex2(a.y)));
+                        Et2 = add2(Et2, make_float2(ex2(b.x), ex2(b.y)));
                     }
                 }
             });
-        }
         {
-            const float wz = warp_max(mz), wt = warp_max(mt);
-            const float ez = warp_sum((Ez2.x + Ez2.y) * to_ref(mz, wz));
-            const float et = warp_sum((Et2.x + Et2.y) * to_ref(mt, wt));
+            const float ez = warp_sum(Ez2.x + Ez2.y), et = warp_sum(Et2.x + Et2.y);
             const bool werr = __any_sync(0xffffffffu, !landed);
             if (lane == 0) {
-                s_slot[warp] = make_float4(wz, werr ? -1.f : ez, wt, et);  // a negative sum flags a failed copy
+                s_slot[warp] = make_float4(mz, werr ? -1.f : ez, mt, et);  // a negative sum flags a failed copy
             }
             if (warp != 0) named_arrive(1);
         }
@@ -1143,7 +1108,7 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
         // place of the chunk's logits) and Q = sum q; JSD: KL(p||m) and KL(q||m) in bits
         float2 A2 = f2(0.f), B2 = f2(0.f), C2 = f2(0.f);
         if (!jsd_trivial) {
-            sweep_tm<In, false, false, false, false, !kJsd>(tw, tsh, nv, tail, tz, tt,
+            sweep_tm<In, false, false, false, false, !kJsd, kJsd ? kTmJsdG : kTmG>(tw, tsh, nv, tail, tz, tt,
                 [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4& zr, uint4& tr) {
                     constexpr int kCnt = decltype(tag)::value;
                     constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && !kJsd;
@@ -1262,7 +1227,7 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
             if (tid < tail) orow[tail0 + tid] = fmaf(k2, fabsf(tq), k1 * tq);
         } else {
             const float2 cvs = f2(cv + p.lg_scale), cus = f2(cu + p.lg_scale);
-            sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, tail, tz, tt,
+            sweep_tm<In, false, false, false, false, false, kTmJsdG>(tw, tsh, nv, tail, tz, tt,
                 [&](const float* z, const float* t, auto tag, int j0, float, float, bool, uint4&, uint4&) {
                     constexpr int kCnt = decltype(tag)::value;
                     float gr[kCnt];
@@ -1488,7 +1453,7 @@ static osd_status distill_run(const void* draft_logits, const void* target_logit
                          row_ok(d_stride_g, G) && row_ok(d_stride_p, p_rows) && row_ok(t_stride_g, G) &&
                          row_ok(t_stride_p, p_rows);
     // the TMEM-staged runs (if the span fits) for the kinds with a second pass, where
-    // they measured faster: TVD 85.1 % against 70.1 % of the HBM peak, JSD 70.1 %
+    // they measured faster: TVD 94.6 % against 70.1 % of the HBM peak, JSD 71.3 %
     // against 63.0 % (65536 x 32000 bf16); FKL, RKL and CE, near the bandwidth roof on
     // the per-row kernel, measured 1-13 points slower on an earlier form of them
     const bool tm_path = aligned && !accepted && (kind == OSD_TVD || kind == OSD_JSD);
