@@ -720,14 +720,17 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
 // of row i, with the shared-memory footprint of one staged span per CTA.  The
 // hardware schedules the runs like any grid (no assumption on how many
 // clusters are resident), and masked-out rows of a run cost one mask read.
-// 16-byte-aligned rows; TVD and JSD, the kinds with a second pass over the
-// normalised distributions (FKL, RKL and CE measured slower on an earlier form of
-// these runs than on the per-row kernel).  A row costs one CTA barrier (the
-// staging buffer is free) and two exchanges of partials within the cluster.
+// 16-byte-aligned rows; TVD, JSD and RKL (FKL and CE measured slower on an
+// earlier form of these runs than on the per-row kernel).  A row costs one CTA
+// barrier (the staging buffer is free) and two exchanges within the cluster:
+// TVD and JSD exchange the normalisers, then the sums of pass 2; RKL the maxima
+// with its pivot, then the sums and its moment.
 constexpr int kTmThreads = 128;  // one warp per tensor-memory lane quarter
 constexpr int kTmG = 2;          // chunk slots per round of tensor-memory loads
 constexpr int kTmRows = 8;       // rows per cluster run
 constexpr int kTmJsdG = 1;       // JSD's passes 2 and 3: one chunk slot per round (no spills at 72 registers)
+constexpr bool kTmRkl = true;     // RKL on these runs too
+constexpr int kTmRklG = 1;       // RKL pass 1: one chunk slot per round (no spills at 72 registers)
 constexpr int kTmMaxChunks = 4096;  // 16-byte chunks per span (<= 256 columns; longer spans stage as above)
 
 struct TmShape {
@@ -830,17 +833,17 @@ __device__ __forceinline__ void unpack_q(const uint4& zr, const uint4& tr, float
     }
 }
 
-// A row's statistics travel without cluster barriers: each warp reduces its
-// partial and leaves it in a slot of its CTA (arriving on named barrier 1, where
-// warp 0 waits); warp 0 merges the slots into the CTA's partial and pushes it
-// with st.async into slot `rank` of every CTA's receive buffer, where it
-// completes 16 bytes on that CTA's barrier for the pass; warp 0 of each CTA then
-// merges the csize partials, in rank order, and hands the result to the other
-// warps through named barrier 2 (they wait, it arrives).  Every
-// CTA sees the same partials in the same order, so all reach the same bits.  The
-// two passes use two receive buffers and barriers: a CTA pushes its next partial
-// for a pass only after every CTA's partial of the pass in between has reached
-// it, and that one comes from each peer only once the peer has read the buffer.
+// A row's statistics travel without cluster barriers.  In an exchange each warp
+// leaves its value (the same in all its lanes) in a slot of its CTA and arrives
+// on named barrier 1, where warp 0 waits; warp 0 merges the slots into the CTA's
+// partial and pushes it with st.async into slot `rank` of every CTA's receive
+// buffer for that exchange, completing 16 bytes on that CTA's barrier; it then
+// merges the csize partials, in rank order, writes the result for the other
+// warps and arrives on named barrier 2, where they wait.  Every CTA merges the
+// same partials in the same order, so all reach the same bits.  A row makes two
+// exchanges, each with its own receive buffer and barrier: a CTA pushes its
+// next partial of an exchange only after every CTA's partial of the other one
+// has reached it, which each peer sends only once it has read the buffer.
 __device__ __forceinline__ float warp_max(float x) {
     for (int off = 16; off > 0; off >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, off));
     return x;
@@ -850,11 +853,27 @@ __device__ __forceinline__ float warp_sum(float x) {
     for (int off = 16; off > 0; off >>= 1) x += __shfl_xor_sync(0xffffffffu, x, off);
     return x;
 }
+__device__ __forceinline__ int warp_or(int x) {
+    for (int off = 16; off > 0; off >>= 1) x |= __shfl_xor_sync(0xffffffffu, x, off);
+    return x;
+}
+// RKL: the draft maximum with the target logit at it (the larger one on ties) in
+// .x/.y of every lane
+__device__ __forceinline__ float2 warp_max_pivot(float m, float t) {
+    for (int off = 16; off > 0; off >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, m, off), t2 = __shfl_xor_sync(0xffffffffu, t, off);
+        if (pivot_wins(m2, t2, m, t)) {
+            m = m2;
+            t = t2;
+        }
+    }
+    return make_float2(m, t);
+}
 // log2 of a sum of exponentials that is at least 1 (the term of the maximum):
 // the exponent plus lg2.approx of the mantissa in [1, 2), absolute error about
-// 2^-22 there; anything else (0, inf, NaN) through log2f
+// 2^-22 there; anything else (0 of a row with no mass, inf, NaN) straight through lg2.approx
 __device__ __forceinline__ float log2_sum(float x) {
-    if (!(x >= 1.f && x <= 3.0e38f)) return log2f(x);
+    if (!(x >= 1.f && x <= 3.0e38f)) return lg2(x);
     const uint32_t b = __float_as_uint(x);
     return static_cast<float>(static_cast<int>(b >> 23) - 127) + lg2(__uint_as_float((b & 0x007fffffu) | 0x3f800000u));
 }
@@ -867,21 +886,25 @@ __device__ __forceinline__ void named_arrive(int id) {
 __device__ __forceinline__ void named_sync(int id) {
     asm volatile("bar.sync %0, %1;" :: "r"(id), "n"(kTmThreads) : "memory");
 }
+// The flags of an RKL row, OR-ed over the cluster in the .w of its second exchange.
+constexpr int kTmNinf = 1;    // some logit is -inf
+constexpr int kTmRklInf = 2;  // a finite draft logit meets a -inf target logit: the loss is +inf
 
 template <typename In, int kKind>
 __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p, TmShape tsh) {
-    static_assert(kKind == OSD_TVD || kKind == OSD_JSD, "the TMEM-staged runs serve TVD and JSD");
+    static_assert(kKind == OSD_TVD || kKind == OSD_JSD || kKind == OSD_RKL,
+                  "the TMEM-staged runs serve TVD, JSD and RKL");
     constexpr int kT = kTmThreads, kW = kT / 32;
     constexpr int kVec = Elem<In>::kVec;
-    constexpr bool kJsd = kKind == OSD_JSD;
-    // TVD: exponent arguments x c - m c as one fma; JSD: logits clamped to -1e30, (x - m) c
+    constexpr bool kJsd = kKind == OSD_JSD, kTvd = kKind == OSD_TVD, kRkl = kKind == OSD_RKL;
+    // TVD, RKL: exponent arguments x c - m c as one fma; JSD: logits clamped to -1e30, (x - m) c
     constexpr bool kFold = !kJsd;
     extern __shared__ __align__(128) unsigned char dsm[];
     __shared__ __align__(8) uint64_t bar, pbar1, pbar2;
     __shared__ uint32_t s_taddr;
-    __shared__ float4 s_slot[kW];  // the warps' partials of the pass in progress
-    __shared__ float4 s_res;       // warp 0's merged result of the pass in progress ...
-    __shared__ int s_rerr;         // ... and whether the row failed
+    __shared__ float4 s_slot[kW];  // the warps' values of the exchange in progress
+    __shared__ float4 s_res;       // its merged result ...
+    __shared__ int s_rerr;         // ... and whether a wait for it gave up
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int csize = p.csize;
@@ -896,8 +919,8 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
     const uint32_t bytes = static_cast<uint32_t>(tail0 * sizeof(In));
     In* zs = reinterpret_cast<In*>(dsm);
     In* ts = zs + p.span;
-    float4* recv1 = reinterpret_cast<float4*>(ts + p.span);  // [csize] CTA partials of pass 0+1
-    float4* recv2 = recv1 + csize;                          // [csize] CTA partials of pass 2
+    float4* recv1 = reinterpret_cast<float4*>(ts + p.span);  // [csize] CTA partials of the first exchange
+    float4* recv2 = recv1 + csize;                          // [csize] CTA partials of the second
 
     // tensor memory for this CTA (the launch keeps resident CTAs x columns <= 512,
     // so the allocation never waits), and the barriers
@@ -917,6 +940,50 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
     }
     tm_fence_after_sync();
     const uint32_t tw = s_taddr + (static_cast<uint32_t>(32 * warp) << 16);
+
+    uint32_t pph = 0;      // pbar1 and pbar2: one phase per row
+    bool gave_up = false;  // warp 0: a wait for the peers' partials ran out
+    // One exchange: v is this warp's value, merge(x) reduces x over the lanes of
+    // warp 0 (lanes past the valid ones hold `ident`) into the same value in
+    // every lane, and warp 0 turns the cluster's merge m into the row's values
+    // with finish(m, bad) (bad: the row failed); returns them in every thread,
+    // `failed` set where a wait gave up or finish found the row bad.
+    auto exchange = [&](float4 v, float4 ident, uint64_t* pbar, float4* recv, auto&& merge, auto&& finish,
+                        bool& failed) {
+        if (lane == 0) s_slot[warp] = v;
+        if (warp != 0) {
+            named_arrive(1);
+            named_sync(2);
+            failed = s_rerr != 0;
+            return s_res;
+        }
+        named_sync(1);
+        const float4 part = merge(lane < kW ? s_slot[lane] : ident);
+        float4 o = ident;
+        bool err = false;
+        if (csize > 1) {
+            if (lane < csize)  // into slot `rank` of CTA `lane`
+                st_async_v4(map_rank(&recv[rank], static_cast<uint32_t>(lane)), part,
+                            map_rank(pbar, static_cast<uint32_t>(lane)));
+            if (lane == 0) mbar_arrive_expect_tx(pbar, static_cast<uint32_t>(csize) * 16u);
+            if (!mbar_wait_cluster_bounded(pbar, pph, kTmPartWaitNs)) {
+                err = true;
+                gave_up = true;
+            }
+            if (lane < csize) o = recv[lane];
+        } else if (lane == 0) {
+            o = part;
+        }
+        bool bad = false;
+        const float4 r = finish(merge(o), bad);
+        failed = __any_sync(0xffffffffu, err) || bad;
+        if (lane == 0) {
+            s_res = r;
+            s_rerr = failed;
+        }
+        named_arrive(2);
+        return r;
+    };
 
     float nz = 0.f, nt = 0.f;  // the ragged tail entry (tid < tail) of the row in flight ...
     float tz = 0.f, tt = 0.f, tq = 0.f;  // ... and of this row (TVD: tq = q sign(q - p) there)
@@ -965,11 +1032,11 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
         if (m == kNegInf) return 0.f;
         return kFold ? ex2(__fmul_rn(m, c) - __fmul_rn(g, c)) : ex2((m - g) * c);
     };
+    // the exact part of m c that rn(m c) drops (TVD, RKL: the terms' exponents carry it)
+    auto fold_err = [c](float m) { return (kFold && m != kNegInf) ? fmaf(m, c, -__fmul_rn(m, c)) : 0.f; };
     const float beta = p.beta;
     const bool jsd_trivial = kJsd && (beta == 0.f || beta == 1.f);
     uint32_t phase = 0;  // the staging barrier's phase for this row
-    uint32_t pph = 0;    // pbar1 and pbar2: one phase per row
-    bool gave_up = false;  // warp 0: a wait for the peers' partials ran out
     bool stop = false;
     for (long long next; row < r1; row = next, phase ^= 1u) {
         next = row + 1;
@@ -1005,201 +1072,249 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                 pend_phase = phase ^ 1u;
             }
         }
+        const bool werr = __any_sync(0xffffffffu, !landed);
 
-        float mz = kNegInf, mt = kNegInf;
-        float2 Ez2 = f2(0.f), Et2 = f2(0.f);
-        // ---- pass 0: this warp's maxima (JSD: clamped logits kept), then pass 1:
-        // sums of 2^((x - m) c) against them
+        // ---- pass 0: this warp's maxima (JSD: clamped logits kept; RKL: with the
+        // target logit at the draft maximum)
+        float mz = kNegInf, mt = kNegInf, tp = kNegInf;
         sweep_tm<In, kJsd, kJsd, true, false, kJsd>(tw, tsh, nv, tail, tz, tt,
-            [&](const float*, const float*, auto, int, float cz, float ct, bool, uint4&, uint4&) {
-                mz = fmaxf(mz, cz);
+            [&](const float* z, const float* t, auto tag, int, float cz, float ct, bool, uint4&, uint4&) {
+                if constexpr (kRkl) {
+                    constexpr int kCnt = decltype(tag)::value;
+                    if (cz > mz) {
+                        mz = cz;
+#pragma unroll
+                        for (int e = kCnt - 1; e >= 0; --e)
+                            if (z[e] == cz) tp = t[e];
+                    }
+                } else {
+                    mz = fmaxf(mz, cz);
+                }
                 mt = fmaxf(mt, ct);
             });
-        mz = warp_max(mz);
-        mt = warp_max(mt);
-        // (TVD: a warp whose entries are all -inf takes m c = 0, and its terms 2^-inf = 0)
-        const float Mz = mz == kNegInf ? 0.f : __fmul_rn(mz, c), Mt = mt == kNegInf ? 0.f : __fmul_rn(mt, c);
-        sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, tail, tz, tt,
-            [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4&, uint4&) {
-                constexpr int kCnt = decltype(tag)::value;
-                if constexpr (kCnt == 1) {
-                    Ez2.x += kFold ? ex2(fmaf(z[0], c, -Mz)) : ex2((z[0] - mz) * c);
-                    Et2.x += kFold ? ex2(fmaf(t[0], c, -Mt)) : ex2((t[0] - mt) * c);
-                } else {
-#pragma unroll
-                    for (int e = 0; e < kCnt; e += 2) {
-                        const float2 zz = make_float2(z[e], z[e + 1]), tt2 = make_float2(t[e], t[e + 1]);
-                        const float2 a = kFold ? fma2(zz, f2(c), f2(-Mz)) : mul2(sub2(zz, f2(mz)), f2(c));
-                        const float2 b = kFold ? fma2(tt2, f2(c), f2(-Mt)) : mul2(sub2(tt2, f2(mt)), f2(c));
-                        Ez2 = add2(Ez2, make_float2(ex2(a.x), ex2(a.y)));
-                        Et2 = add2(Et2, make_float2(ex2(b.x), ex2(b.y)));
-                    }
-                }
-            });
-        {
-            const float ez = warp_sum(Ez2.x + Ez2.y), et = warp_sum(Et2.x + Et2.y);
-            const bool werr = __any_sync(0xffffffffu, !landed);
-            if (lane == 0) {
-                s_slot[warp] = make_float4(mz, werr ? -1.f : ez, mt, et);  // a negative sum flags a failed copy
-            }
-            if (warp != 0) named_arrive(1);
-        }
-        float gz, gt, cu, cv;
-        bool row_err;
-        if (warp == 0) {
-            named_sync(1);
-            float4 s = lane < kW ? s_slot[lane] : make_float4(kNegInf, 0.f, kNegInf, 0.f);
-            bool err = s.y < 0.f;
-            s.y = fmaxf(s.y, 0.f);
-            const float cz = warp_max(s.x), ct = warp_max(s.z);
-            float4 part = make_float4(cz, warp_sum(s.y * to_ref(s.x, cz)), ct, warp_sum(s.w * to_ref(s.z, ct)));
-            if (__any_sync(0xffffffffu, err)) part.y = -1.f;
-            float4 o = make_float4(kNegInf, 0.f, kNegInf, 0.f);
-            if (csize > 1) {
-                if (lane < csize)  // to slot `rank` of CTA `lane`
-                    st_async_v4(map_rank(&recv1[rank], lane), part, map_rank(&pbar1, lane));
-                if (lane == 0) mbar_arrive_expect_tx(&pbar1, static_cast<uint32_t>(csize) * 16u);
-                if (!mbar_wait_cluster_bounded(&pbar1, pph, kTmPartWaitNs)) {
-                    err = true;
-                    gave_up = true;
-                }
-                if (lane < csize) o = recv1[lane];
-            } else if (lane == 0) {
-                o = part;
-            }
-            err |= o.y < 0.f;
-            o.y = fmaxf(o.y, 0.f);
-            gz = warp_max(o.x);
-            gt = warp_max(o.z);
-            const float Ez = warp_sum(o.y * to_ref(o.x, gz)), Et = warp_sum(o.w * to_ref(o.z, gt));
-            float dz = 0.f, dt = 0.f;  // TVD: the rounding of m c in the terms' exponents
-            if (kFold) {
-                if (gz != kNegInf) dz = fmaf(gz, c, -__fmul_rn(gz, c));
-                if (gt != kNegInf) dt = fmaf(gt, c, -__fmul_rn(gt, c));
-            }
-            cu = -log2_sum(Et) + dt;
-            cv = -log2_sum(Ez) + dz;
-            row_err = __any_sync(0xffffffffu, err);
-            if (lane == 0) {
-                s_res = make_float4(gz, gt, cu, cv);
-                s_rerr = row_err;
-            }
-            named_arrive(2);
+        if constexpr (kRkl) {
+            const float2 pv = warp_max_pivot(mz, tp);
+            mz = pv.x;
+            tp = pv.y;
         } else {
-            named_sync(2);
-            const float4 r = s_res;
-            gz = r.x;
-            gt = r.y;
-            cu = r.z;
-            cv = r.w;
-            row_err = s_rerr != 0;
+            mz = warp_max(mz);
         }
-        if (row_err) {  // the row and the rest of the run report NaN
-            if (rank == 0 && tid == 0) {
-                p.loss[row] = __int_as_float(0x7fc00000);
-                if (p.status) atomicExch(p.status, static_cast<int32_t>(OSD_ERR_TIMEOUT));
-            }
-            stop = true;
-            continue;
-        }
+        mt = warp_max(mt);
 
-        // ---- pass 2: divergence terms with the global normalisers.  TVD: A = sum
-        // |q - p|, S = sum q' with q' = q sign(q - p) (kept in tensor memory in
-        // place of the chunk's logits) and Q = sum q; JSD: KL(p||m) and KL(q||m) in bits
-        float2 A2 = f2(0.f), B2 = f2(0.f), C2 = f2(0.f);
-        if (!jsd_trivial) {
-            sweep_tm<In, false, false, false, false, !kJsd, kJsd ? kTmJsdG : kTmG>(tw, tsh, nv, tail, tz, tt,
-                [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4& zr, uint4& tr) {
+        float gz, gt, cu = 0.f, cv;  // the row's maxima, and log2 p = (t - gt) c + cu, log2 q = (z - gz) c + cv
+        float K = 0.f;         // RKL: sum_j q_j ((z_j - gz) - (t_j - tp)) / tau
+        int flags = 0;         // RKL: kTmNinf | kTmRklInf over the row
+        float sa = 0.f, sb = 0.f;  // TVD: k1, k2 of the gradient; JSD: S = sum q log2(q/m) (in sa)
+        bool row_err;
+        float loss = 0.f;
+        if constexpr (!kRkl) {
+            // ---- pass 1: sums of 2^((x - m) c) against the warp's maxima (TVD: a warp
+            // whose entries are all -inf takes m c = 0, and its terms 2^-inf = 0)
+            float2 Ez2 = f2(0.f), Et2 = f2(0.f);
+            const float Mz = mz == kNegInf ? 0.f : __fmul_rn(mz, c), Mt = mt == kNegInf ? 0.f : __fmul_rn(mt, c);
+            sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, tail, tz, tt,
+                [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4&, uint4&) {
                     constexpr int kCnt = decltype(tag)::value;
-                    constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && !kJsd;
-                    const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw4[4] = {tr.x, tr.y, tr.z, tr.w};
-                    [[maybe_unused]] float qs[kCnt];
+                    if constexpr (kCnt == 1) {
+                        Ez2.x += kFold ? ex2(fmaf(z[0], c, -Mz)) : ex2((z[0] - mz) * c);
+                        Et2.x += kFold ? ex2(fmaf(t[0], c, -Mt)) : ex2((t[0] - mt) * c);
+                    } else {
 #pragma unroll
-                    for (int e = 0; e < kCnt; e += 2) {
-                        const bool two = (e + 1 < kCnt);
-                        float2 u, v;
-                        if constexpr (kRaw) {
-                            u = fma2(bf16x2_minus(tw4[e / 2], gt), f2(c), f2(cu));
-                            v = fma2(bf16x2_minus(zw[e / 2], gz), f2(c), f2(cv));
-                        } else {
-                            u = fma2(sub2(make_float2(t[e], two ? t[e + 1] : t[e]), f2(gt)), f2(c), f2(cu));
-                            v = fma2(sub2(make_float2(z[e], two ? z[e + 1] : z[e]), f2(gz)), f2(c), f2(cv));
+                        for (int e = 0; e < kCnt; e += 2) {
+                            const float2 zz = make_float2(z[e], z[e + 1]), tt2 = make_float2(t[e], t[e + 1]);
+                            const float2 a = kFold ? fma2(zz, f2(c), f2(-Mz)) : mul2(sub2(zz, f2(mz)), f2(c));
+                            const float2 b = kFold ? fma2(tt2, f2(c), f2(-Mt)) : mul2(sub2(tt2, f2(mt)), f2(c));
+                            Ez2 = add2(Ez2, make_float2(ex2(a.x), ex2(a.y)));
+                            Et2 = add2(Et2, make_float2(ex2(b.x), ex2(b.y)));
                         }
-                        const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
-                        if constexpr (kJsd) {
-                            const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
-                            const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
-                            const float2 pw = two ? pj : make_float2(pj.x, 0.f);
-                            const float2 qw = two ? qj : make_float2(qj.x, 0.f);
-                            A2 = fma2(pw, sub2(u, lm), A2);
-                            B2 = fma2(qw, sub2(v, lm), B2);
-                        } else {
-                            const float2 df = sub2(qj, pj);
-                            const float2 qq = make_float2(copysignf(qj.x, df.x), copysignf(qj.y, df.y));
-                            qs[e] = qq.x;
-                            if (two) qs[e + 1] = qq.y;
-                            A2.x += fabsf(df.x);
-                            if (two) A2.y += fabsf(df.y);
-                            B2 = add2(B2, two ? qq : make_float2(qq.x, 0.f));
-                            C2 = add2(C2, two ? qj : make_float2(qj.x, 0.f));
-                        }
-                    }
-                    if constexpr (!kJsd) {
-                        if constexpr (kCnt == 1) tq = qs[0];
-                        else pack_q<In>(qs, zr, tr);  // written back to tensor memory by the sweep
                     }
                 });
-        }
-        {
-            const float wa = warp_sum(A2.x + A2.y), wb = warp_sum(B2.x + B2.y);
-            const float wc = kJsd ? 0.f : warp_sum(C2.x + C2.y);
-            if (lane == 0) {
-                s_slot[warp] = make_float4(wa, wb, wc, 0.f);
-            }
-            if (warp != 0) named_arrive(1);
-        }
-        float sa, sb, sc;
-        if (warp == 0) {
-            named_sync(1);
-            bool err = false;
-            const float4 s = lane < kW ? s_slot[lane] : make_float4(0.f, 0.f, 0.f, 0.f);
-            const float4 part = make_float4(warp_sum(s.x), warp_sum(s.y), kJsd ? 0.f : warp_sum(s.z), 0.f);
-            float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (csize > 1) {
-                if (lane < csize) st_async_v4(map_rank(&recv2[rank], lane), part, map_rank(&pbar2, lane));
-                if (lane == 0) mbar_arrive_expect_tx(&pbar2, static_cast<uint32_t>(csize) * 16u);
-                if (!mbar_wait_cluster_bounded(&pbar2, pph, kTmPartWaitNs)) {
-                    err = true;
-                    gave_up = true;
+            // ---- exchange 1: the row's maxima and normalisers (a negative sum flags a failed copy)
+            const float4 v1 = make_float4(mz, werr ? -1.f : warp_sum(Ez2.x + Ez2.y), mt, warp_sum(Et2.x + Et2.y));
+            bool failed = false;
+            const float4 r1v = exchange(v1, make_float4(kNegInf, 0.f, kNegInf, 0.f), &pbar1, recv1,
+                [&](float4 x) {
+                    const bool e = __any_sync(0xffffffffu, x.y < 0.f);
+                    x.y = fmaxf(x.y, 0.f);
+                    const float g1 = warp_max(x.x), g2 = warp_max(x.z);
+                    const float s1 = warp_sum(x.y * to_ref(x.x, g1)), s2 = warp_sum(x.w * to_ref(x.z, g2));
+                    return make_float4(g1, e ? -1.f : s1, g2, s2);
+                },
+                [&](float4 m, bool& bad) {  // -> (gz, gt, cu, cv)
+                    bad = m.y < 0.f;
+                    return make_float4(m.x, m.z, -log2_sum(m.w) + fold_err(m.z), -log2_sum(m.y) + fold_err(m.x));
+                }, failed);
+            row_err = failed;
+            gz = r1v.x;
+            gt = r1v.y;
+            cu = r1v.z;
+            cv = r1v.w;
+            if (row_err) {  // the row and the rest of the run report NaN
+                if (rank == 0 && tid == 0) {
+                    p.loss[row] = __int_as_float(0x7fc00000);
+                    if (p.status) atomicExch(p.status, static_cast<int32_t>(OSD_ERR_TIMEOUT));
                 }
-                if (lane < csize) o = recv2[lane];
-            } else if (lane == 0) {
-                o = part;
+                stop = true;
+                continue;
             }
-            sa = warp_sum(o.x);
-            sb = warp_sum(o.y);
-            sc = kJsd ? 0.f : warp_sum(o.z);
-            row_err = __any_sync(0xffffffffu, err);
-            if (lane == 0) {
-                s_res = make_float4(sa, sb, sc, 0.f);
-                s_rerr = row_err;
+            {
+                // ---- pass 2: divergence terms with the global normalisers.  TVD: A = sum
+                // |q - p|, S = sum q' with q' = q sign(q - p) (kept in tensor memory in
+                // place of the chunk's logits) and Q = sum q; JSD: KL(p||m) and KL(q||m) in bits
+                float2 A2 = f2(0.f), B2 = f2(0.f), C2 = f2(0.f);
+                if (!jsd_trivial) {
+                    sweep_tm<In, false, false, false, false, kTvd, kJsd ? kTmJsdG : kTmG>(tw, tsh, nv, tail, tz, tt,
+                        [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4& zr, uint4& tr) {
+                            constexpr int kCnt = decltype(tag)::value;
+                            constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && kTvd;
+                            const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw4[4] = {tr.x, tr.y, tr.z, tr.w};
+                            [[maybe_unused]] float qs[kCnt];
+#pragma unroll
+                            for (int e = 0; e < kCnt; e += 2) {
+                                const bool two = (e + 1 < kCnt);
+                                float2 u, v;
+                                if constexpr (kRaw) {
+                                    u = fma2(bf16x2_minus(tw4[e / 2], gt), f2(c), f2(cu));
+                                    v = fma2(bf16x2_minus(zw[e / 2], gz), f2(c), f2(cv));
+                                } else {
+                                    u = fma2(sub2(make_float2(t[e], two ? t[e + 1] : t[e]), f2(gt)), f2(c), f2(cu));
+                                    v = fma2(sub2(make_float2(z[e], two ? z[e + 1] : z[e]), f2(gz)), f2(c), f2(cv));
+                                }
+                                const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
+                                if constexpr (kJsd) {
+                                    const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
+                                    const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
+                                    const float2 pw = two ? pj : make_float2(pj.x, 0.f);
+                                    const float2 qw = two ? qj : make_float2(qj.x, 0.f);
+                                    A2 = fma2(pw, sub2(u, lm), A2);
+                                    B2 = fma2(qw, sub2(v, lm), B2);
+                                } else {
+                                    const float2 df = sub2(qj, pj);
+                                    const float2 qq = make_float2(copysignf(qj.x, df.x), copysignf(qj.y, df.y));
+                                    qs[e] = qq.x;
+                                    if (two) qs[e + 1] = qq.y;
+                                    A2.x += fabsf(df.x);
+                                    if (two) A2.y += fabsf(df.y);
+                                    B2 = add2(B2, two ? qq : make_float2(qq.x, 0.f));
+                                    C2 = add2(C2, two ? qj : make_float2(qj.x, 0.f));
+                                }
+                            }
+                            if constexpr (kTvd) {
+                                if constexpr (kCnt == 1) tq = qs[0];
+                                else pack_q<In>(qs, zr, tr);  // written back to tensor memory by the sweep
+                            }
+                        });
+                }
+                // ---- exchange 2: the sums of pass 2
+                const float4 v2 = make_float4(warp_sum(A2.x + A2.y), warp_sum(B2.x + B2.y),
+                                              kJsd ? 0.f : warp_sum(C2.x + C2.y), 0.f);
+                // -> TVD (loss, k1, k2) with the gradient k1 q' + k2 |q'| below; JSD (loss, S)
+                const float4 r2v = exchange(v2, make_float4(0.f, 0.f, 0.f, 0.f), &pbar2, recv2,
+                    [&](float4 x) {
+                        return make_float4(warp_sum(x.x), warp_sum(x.y), kJsd ? 0.f : warp_sum(x.z), 0.f);
+                    },
+                    [&](float4 m, bool&) {
+                        if constexpr (kJsd)
+                            return make_float4(jsd_trivial ? 0.f : kLn2 * (beta * m.x + (1.f - beta) * m.y), m.y, 0.f, 0.f);
+                        else
+                            return make_float4(0.5f * m.x, 0.5f * m.z * inv_tau, -0.5f * m.y * inv_tau, 0.f);
+                    }, failed);
+                row_err = failed;
+                loss = r2v.x;
+                sa = r2v.y;
+                sb = r2v.z;
             }
-            named_arrive(2);
         } else {
-            named_sync(2);
-            const float4 r = s_res;
-            sa = r.x;
-            sb = r.y;
-            sc = r.z;
-            row_err = s_rerr != 0;
+            // ---- exchange 1: the row's maxima and pivot (w flags a failed copy)
+            bool failed = false;
+            const float4 r1v = exchange(make_float4(mz, tp, mt, werr ? 1.f : 0.f),
+                                        make_float4(kNegInf, kNegInf, kNegInf, 0.f), &pbar1, recv1,
+                [&](float4 x) {
+                    const float2 pv = warp_max_pivot(x.x, x.y);
+                    return make_float4(pv.x, pv.y, warp_max(x.z), warp_max(x.w));
+                },
+                [&](float4 m, bool& bad) {
+                    bad = m.w != 0.f;
+                    return m;
+                }, failed);
+            row_err = failed;
+            gz = r1v.x;
+            gt = r1v.z;
+            // the pivot cancels from the loss and the gradient; a -inf one (a -inf target
+            // logit at the draft maximum, or no draft mass) becomes 0
+            tp = r1v.y == kNegInf ? 0.f : r1v.y;
+            if (row_err) {  // the row and the rest of the run report NaN
+                if (rank == 0 && tid == 0) {
+                    p.loss[row] = __int_as_float(0x7fc00000);
+                    if (p.status) atomicExch(p.status, static_cast<int32_t>(OSD_ERR_TIMEOUT));
+                }
+                stop = true;
+                continue;
+            }
+            {
+                // ---- pass 1: the sums and the RKL moment X = sum_j e_j ((z_j - gz) - (t_j - tp))
+                // against the row's maxima (a row with no mass takes m c = 0)
+                float2 Ez2 = f2(0.f), Et2 = f2(0.f), X2 = f2(0.f);
+                bool ninf = false, rinf = false;
+                const float Mz = gz == kNegInf ? 0.f : __fmul_rn(gz, c), Mt = gt == kNegInf ? 0.f : __fmul_rn(gt, c);
+                const float2 gz2 = f2(gz), tp2 = f2(tp);
+                sweep_tm<In, false, false, false, true, false, kTmRklG>(tw, tsh, nv, tail, tz, tt,
+                    [&](const float* z, const float* t, auto tag, int, float, float, bool cninf, uint4&, uint4&) {
+                        constexpr int kCnt = decltype(tag)::value;
+                        if (kCnt == 1 || cninf) {  // element-wise, with the guards a -inf needs
+                            ninf |= cninf;
+#pragma unroll
+                            for (int e = 0; e < kCnt; ++e) {
+                                const float ez = ex2(fmaf(z[e], c, -Mz));
+                                Ez2.x += ez;
+                                Et2.x += ex2(fmaf(t[e], c, -Mt));
+                                if (z[e] != kNegInf) {
+                                    if (t[e] == kNegInf) rinf = true;  // q > 0 = p: the loss is +inf
+                                    else X2.x = fmaf(ez, (z[e] - gz) - (t[e] - tp), X2.x);
+                                }
+                            }
+                        } else {
+#pragma unroll
+                            for (int e = 0; e < kCnt; e += 2) {
+                                const float2 zz = make_float2(z[e], z[e + 1]), tt2 = make_float2(t[e], t[e + 1]);
+                                const float2 a = fma2(zz, f2(c), f2(-Mz)), b = fma2(tt2, f2(c), f2(-Mt));
+                                const float2 ez = make_float2(ex2(a.x), ex2(a.y));
+                                Ez2 = add2(Ez2, ez);
+                                Et2 = add2(Et2, make_float2(ex2(b.x), ex2(b.y)));
+                                X2 = fma2(ez, sub2(sub2(zz, gz2), sub2(tt2, tp2)), X2);
+                            }
+                        }
+                    });
+                // ---- exchange 2: the sums, the moment and the flags (OR-ed as bits in w)
+                const int wf = warp_or((ninf ? kTmNinf : 0) | (rinf ? kTmRklInf : 0));
+                const float4 v2 = make_float4(warp_sum(Ez2.x + Ez2.y), warp_sum(Et2.x + Et2.y),
+                                              warp_sum(X2.x + X2.y), __int_as_float(wf));
+                // -> (loss, cv, K, flags)
+                const float4 r2v = exchange(v2, make_float4(0.f, 0.f, 0.f, 0.f), &pbar2, recv2,
+                    [&](float4 x) {
+                        return make_float4(warp_sum(x.x), warp_sum(x.y), warp_sum(x.z),
+                                           __int_as_float(warp_or(__float_as_int(x.w))));
+                    },
+                    [&](float4 m, bool&) {
+                        const float Ez = m.x, Et = m.y, X = m.z;
+                        const float dz = fold_err(gz), dt = fold_err(gt);
+                        const float lr = logf(Ez / Et) - kLn2 * (dz - dt);
+                        const float l = (__float_as_int(m.w) & kTmRklInf) ? __builtin_huge_valf()
+                                                                          : (X / Ez + (gt - tp)) * inv_tau - lr;
+                        return make_float4(l, -log2_sum(Ez) + dz, X / Ez * inv_tau, m.w);
+                    }, failed);
+                row_err = failed;
+                loss = r2v.x;
+                cv = r2v.y;
+                K = r2v.z;
+                flags = __float_as_int(r2v.w);
+            }
         }
-
         if (rank == 0 && tid == 0) {
-            const float loss = kJsd ? (jsd_trivial ? 0.f : kLn2 * (beta * sa + (1.f - beta) * sb)) : 0.5f * sa;
             p.loss[row] = row_err ? __int_as_float(0x7fc00000) : loss;
             if (row_err && p.status) atomicExch(p.status, static_cast<int32_t>(OSD_ERR_TIMEOUT));
         }
-        if (row_err) {
+        if (row_err) {  // the row and the rest of the run report NaN
             stop = true;
             continue;
         }
@@ -1207,11 +1322,11 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
 
         // ---- pass 3: d loss / d draft logits of the span
         float* orow = p.dlogits + row * V + e0;
-        if constexpr (!kJsd) {
+        if constexpr (kTvd) {
             // d TVD / d z = q (s Q - S) / (2 tau) with s = sign(q - p), S = sum q s
             // and Q = sum q (1 up to rounding; summed, it cancels S exactly where
             // every s is the same): k1 q' + k2 |q'| with k1 = Q / (2 tau), k2 = -S / (2 tau)
-            const float k1 = 0.5f * sc * inv_tau, k2 = -0.5f * sb * inv_tau;
+            const float k1 = sa, k2 = sb;
             sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, 0, tz, tt,
                 [&](const float*, const float*, auto tag, int j0, float, float, bool, uint4& zr, uint4& tr) {
                     constexpr int kCnt = decltype(tag)::value;
@@ -1226,25 +1341,47 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                 });
             if (tid < tail) orow[tail0 + tid] = fmaf(k2, fabsf(tq), k1 * tq);
         } else {
+            // JSD: q (log2(q/m) - S), every probability carrying the gradient's factor,
+            // which cancels in log2(q/m); RKL: q ((z - gz) - (t - tp) - X / E) / tau^2,
+            // q carrying 1 / tau, and 0 where q = 0 meets an infinite log-ratio
             const float2 cvs = f2(cv + p.lg_scale), cus = f2(cu + p.lg_scale);
-            sweep_tm<In, false, false, false, false, false, kTmJsdG>(tw, tsh, nv, tail, tz, tt,
-                [&](const float* z, const float* t, auto tag, int j0, float, float, bool, uint4&, uint4&) {
+            const bool has_ninf = (flags & kTmNinf) != 0;
+            sweep_tm<In, false, false, false, false, false, kJsd ? kTmJsdG : kTmG>(tw, tsh, nv, tail, tz, tt,
+                [&](const float* z, const float* t, auto tag, int j0, float, float, bool, uint4& zr, uint4& tr) {
                     constexpr int kCnt = decltype(tag)::value;
+                    // RKL's bf16 chunks take x - m from the packed words (mixed-precision subtracts)
+                    constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && kRkl;
+                    const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw4[4] = {tr.x, tr.y, tr.z, tr.w};
+                    auto zdiff = [&](int e, float m) {
+                        if constexpr (kRaw) return bf16x2_minus(zw[e / 2], m);
+                        else return sub2(make_float2(z[e], (e + 1 < kCnt) ? z[e + 1] : z[e]), f2(m));
+                    };
+                    auto tdiff = [&](int e, float m) {
+                        if constexpr (kRaw) return bf16x2_minus(tw4[e / 2], m);
+                        else return sub2(make_float2(t[e], (e + 1 < kCnt) ? t[e + 1] : t[e]), f2(m));
+                    };
                     float gr[kCnt];
 #pragma unroll
                     for (int e = 0; e < kCnt; e += 2) {
                         const bool two = (e + 1 < kCnt);
+                        const float2 zd = zdiff(e, gz);
+                        const float2 v = fma2(zd, f2(c), cvs);
+                        const float2 qj = make_float2(ex2(v.x), ex2(v.y));
                         float2 gg;
-                        if (jsd_trivial) {
+                        if constexpr (kRkl) {
+                            gg = mul2(qj, fma2(sub2(zd, tdiff(e, tp)), f2(inv_tau), f2(-K)));
+                            if (has_ninf) {
+                                if (!(qj.x > 0.f)) gg.x = 0.f;
+                                if (!(qj.y > 0.f)) gg.y = 0.f;
+                            }
+                        } else if (jsd_trivial) {
                             gg = f2(0.f);
                         } else {
-                            const float2 v = fma2(sub2(make_float2(z[e], two ? z[e + 1] : z[e]), f2(gz)), f2(c), cvs);
-                            const float2 u = fma2(sub2(make_float2(t[e], two ? t[e + 1] : t[e]), f2(gt)), f2(c), cus);
-                            const float2 qj = make_float2(ex2(v.x), ex2(v.y));
+                            const float2 u = fma2(tdiff(e, gt), f2(c), cus);
                             const float2 pj = make_float2(ex2(u.x), ex2(u.y));
                             const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
                             const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
-                            gg = mul2(qj, sub2(sub2(v, lm), f2(sb)));
+                            gg = mul2(qj, sub2(sub2(v, lm), f2(sa)));
                         }
                         gr[e] = gg.x;
                         if (two) gr[e + 1] = gg.y;
@@ -1429,7 +1566,11 @@ static cudaError_t launch_distill_tm(const DistParams& dp, long long rows, cudaS
 }
 template <typename In>
 static cudaError_t launch_distill_tm_kind(osd_loss kind, const DistParams& dp, long long rows, cudaStream_t s) {
-    return (kind == OSD_JSD) ? launch_distill_tm<In, OSD_JSD>(dp, rows, s) : launch_distill_tm<In, OSD_TVD>(dp, rows, s);
+    switch (kind) {
+        case OSD_JSD: return launch_distill_tm<In, OSD_JSD>(dp, rows, s);
+        case OSD_RKL: return launch_distill_tm<In, OSD_RKL>(dp, rows, s);
+        default: return launch_distill_tm<In, OSD_TVD>(dp, rows, s);
+    }
 }
 
 // Shared by both entry points: argument checks, shape, and the launch.
@@ -1452,11 +1593,11 @@ static osd_status distill_run(const void* draft_logits, const void* target_logit
                          aligned_to(dlogits, 16) && (size_t(V) * 4) % 16 == 0 &&
                          row_ok(d_stride_g, G) && row_ok(d_stride_p, p_rows) && row_ok(t_stride_g, G) &&
                          row_ok(t_stride_p, p_rows);
-    // the TMEM-staged runs (if the span fits) for the kinds with a second pass, where
-    // they measured faster: TVD 94.6 % against 70.1 % of the HBM peak, JSD 71.3 %
-    // against 63.0 % (65536 x 32000 bf16); FKL, RKL and CE, near the bandwidth roof on
-    // the per-row kernel, measured 1-13 points slower on an earlier form of them
-    const bool tm_path = aligned && !accepted && (kind == OSD_TVD || kind == OSD_JSD);
+    // the TMEM-staged runs (if the span fits) for TVD, JSD and RKL, where they
+    // measured faster: TVD 94.7 % against 70.1 % of the HBM peak, JSD 71.6 % against
+    // 63.0 %, RKL 95.1 % against 86.4 % (65536 x 32000 bf16); FKL and CE, at 90.9 %
+    // and 96.3 % on the per-row kernel, measured slower on an earlier form of them
+    const bool tm_path = aligned && !accepted && (kind == OSD_TVD || kind == OSD_JSD || (kTmRkl && kind == OSD_RKL));
     int csize = 1, span = V;
     // JSD, with the most work per entry, stages best in longer spans on the per-row
     // kernel; the TMEM-staged runs take the 32 KB spans for every kind.  (At
