@@ -359,7 +359,9 @@ def run_ours(args):
                 # the distill counters were taken on the RKL and TVD launches of the default step
                 "traffic": ((_traffic("distill", DISTILL_SOURCES) if kinds == ["rkl", "tvd"] else None)
                             if top == "distill" else _traffic("verify", VERIFY_SOURCES)),
-                "kernel": "distill_kernel" if top == "distill" else "row_stats_kernel + verify_finalize_kernel",
+                "kernel": (" + ".join(("distill_tm_kernel " if k in ("rkl", "tvd", "jsd") else "distill_kernel ")
+                                      + k.upper() for k in kinds) if top == "distill"
+                           else "row_stats_kernel + verify_finalize_kernel"),
                 "peak_source": peak_src}
 
     e2e = None
