@@ -9,6 +9,7 @@ and torch's allocations where they were.
 This file is collected last on purpose, and it needs nothing from the other
 tests: it passes alone in a fresh process and after the rest of the suite."""
 import ctypes
+import gc
 
 import numpy as np
 import pytest
@@ -65,17 +66,24 @@ def test_noalloc_allocates_nothing(osd):
     # the kernels' module is loaded (with the array in it) by a plain osd_verify call first
     osd.osd_verify(inp["draft"], inp["target"], inp["tokens"], inp["uniforms"], 1.0)
     outs = [_outputs(spec.B, spec.k, dev) for _ in range(3)]
-    torch.cuda.synchronize()
-    alloc0 = torch.cuda.memory_allocated(dev)
-    reserved0 = torch.cuda.memory_reserved(dev)
-    free0, _ = torch.cuda.mem_get_info(dev)
-    for out in outs:
-        osd.osd_verify_noalloc(inp["draft"], inp["target"], inp["tokens"], inp["uniforms"], 1.0, out)
+    # earlier tests' tensors held in reference cycles would otherwise be freed by the
+    # cyclic collector in the middle of the measurement
+    gc.collect()
+    gc.disable()
+    try:
         torch.cuda.synchronize()
-        assert torch.cuda.memory_allocated(dev) == alloc0
-        assert torch.cuda.memory_reserved(dev) == reserved0
-        free1, _ = torch.cuda.mem_get_info(dev)
-        assert free1 == free0, f"device free memory moved by {free0 - free1} bytes"
+        alloc0 = torch.cuda.memory_allocated(dev)
+        reserved0 = torch.cuda.memory_reserved(dev)
+        free0, _ = torch.cuda.mem_get_info(dev)
+        for out in outs:
+            osd.osd_verify_noalloc(inp["draft"], inp["target"], inp["tokens"], inp["uniforms"], 1.0, out)
+            torch.cuda.synchronize()
+            assert torch.cuda.memory_allocated(dev) == alloc0
+            assert torch.cuda.memory_reserved(dev) == reserved0
+            free1, _ = torch.cuda.mem_get_info(dev)
+            assert free1 == free0, f"device free memory moved by {free0 - free1} bytes"
+    finally:
+        gc.enable()
     _same(outs[1], outs[0])
     _same(outs[2], outs[0])
 
