@@ -600,7 +600,7 @@ __global__ void __launch_bounds__(kFuseThreads) verify_fused_kernel(FinParams p)
     constexpr int kWarps = kFuseThreads / 32;
     constexpr int kMaxRows = 2 * OSD_VERIFY_MAX_K + 1;
     extern __shared__ __align__(128) unsigned char fsm[];
-    __shared__ __align__(8) uint64_t bar;
+    __shared__ __align__(8) uint64_t rbar[kMaxRows];  // one staging barrier per row
     __shared__ SeqSmem sh;
     __shared__ DrawSmem ds;
     __shared__ MaxSum part_ms[kMaxRows * kFuseParts];
@@ -619,11 +619,14 @@ __global__ void __launch_bounds__(kFuseThreads) verify_fused_kernel(FinParams p)
     float* s_sub = reinterpret_cast<float*>(fsm + size_t(nrows) * p.span * sizeof(In));
     const uint32_t bytes = static_cast<uint32_t>(n * sizeof(In));  // a multiple of 16 on this path
 
-    // ---- stage every row's span (one barrier, all the copies in flight at once)
+    // ---- stage every row's span (all the copies in flight at once, a barrier per row,
+    // so that a row's statistics start as soon as it has landed)
     if (tid == 0) {
-        mbar_init(&bar, 1);
-        mbar_arrive_expect_tx(&bar, bytes * static_cast<uint32_t>(nrows));
-        for (int r = 0; r < nrows; ++r) bulk_g2s(rows + size_t(r) * p.span, fused_src<In>(p, b, r, e0), bytes, &bar);
+        for (int r = 0; r < nrows; ++r) mbar_init(&rbar[r], 1);
+        for (int r = 0; r < nrows; ++r) {
+            mbar_arrive_expect_tx(&rbar[r], bytes);
+            bulk_g2s(rows + size_t(r) * p.span, fused_src<In>(p, b, r, e0), bytes, &rbar[r]);
+        }
     }
     // meanwhile the draft tokens, the two logits each accept test needs, and the uniforms
     int bad = 0;
@@ -642,36 +645,38 @@ __global__ void __launch_bounds__(kFuseThreads) verify_fused_kernel(FinParams p)
     }
     if (warp == kWarps - 2)
         for (int i = lane; i <= k; i += 32) sh.u[i] = p.uniforms[size_t(b) * (k + 1) + i];
-    __syncthreads();  // the barrier is initialised before anyone waits on it
-    const int timed_out = mbar_wait_bounded(&bar, 0, kFuseWaitNs) ? 0 : 1;
+    __syncthreads();  // the barriers are initialised before anyone waits on them
     bad = __syncthreads_or(bad);
-    const int tmo = __syncthreads_or(timed_out);
-    if (tmo) mbar_wait_bounded(&bar, 0, kFuseWaitNs);  // a copy that gave up gets a last chance to land
-    if (tid == 0) s_tmo = tmo;
+    // every row's copy has landed (or its wait gave up) before this CTA leaves
+    auto wait_all = [&]() {
+        int t = 0;
+        for (int r = 0; r < nrows; ++r) t |= mbar_wait_bounded(&rbar[r], 0, kFuseWaitNs) ? 0 : 1;
+        return t;
+    };
     if (bad) {  // uniform over the cluster, before any distributed shared memory access
+        wait_all();
         if (rank == 0) seq_write_bad<kFuseThreads>(p, b);
         return;
     }
 
-    // ---- span statistics of every row: warp items (row, part), then per row over the parts
+    // ---- span statistics of every row: warp items (row, part), each its row's
+    // maximum first, then the sum of 2^((x - m) c) against it; then per row over the parts
     const int nch = n / kVec;
     const float ch = p.c_hi, cl = p.c_lo;
+    int timed_out = 0;
     for (int it = warp; it < nrows * kFuseParts; it += kWarps) {
         const int r = it / kFuseParts, part = it - r * kFuseParts;
+        if (!mbar_wait_bounded(&rbar[r], 0, kFuseWaitNs)) timed_out = 1;
         const In* row = rows + size_t(r) * p.span;
         const int c0 = nch * part / kFuseParts, c1 = nch * (part + 1) / kFuseParts;
         float m = kNegInf;
+        for (int c = c0 + lane; c < c1; c += 32) m = fmaxf(m, E::max_raw(lds_v4(row + c * kVec)));
+        for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
         float2 s2 = f2(0.f);
-        for (int c = c0 + lane; c < c1; c += 32) {
-            const uint4 w = lds_v4(row + c * kVec);
-            const float cm = E::max_raw(w);
-            if (cm > m) {
-                s2 = (m == kNegInf) ? f2(0.f) : mul2(s2, f2(ex2(mul_c(m - cm, ch, cl))));
-                m = cm;
-            }
-            if (m != kNegInf) {
+        if (m != kNegInf) {
+            for (int c = c0 + lane; c < c1; c += 32) {
                 float x[kVec];
-                E::unpack(w, x);
+                E::unpack(lds_v4(row + c * kVec), x);
 #pragma unroll
                 for (int e = 0; e < kVec; e += 2) {
                     const float2 d = sub2(make_float2(x[e], x[e + 1]), f2(m));
@@ -680,11 +685,13 @@ __global__ void __launch_bounds__(kFuseThreads) verify_fused_kernel(FinParams p)
                 }
             }
         }
-        MaxSum acc{m, s2.x + s2.y};
-        acc = warp_reduce(acc, [ch, cl](MaxSum x, MaxSum z) { return merge_ms(x, z, ch, cl); });
-        if (lane == 0) part_ms[it] = acc;
+        float s = s2.x + s2.y;
+        for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+        if (lane == 0) part_ms[it] = MaxSum{m, s};
     }
-    __syncthreads();
+    const int tmo = __syncthreads_or(timed_out);
+    if (tmo) wait_all();  // a copy that gave up gets a last chance to land
+    if (tid == 0) s_tmo = tmo;
     if (tid < nrows) {
         MaxSum acc = part_ms[tid * kFuseParts];
         for (int q = 1; q < kFuseParts; ++q) acc = merge_ms(acc, part_ms[tid * kFuseParts + q], ch, cl);
