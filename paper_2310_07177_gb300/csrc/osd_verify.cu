@@ -43,6 +43,7 @@ namespace osd {
 
 constexpr int kFinThreads = 128;
 constexpr int kFinMaxCluster = 8;
+constexpr uint64_t kDrawWaitNs = 3000000000ull;  // bound on the wait for the pushed span totals
 constexpr int kFinMaxSub = 8192;  // sub-tiles of one CTA's vocabulary span (>= span / 32)
 constexpr int kFinUnroll = 4;     // sub-tiles of loads in flight per warp
 
@@ -276,6 +277,9 @@ struct DrawSmem {
     unsigned long long span_total;
     unsigned long long tau, W, base;
     int owner, mode, tile;
+    // pushed span totals (the one-launch kernel): slot r from CTA r, completing on tbar
+    unsigned long long totals[kFinMaxCluster];
+    uint64_t tbar;
 };
 
 // The extra token of sequence b (Appendix A.1; reading 4 and 4b for the
@@ -288,10 +292,15 @@ struct DrawSmem {
 // draft rows at position a is trow[j - off], zrow[j - off], in shared memory when
 // kSmem (a staged span) and global memory otherwise; trow_g is the whole target
 // row in global memory, for the case W = 0 (argmax of p_a).  s_sub holds at least
-// n / (32 kW) floats.  Every thread calls it; it ends having arrived (relaxed) at
-// the cluster barrier, and the caller waits there before it exits.
-template <typename In, bool kVecPath, int kThreads, bool kSmem>
-__device__ __forceinline__ void residual_draw(const FinParams& p, int b, int a, const SeqSmem& sh, int rank,
+// n / (32 kW) floats.  Every thread calls it.  Without kPush the totals are read
+// from the peers' shared memory after a cluster barrier, and the draw ends
+// having arrived (relaxed) at the cluster barrier, where the caller waits before
+// it exits.  With kPush (ds.tbar initialised with count 1 and visible to the
+// cluster) each CTA pushes its total by st.async into slot `rank` of every CTA's
+// ds.totals and waits on its own ds.tbar: no cluster barrier, nothing read from
+// a peer.  Returns false if that wait gave up (the draw is then not made).
+template <typename In, bool kVecPath, int kThreads, bool kSmem, bool kPush = false>
+__device__ __forceinline__ bool residual_draw(const FinParams& p, int b, int a, const SeqSmem& sh, int rank,
                                               int e0, int n, const In* trow, const In* zrow, int off,
                                               const In* trow_g, float* s_sub, DrawSmem& ds) {
     using E = Elem<In>;
@@ -388,20 +397,31 @@ __device__ __forceinline__ void residual_draw(const FinParams& p, int b, int a, 
     }
     __syncthreads();
     // span total, exact, reduced across warp 0
+    bool got = true;
     if (warp == 0) {
         unsigned long long part = 0ull;
         for (int s2 = lane; s2 < nsub; s2 += 32) part += fix_of(s_sub[s2]);
         part = warp_sum_u64(part);
         if (lane == 0) ds.span_total = part;
+        if (kPush && p.csize > 1) {
+            if (lane < p.csize)
+                st_async_u64(map_rank(&ds.totals[rank], static_cast<uint32_t>(lane)), part,
+                             map_rank(&ds.tbar, static_cast<uint32_t>(lane)));
+            if (lane == 0) mbar_arrive_expect_tx(&ds.tbar, static_cast<uint32_t>(p.csize) * 8u);
+            got = __all_sync(0xffffffffu, mbar_wait_cluster_bounded(&ds.tbar, 0, kDrawWaitNs));
+        }
     }
-    if (p.csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
+    if (!kPush && p.csize > 1) cluster_sync_publish(tid == 0); else __syncthreads();
 
     // warp 0 of every CTA derives W, tau = floor(u W) and the owning CTA identically:
     // lane r holds CTA r's total, a warp scan gives the prefix in rank order
-    if (warp == 0) {
+    if (warp == 0 && got) {
         const float u = sh.u[k];
         unsigned long long tot = 0ull;
-        if (lane < p.csize) tot = (lane == rank) ? ds.span_total : ld_dsmem_u64(map_rank(&ds.span_total, lane));
+        if (lane < p.csize) {
+            if (kPush) tot = (p.csize > 1) ? ds.totals[lane] : ds.span_total;
+            else tot = (lane == rank) ? ds.span_total : ld_dsmem_u64(map_rank(&ds.span_total, lane));
+        }
         const unsigned long long incl = warp_incl_scan_u64(tot);
         const unsigned long long W = __shfl_sync(0xffffffffu, incl, 31);
         const unsigned long long tau = fix_scale(u, W);
@@ -458,8 +478,10 @@ __device__ __forceinline__ void residual_draw(const FinParams& p, int b, int a, 
         }
         if (lane == 0) { ds.owner = owner; ds.mode = mode; ds.tau = tau; ds.W = W; ds.base = base; ds.tile = tile; }
     }
+    if (warp == 0 && lane == 0 && !got) ds.owner = -1;
     __syncthreads();
-    if (p.csize > 1) cluster_arrive_relaxed();  // done reading the other CTAs' shared memory
+    if (!kPush && p.csize > 1) cluster_arrive_relaxed();  // done reading the other CTAs' shared memory
+    if (ds.owner < 0) return false;
 
     if (rank == ds.owner && warp == 0) {
         const unsigned long long tau = ds.tau, W = ds.W;
@@ -529,6 +551,7 @@ __device__ __forceinline__ void residual_draw(const FinParams& p, int b, int a, 
             }
         }
     }
+    return true;
 }
 
 template <typename In, bool kVecPath>
@@ -571,8 +594,11 @@ __global__ void __launch_bounds__(kFinThreads) verify_finalize_kernel(FinParams 
 // CTA bulk-copies its vocabulary span of all 2k+1 rows into shared memory,
 // computes the span's statistics of every row from there, merges them across
 // the cluster, runs the accept tests, and draws the extra token from the staged
-// rows (residual_draw) without reading them again.  It runs only when its grid
-// fits in one wave (fused_shape).  At B = 32, k = 5, V = 32000 it measured 23.9 us
+// rows (residual_draw) without reading them again.  The CTAs exchange the span
+// statistics and the residual totals by pushing them with st.async into every
+// peer's shared memory, each CTA waiting on its own barrier: no cluster barrier
+// after the start, no fence, and nothing read from a peer.  It runs only when
+// its grid fits in one wave (fused_shape).  At B = 32, k = 5, V = 32000 it measured 23.9 us
 // in the bench step against 27.1 us for the two launches (512 threads; 256 threads
 // 26.7 us; 16-CTA clusters 38 us).  The greedy pass (T = 0) keeps its two
 // launches: one launch over the k+1 target rows measured 11.2 against 10.3 us.
@@ -582,6 +608,12 @@ constexpr int kFuseParts = 4;           // warp items per row for the span stati
 constexpr int kFuseMaxB = 64;           // at most this many sequences, and the grid in one wave
 constexpr size_t kFuseMaxSmem = 200 * 1024;  // staged rows + sub-tile sums per CTA
 constexpr uint64_t kFuseWaitNs = 1000000000ull;  // bound on the wait for the staged rows
+
+// Byte offset of the one-launch kernel's receive slots in its dynamic shared
+// memory: after the staged rows and the sub-tile sums, 16-byte aligned.
+__host__ __device__ inline size_t fused_recv_offset(int nrows, int span, size_t es) {
+    return (size_t(nrows) * span * es + size_t(span / 128 + 1) * sizeof(float) + 15) / 16 * 16;
+}
 
 // Rows of sequence b staged by this CTA: local row r <= k is target row r, r > k
 // draft row r-k-1; each holds entries [e0, e0 + n) at r * span.
@@ -604,8 +636,8 @@ __global__ void __launch_bounds__(kFuseThreads) verify_fused_kernel(FinParams p)
     __shared__ SeqSmem sh;
     __shared__ DrawSmem ds;
     __shared__ MaxSum part_ms[kMaxRows * kFuseParts];
-    __shared__ MaxSum cta_ms[kMaxRows];  // this CTA's span statistics per row (read by the peers)
-    __shared__ int s_tmo, s_any_tmo;  // a staging copy gave up: this CTA's, any of the cluster's
+    __shared__ __align__(8) uint64_t sbar;  // the cluster's span statistics have arrived
+    __shared__ int s_any_tmo;  // a staging copy (or a wait for the peers) gave up in the cluster
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int csize = p.csize;
@@ -617,12 +649,17 @@ __global__ void __launch_bounds__(kFuseThreads) verify_fused_kernel(FinParams p)
     const int n = min(p.span, V - e0);
     In* rows = reinterpret_cast<In*>(fsm);
     float* s_sub = reinterpret_cast<float*>(fsm + size_t(nrows) * p.span * sizeof(In));
+    // [csize][nrows]: CTA c's span statistics of every row, pushed by CTA c
+    MaxSum* recv_ms = reinterpret_cast<MaxSum*>(fsm + fused_recv_offset(nrows, p.span, sizeof(In)));
     const uint32_t bytes = static_cast<uint32_t>(n * sizeof(In));  // a multiple of 16 on this path
 
     // ---- stage every row's span (all the copies in flight at once, a barrier per row,
     // so that a row's statistics start as soon as it has landed)
     if (tid == 0) {
-        for (int r = 0; r < nrows; ++r) mbar_init(&rbar[r], 1);
+        for (int r = 0; r < nrows; ++r) mbar_init_only(&rbar[r], 1);
+        mbar_init_only(&sbar, 1);
+        mbar_init_only(&ds.tbar, 1);
+        fence_mbarrier_init();
         for (int r = 0; r < nrows; ++r) {
             mbar_arrive_expect_tx(&rbar[r], bytes);
             bulk_g2s(rows + size_t(r) * p.span, fused_src<In>(p, b, r, e0), bytes, &rbar[r]);
@@ -646,6 +683,8 @@ __global__ void __launch_bounds__(kFuseThreads) verify_fused_kernel(FinParams p)
     if (warp == kWarps - 2)
         for (int i = lane; i <= k; i += 32) sh.u[i] = p.uniforms[size_t(b) * (k + 1) + i];
     __syncthreads();  // the barriers are initialised before anyone waits on them
+    // ... and before any peer pushes to them: arrive now, wait before the first push
+    if (csize > 1) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
     bad = __syncthreads_or(bad);
     // every row's copy has landed (or its wait gave up) before this CTA leaves
     auto wait_all = [&]() {
@@ -653,7 +692,7 @@ __global__ void __launch_bounds__(kFuseThreads) verify_fused_kernel(FinParams p)
         for (int r = 0; r < nrows; ++r) t |= mbar_wait_bounded(&rbar[r], 0, kFuseWaitNs) ? 0 : 1;
         return t;
     };
-    if (bad) {  // uniform over the cluster, before any distributed shared memory access
+    if (bad) {  // uniform over the cluster, before any push to a peer
         wait_all();
         if (rank == 0) seq_write_bad<kFuseThreads>(p, b);
         return;
@@ -691,41 +730,41 @@ __global__ void __launch_bounds__(kFuseThreads) verify_fused_kernel(FinParams p)
     }
     const int tmo = __syncthreads_or(timed_out);
     if (tmo) wait_all();  // a copy that gave up gets a last chance to land
-    if (tid == 0) s_tmo = tmo;
+    // ---- the cluster's spans: thread r < nrows merges its row's parts and pushes the
+    // result (a negative sum flags a copy that gave up) into slot `rank` of every CTA;
+    // every CTA then merges the csize slots of each row in rank order (lane c <- CTA c)
     if (tid < nrows) {
         MaxSum acc = part_ms[tid * kFuseParts];
         for (int q = 1; q < kFuseParts; ++q) acc = merge_ms(acc, part_ms[tid * kFuseParts + q], ch, cl);
-        cta_ms[tid] = acc;
+        if (tmo) acc.s = -1.f;
+        if (csize > 1) {
+            asm volatile("barrier.cluster.wait.acquire;" ::: "memory");  // the peers' barriers are ready
+            for (int d = 0; d < csize; ++d)
+                st_async_v2(map_rank(&recv_ms[rank * nrows + tid], static_cast<uint32_t>(d)), make_float2(acc.m, acc.s),
+                            map_rank(&sbar, static_cast<uint32_t>(d)));
+        } else {
+            recv_ms[tid] = acc;
+        }
     }
-    // ---- the cluster's spans: every CTA merges all of them in rank order (lane c <- CTA c)
-    if (csize > 1) cluster_sync_publish(tid < nrows || tid == 0); else __syncthreads();
-    if (warp == 0) {  // did any CTA of the cluster miss its rows?
-        int f = 0;
-        if (lane < csize) f = (lane == rank) ? s_tmo : ld_dsmem_s32(map_rank(&s_tmo, lane));
-        f = __any_sync(0xffffffffu, f != 0);
-        if (lane == 0) s_any_tmo = f;
+    if (csize > 1) {
+        if (tid >= nrows) asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
+        if (tid == 0) mbar_arrive_expect_tx(&sbar, static_cast<uint32_t>(csize * nrows) * 8u);
     }
+    bool got = true;
+    if (csize > 1) got = mbar_wait_cluster_bounded(&sbar, 0, kFuseWaitNs); else __syncthreads();
+    got = __syncthreads_and(got);
+    int any_tmo = got ? 0 : 1;
     for (int r = warp; r < nrows; r += kWarps) {
         MaxSum o{kNegInf, 0.f};
-        if (lane < csize) {
-            if (lane == rank) {
-                o = cta_ms[r];
-            } else {
-                const uint32_t base = map_rank(&cta_ms[r], lane);
-                o.m = ld_dsmem_f32(base + offsetof(MaxSum, m));
-                o.s = ld_dsmem_f32(base + offsetof(MaxSum, s));
-            }
-        }
+        if (lane < csize && got) o = recv_ms[lane * nrows + r];
+        if (__any_sync(0xffffffffu, o.s < 0.f)) any_tmo = 1;
+        o.s = fmaxf(o.s, 0.f);
         o = warp_reduce(o, [ch, cl](MaxSum x, MaxSum z) { return merge_ms(x, z, ch, cl); });
         if (lane == 0) { sh.m[r] = o.m; sh.s[r] = o.s; }
     }
-    __syncthreads();
-    if (s_any_tmo) {  // the GPU did not deliver a row in time: the sequence is reported as bad
+    any_tmo = __syncthreads_or(any_tmo);
+    if (any_tmo) {  // the GPU did not deliver a row in time: the sequence is reported as bad
         if (rank == 0) seq_write_bad<kFuseThreads>(p, b);
-        if (csize > 1) {
-            cluster_arrive_relaxed();
-            cluster_wait();
-        }
         return;
     }
 
@@ -737,8 +776,10 @@ __global__ void __launch_bounds__(kFuseThreads) verify_fused_kernel(FinParams p)
     const In* trow_s = rows + size_t(a) * p.span;
     const In* zrow_s = bonus ? trow_s : rows + size_t(k + 1 + a) * p.span;
     const In* trow_g = static_cast<const In*>(p.target) + (size_t(b) * (k + 1) + a) * V;
-    residual_draw<In, true, kFuseThreads, true>(p, b, a, sh, rank, e0, n, trow_s, zrow_s, e0, trow_g, s_sub, ds);
-    if (csize > 1) cluster_wait();  // keep this CTA's shared memory alive for its peers
+    // (a peer whose pushed total did not arrive in time reports the sequence as bad)
+    if (!residual_draw<In, true, kFuseThreads, true, true>(p, b, a, sh, rank, e0, n, trow_s, zrow_s, e0, trow_g,
+                                                        s_sub, ds))
+        seq_write_bad<kFuseThreads>(p, b);
 }
 
 // ------------------------------------------------------------------ host
@@ -810,7 +851,7 @@ static bool fused_shape(int B, int k, int V, bool greedy, const void* draft, con
     s = (s + 63) / 64 * 64;
     c = (V + s - 1) / s;
     const int nrows = 2 * k + 1;
-    const size_t bytes = size_t(nrows) * s * sizeof(In) + size_t(s / 128 + 1) * sizeof(float);
+    const size_t bytes = fused_recv_offset(nrows, s, sizeof(In)) + size_t(c) * nrows * sizeof(MaxSum);
     if (bytes > kFuseMaxSmem) return false;
     // only in one wave: at B = 32, k = 5, V = 32000 (two CTAs an SM) one launch took
     // 22.2 us against 23.2 us for two; from B = 48 on, past one wave, 34 against 26 us
