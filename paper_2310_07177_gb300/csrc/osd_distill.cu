@@ -17,6 +17,10 @@
 // Every CTA merges the cluster's partials in rank order, so all CTAs of a row
 // see bit-identical statistics.  Logs and exponentials use the hardware
 // lg2/ex2 units in base 2; loss terms are converted to nats at the end.
+//
+// Buffer flushes of 16-byte-aligned rows (FKL, RKL, JSD, TVD) take the
+// TMEM-staged runs of rows further down instead, which overlap the copy of a
+// row with the passes of the one before it.
 #include <algorithm>
 #include <atomic>
 #include <climits>
@@ -35,7 +39,9 @@ namespace osd {
 constexpr int kDistThreads = kRowThreads;      // threads per CTA ...
 constexpr int kDistThreadsWide = 256;          // ... and for spans of kDistWideSpan entries or more, where
 constexpr int kDistWideSpan = 12288;           // FKL, RKL, CE and JSD measured 5-10 % faster (V = 128256)
-constexpr int kDistMaxCluster = 8;
+constexpr int kDistMaxCluster = 8;            // CTAs per row that bound the vocabulary (V limits) ...
+constexpr int kDistMaxClusterWide = 16;       // ... and up to 16 (non-portable clusters) where a row needs
+                                              // more than 8 spans of the target size (V > 65536 bf16)
 constexpr int kDistSpanBytes = 32768;         // target bytes of both rows per CTA
 constexpr int kDistSpanBytesJsd = 49152;      // JSD, with the most work per entry, does best with fewer, longer spans
 constexpr int kDistMaxSmem = 192 * 1024;      // largest staging buffer per CTA
@@ -720,11 +726,11 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
 // of row i, with the shared-memory footprint of one staged span per CTA.  The
 // hardware schedules the runs like any grid (no assumption on how many
 // clusters are resident), and masked-out rows of a run cost one mask read.
-// 16-byte-aligned rows; TVD, JSD and RKL (FKL and CE measured slower on an
-// earlier form of these runs than on the per-row kernel).  A row costs one CTA
-// barrier (the staging buffer is free) and two exchanges within the cluster:
-// TVD and JSD exchange the normalisers, then the sums of pass 2; RKL the maxima
-// with its pivot, then the sums and its moment.
+// 16-byte-aligned rows; TVD, JSD, RKL and FKL (CE, which needs no second
+// exchange, stays on the per-row kernel, at 96 % of the HBM peak there).  A row
+// costs one CTA barrier (the staging buffer is free) and two exchanges within
+// the cluster: TVD and JSD exchange the normalisers, then the sums of pass 2;
+// RKL and FKL the maxima (RKL with its pivot), then the sums and the moment.
 constexpr int kTmThreads = 128;  // one warp per tensor-memory lane quarter
 constexpr int kTmG = 2;          // chunk slots per round of tensor-memory loads
 constexpr int kTmRows = 8;       // rows per cluster run
@@ -737,10 +743,11 @@ struct TmShape {
     int slots;       // 16-byte chunks of each row per thread
     int t_off;       // first column of the target words (z words from column 0)
     uint32_t ncols;  // tensor-memory columns per CTA
-    // runs, longest first: rows [0, end8) in runs of kTmRows, [end8, end2) in runs
-    // of 2, then runs of one row; n8 and n2 runs of the first two kinds
+    // runs, longest first: rows [0, end8) in runs of `run` (8, 4 or 2), [end8, end2)
+    // in runs of 2, then runs of one row; n8 and n2 runs of the first two kinds
     long long end8, end2;
     int n8, n2;
+    int run;
 };
 
 // This thread's chunks of a span held in tensor memory: slot s is chunk
@@ -892,11 +899,13 @@ constexpr int kTmRklInf = 2;  // a finite draft logit meets a -inf target logit:
 
 template <typename In, int kKind>
 __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p, TmShape tsh) {
-    static_assert(kKind == OSD_TVD || kKind == OSD_JSD || kKind == OSD_RKL,
-                  "the TMEM-staged runs serve TVD, JSD and RKL");
+    static_assert(kKind == OSD_TVD || kKind == OSD_JSD || kKind == OSD_RKL || kKind == OSD_FKL,
+                  "the TMEM-staged runs serve TVD, JSD, RKL and FKL");
     constexpr int kT = kTmThreads, kW = kT / 32;
     constexpr int kVec = Elem<In>::kVec;
     constexpr bool kJsd = kKind == OSD_JSD, kTvd = kKind == OSD_TVD, kRkl = kKind == OSD_RKL;
+    constexpr bool kFkl = kKind == OSD_FKL;
+    constexpr bool kMom = kRkl || kFkl;  // the maxima go round first, then the sums with the loss moment
     // TVD, RKL: exponent arguments x c - m c as one fma; JSD: logits clamped to -1e30, (x - m) c
     constexpr bool kFold = !kJsd;
     extern __shared__ __align__(128) unsigned char dsm[];
@@ -1006,8 +1015,8 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
     // this cluster's run of rows; masked-out rows get loss 0 and are skipped
     long long r0, r1;
     if (cid < tsh.n8) {
-        r0 = static_cast<long long>(cid) * kTmRows;
-        r1 = min(tsh.end8, r0 + kTmRows);
+        r0 = static_cast<long long>(cid) * tsh.run;
+        r1 = min(tsh.end8, r0 + tsh.run);
     } else if (cid < tsh.n8 + tsh.n2) {
         r0 = tsh.end8 + 2ll * (cid - tsh.n8);
         r1 = min(tsh.end2, r0 + 2);
@@ -1107,7 +1116,7 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
         float sa = 0.f, sb = 0.f;  // TVD: k1, k2 of the gradient; JSD: S = sum q log2(q/m) (in sa)
         bool row_err;
         float loss = 0.f;
-        if constexpr (!kRkl) {
+        if constexpr (!kMom) {
             // ---- pass 1: sums of 2^((x - m) c) against the warp's maxima (TVD: a warp
             // whose entries are all -inf takes m c = 0, and its terms 2^-inf = 0)
             float2 Ez2 = f2(0.f), Et2 = f2(0.f);
@@ -1225,7 +1234,7 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                 sb = r2v.z;
             }
         } else {
-            // ---- exchange 1: the row's maxima and pivot (w flags a failed copy)
+            // ---- exchange 1: the row's maxima, with RKL's pivot (w flags a failed copy)
             bool failed = false;
             const float4 r1v = exchange(make_float4(mz, tp, mt, werr ? 1.f : 0.f),
                                         make_float4(kNegInf, kNegInf, kNegInf, 0.f), &pbar1, recv1,
@@ -1252,8 +1261,9 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                 continue;
             }
             {
-                // ---- pass 1: the sums and the RKL moment X = sum_j e_j ((z_j - gz) - (t_j - tp))
-                // against the row's maxima (a row with no mass takes m c = 0)
+                // ---- pass 1: the sums and the loss moment against the row's maxima (a row
+                // with no mass takes m c = 0): RKL X = sum_j e_z,j ((z_j - gz) - (t_j - tp)),
+                // FKL X = sum_j e_t,j (t_j - z_j)
                 float2 Ez2 = f2(0.f), Et2 = f2(0.f), X2 = f2(0.f);
                 bool ninf = false, rinf = false;
                 const float Mz = gz == kNegInf ? 0.f : __fmul_rn(gz, c), Mt = gt == kNegInf ? 0.f : __fmul_rn(gt, c);
@@ -1266,11 +1276,16 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
 #pragma unroll
                             for (int e = 0; e < kCnt; ++e) {
                                 const float ez = ex2(fmaf(z[e], c, -Mz));
+                                const float et = ex2(fmaf(t[e], c, -Mt));
                                 Ez2.x += ez;
-                                Et2.x += ex2(fmaf(t[e], c, -Mt));
-                                if (z[e] != kNegInf) {
-                                    if (t[e] == kNegInf) rinf = true;  // q > 0 = p: the loss is +inf
-                                    else X2.x = fmaf(ez, (z[e] - gz) - (t[e] - tp), X2.x);
+                                Et2.x += et;
+                                if constexpr (kRkl) {
+                                    if (z[e] != kNegInf) {
+                                        if (t[e] == kNegInf) rinf = true;  // q > 0 = p: the loss is +inf
+                                        else X2.x = fmaf(ez, (z[e] - gz) - (t[e] - tp), X2.x);
+                                    }
+                                } else if (et > 0.f) {  // p > 0 = q makes X, and the loss, +inf
+                                    X2.x = fmaf(et, t[e] - z[e], X2.x);
                                 }
                             }
                         } else {
@@ -1279,9 +1294,11 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                                 const float2 zz = make_float2(z[e], z[e + 1]), tt2 = make_float2(t[e], t[e + 1]);
                                 const float2 a = fma2(zz, f2(c), f2(-Mz)), b = fma2(tt2, f2(c), f2(-Mt));
                                 const float2 ez = make_float2(ex2(a.x), ex2(a.y));
+                                const float2 et = make_float2(ex2(b.x), ex2(b.y));
                                 Ez2 = add2(Ez2, ez);
-                                Et2 = add2(Et2, make_float2(ex2(b.x), ex2(b.y)));
-                                X2 = fma2(ez, sub2(sub2(zz, gz2), sub2(tt2, tp2)), X2);
+                                Et2 = add2(Et2, et);
+                                if constexpr (kRkl) X2 = fma2(ez, sub2(sub2(zz, gz2), sub2(tt2, tp2)), X2);
+                                else X2 = fma2(et, sub2(tt2, zz), X2);
                             }
                         }
                     });
@@ -1289,7 +1306,7 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                 const int wf = warp_or((ninf ? kTmNinf : 0) | (rinf ? kTmRklInf : 0));
                 const float4 v2 = make_float4(warp_sum(Ez2.x + Ez2.y), warp_sum(Et2.x + Et2.y),
                                               warp_sum(X2.x + X2.y), __int_as_float(wf));
-                // -> (loss, cv, K, flags)
+                // -> (loss, cv, K, flags); FKL (loss, cv, cu, flags)
                 const float4 r2v = exchange(v2, make_float4(0.f, 0.f, 0.f, 0.f), &pbar2, recv2,
                     [&](float4 x) {
                         return make_float4(warp_sum(x.x), warp_sum(x.y), warp_sum(x.z),
@@ -1299,6 +1316,9 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                         const float Ez = m.x, Et = m.y, X = m.z;
                         const float dz = fold_err(gz), dt = fold_err(gt);
                         const float lr = logf(Ez / Et) - kLn2 * (dz - dt);
+                        if constexpr (kFkl)
+                            return make_float4((X / Et - (gt - gz)) * inv_tau + lr, -log2_sum(Ez) + dz,
+                                               -log2_sum(Et) + dt, m.w);
                         const float l = (__float_as_int(m.w) & kTmRklInf) ? __builtin_huge_valf()
                                                                           : (X / Ez + (gt - tp)) * inv_tau - lr;
                         return make_float4(l, -log2_sum(Ez) + dz, X / Ez * inv_tau, m.w);
@@ -1306,7 +1326,8 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                 row_err = failed;
                 loss = r2v.x;
                 cv = r2v.y;
-                K = r2v.z;
+                if constexpr (kFkl) cu = r2v.z;
+                else K = r2v.z;
                 flags = __float_as_int(r2v.w);
             }
         }
@@ -1343,14 +1364,15 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
         } else {
             // JSD: q (log2(q/m) - S), every probability carrying the gradient's factor,
             // which cancels in log2(q/m); RKL: q ((z - gz) - (t - tp) - X / E) / tau^2,
-            // q carrying 1 / tau, and 0 where q = 0 meets an infinite log-ratio
+            // q carrying 1 / tau, and 0 where q = 0 meets an infinite log-ratio; FKL:
+            // q - p, both carrying 1 / tau
             const float2 cvs = f2(cv + p.lg_scale), cus = f2(cu + p.lg_scale);
             const bool has_ninf = (flags & kTmNinf) != 0;
             sweep_tm<In, false, false, false, false, false, kJsd ? kTmJsdG : kTmG>(tw, tsh, nv, tail, tz, tt,
                 [&](const float* z, const float* t, auto tag, int j0, float, float, bool, uint4& zr, uint4& tr) {
                     constexpr int kCnt = decltype(tag)::value;
                     // RKL's bf16 chunks take x - m from the packed words (mixed-precision subtracts)
-                    constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && kRkl;
+                    constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && kMom;
                     const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw4[4] = {tr.x, tr.y, tr.z, tr.w};
                     auto zdiff = [&](int e, float m) {
                         if constexpr (kRaw) return bf16x2_minus(zw[e / 2], m);
@@ -1374,6 +1396,9 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                                 if (!(qj.x > 0.f)) gg.x = 0.f;
                                 if (!(qj.y > 0.f)) gg.y = 0.f;
                             }
+                        } else if constexpr (kFkl) {  // (q - p) / tau
+                            const float2 u = fma2(tdiff(e, gt), f2(c), cus);
+                            gg = sub2(qj, make_float2(ex2(u.x), ex2(u.y)));
                         } else if (jsd_trivial) {
                             gg = f2(0.f);
                         } else {
@@ -1415,9 +1440,30 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
 }
 
 // ------------------------------------------------------------------ host
+// Clusters of more than 8 CTAs need the kernel's non-portable opt-in, set once
+// per kernel and device (a function attribute of this process, no device setting).
+template <auto kern>
+static cudaError_t allow_wide_clusters() {
+    static std::atomic<int> done[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidValue;
+    if (!done[dev].load(std::memory_order_relaxed)) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return e;
+        done[dev].store(1, std::memory_order_relaxed);
+    }
+    return cudaSuccess;
+}
+
 template <typename In, int kKind, bool kAligned, int kT>
 static cudaError_t launch_distill_kind(const DistParams& dp, long long rows, size_t smem, cudaStream_t s) {
     auto kern = distill_kernel<In, kKind, kAligned, kT>;
+    if (dp.csize > 8) {
+        const cudaError_t e = allow_wide_clusters<distill_kernel<In, kKind, kAligned, kT>>();
+        if (e != cudaSuccess) return e;
+    }
     if (smem > 48 * 1024) {
         // the opt-in is per device and kernel; set it once, so that later calls
         // (including ones under stream capture) make no attribute call
@@ -1473,8 +1519,14 @@ static cudaError_t launch_distill_dtype(osd_loss kind, const DistParams& dp, lon
 struct TmLaunch {
     TmShape shape;
     size_t smem;
-    int occ;  // resident CTAs an SM
+    int occ;       // resident CTAs an SM
+    int clusters;  // resident clusters of csize CTAs on the GPU
 };
+// An empty kernel with the TMEM-staged runs' block size and bound on resident
+// CTAs.  The cluster occupancy query counts, on it, how many clusters the GPU's
+// processing clusters hold at once for a given shared-memory request, which the
+// query cannot do on the TMEM kernel itself.  It is never launched.
+__global__ void __launch_bounds__(kTmThreads, 7) tm_cluster_probe() {}
 template <typename In, int kKind>
 static cudaError_t tm_launch_shape(int span, int csize, TmLaunch* out) {
     constexpr int kVec = Elem<In>::kVec;
@@ -1488,7 +1540,7 @@ static cudaError_t tm_launch_shape(int span, int csize, TmLaunch* out) {
     struct Entry {
         int dev, span, csize;
         size_t smem;
-        int occ;
+        int occ, clusters;
     };
     static std::mutex mu;
     static Entry cache[64];
@@ -1500,9 +1552,10 @@ static cudaError_t tm_launch_shape(int span, int csize, TmLaunch* out) {
         std::lock_guard<std::mutex> lock(mu);
         for (int i = 0; i < n_cache; ++i)
             if (cache[i].dev == dev && cache[i].span == span && cache[i].csize == csize) {
-                out->shape = TmShape{slots, t_off, ncols, 0, 0, 0, 0};
+                out->shape = TmShape{slots, t_off, ncols, 0, 0, 0, 0, 0};
                 out->smem = cache[i].smem;
                 out->occ = cache[i].occ;
+                out->clusters = cache[i].clusters;
                 return cudaSuccess;
             }
     }
@@ -1529,21 +1582,75 @@ static cudaError_t tm_launch_shape(int span, int csize, TmLaunch* out) {
             allowed[dev] = static_cast<int>(smem);
         }
     }
-    int occ = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, kern, kTmThreads, smem);
+    // Resident CTAs an SM, from the kernel's limits: the occupancy query reports one
+    // CTA an SM for this kernel (it allocates tensor memory) whatever the
+    // resources asked for, while ncu shows seven resident at 32 KB spans
+    cudaFuncAttributes fa;
+    e = cudaFuncGetAttributes(&fa, kern);
     if (e != cudaSuccess) return e;
-    if (occ < 1 || occ * static_cast<int>(ncols) > 512) return cudaErrorInvalidValue;
+    int reserved = 0, regs_sm = 0, blocks_sm = 0, threads_sm = 0;
+    if ((e = cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&regs_sm, cudaDevAttrMaxRegistersPerMultiprocessor, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&blocks_sm, cudaDevAttrMaxBlocksPerMultiprocessor, dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&threads_sm, cudaDevAttrMaxThreadsPerMultiProcessor, dev)) != cudaSuccess)
+        return e;
+    const int regs_warp = (fa.numRegs * 32 + 255) / 256 * 256;  // allocated per warp in units of 256
+    int occ = std::min(blocks_sm, threads_sm / kTmThreads);
+    occ = std::min(occ, static_cast<int>(size_t(smem_sm) / (smem + fa.sharedSizeBytes + size_t(reserved))));
+    occ = std::min(occ, regs_sm / (regs_warp * (kTmThreads / 32)));
+    occ = std::min(occ, static_cast<int>(512 / ncols));
+    if (occ < 1) return cudaErrorInvalidValue;
+    // resident clusters: the probe with this launch's shared memory (static included),
+    // bounded by the SM count x occ / csize
+    int clusters = std::max(1, device_sms() * occ / csize);
+    {
+        const size_t probe_smem = smem + fa.sharedSizeBytes;
+        static int probe_allowed[64] = {};
+        static bool probe_wide[64] = {};
+        std::lock_guard<std::mutex> lock(mu);
+        if (probe_allowed[dev] < static_cast<int>(probe_smem)) {
+            e = cudaFuncSetAttribute(tm_cluster_probe, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     static_cast<int>(probe_smem));
+            if (e != cudaSuccess) return e;
+            probe_allowed[dev] = static_cast<int>(probe_smem);
+        }
+        if (csize > 8 && !probe_wide[dev]) {
+            e = cudaFuncSetAttribute(tm_cluster_probe, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+            if (e != cudaSuccess) return e;
+            probe_wide[dev] = true;
+        }
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(static_cast<unsigned>(csize));
+        cfg.blockDim = dim3(kTmThreads);
+        cfg.dynamicSmemBytes = probe_smem;
+        cudaLaunchAttribute attr;
+        attr.id = cudaLaunchAttributeClusterDimension;
+        attr.val.clusterDim.x = static_cast<unsigned>(csize);
+        attr.val.clusterDim.y = 1;
+        attr.val.clusterDim.z = 1;
+        cfg.attrs = &attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        e = cudaOccupancyMaxActiveClusters(&n, tm_cluster_probe, &cfg);
+        if (e != cudaSuccess) return e;
+        if (n >= 1) clusters = std::min(clusters, n);
+    }
     {
         std::lock_guard<std::mutex> lock(mu);
-        if (n_cache < 64) cache[n_cache++] = Entry{dev, span, csize, smem, occ};
+        if (n_cache < 64) cache[n_cache++] = Entry{dev, span, csize, smem, occ, clusters};
     }
-    out->shape = TmShape{slots, t_off, ncols, 0, 0, 0, 0};
+    out->shape = TmShape{slots, t_off, ncols, 0, 0, 0, 0, 0};
     out->smem = smem;
     out->occ = occ;
+    out->clusters = clusters;
     return cudaSuccess;
 }
 template <typename In, int kKind>
 static cudaError_t launch_distill_tm(const DistParams& dp, long long rows, cudaStream_t s) {
+    if (dp.csize > 8) {
+        const cudaError_t e = allow_wide_clusters<distill_tm_kernel<In, kKind>>();
+        if (e != cudaSuccess) return e;
+    }
     TmLaunch tl;
     const cudaError_t e = tm_launch_shape<In, kKind>(dp.span, dp.csize, &tl);
     if (e != cudaSuccess) return e;
@@ -1551,22 +1658,28 @@ static cudaError_t launch_distill_tm(const DistParams& dp, long long rows, cudaS
     // the last rows, in runs of 2 and then of 1, even out the clusters' finishing
     // times (K = the clusters resident at once: the last K rows singly, the 2K
     // before them in pairs).  With runs of 8 throughout, 6554 rows over about 228
-    // resident clusters left some clusters 32 rows and others 24.
-    const long long K = std::max<long long>(1, static_cast<long long>(device_sms()) * tl.occ / dp.csize);
+    // resident clusters left some clusters 32 rows and others 24.  The long runs
+    // are 8 rows from 16 K rows on, 4 from 8 K, else 2: with few rows per cluster
+    // more, shorter runs did better than one wave of long ones (256 rows of 128256
+    // over 47 resident 16-CTA clusters: runs of 2, 67.6 us; one wave of runs of 6,
+    // 71.7 us), the 16 CTAs of a row waiting on each other twice a row.
+    const long long K = tl.clusters;
     const long long ones = std::min(rows, K);
     const long long twos = std::min(rows - ones, 2 * K);
     TmShape sh = tl.shape;
+    sh.run = rows >= 16 * K ? kTmRows : (rows >= 8 * K ? 4 : 2);
     sh.end2 = rows - ones;
     sh.end8 = sh.end2 - twos;
-    sh.n8 = static_cast<int>((sh.end8 + kTmRows - 1) / kTmRows);
+    sh.n8 = static_cast<int>((sh.end8 + sh.run - 1) / sh.run);
     sh.n2 = static_cast<int>((twos + 1) / 2);
     const long long runs = sh.n8 + sh.n2 + ones;
-    return launch(distill_tm_kernel<In, kKind>, dim3(static_cast<unsigned>(runs * dp.csize)), dim3(kTmThreads),
-                  tl.smem, s, dp.csize, dp, sh);
+    return launch(distill_tm_kernel<In, kKind>, dim3(static_cast<unsigned>(runs * dp.csize)),
+                  dim3(kTmThreads), tl.smem, s, dp.csize, dp, sh);
 }
 template <typename In>
 static cudaError_t launch_distill_tm_kind(osd_loss kind, const DistParams& dp, long long rows, cudaStream_t s) {
     switch (kind) {
+        case OSD_FKL: return launch_distill_tm<In, OSD_FKL>(dp, rows, s);
         case OSD_JSD: return launch_distill_tm<In, OSD_JSD>(dp, rows, s);
         case OSD_RKL: return launch_distill_tm<In, OSD_RKL>(dp, rows, s);
         default: return launch_distill_tm<In, OSD_TVD>(dp, rows, s);
@@ -1593,11 +1706,14 @@ static osd_status distill_run(const void* draft_logits, const void* target_logit
                          aligned_to(dlogits, 16) && (size_t(V) * 4) % 16 == 0 &&
                          row_ok(d_stride_g, G) && row_ok(d_stride_p, p_rows) && row_ok(t_stride_g, G) &&
                          row_ok(t_stride_p, p_rows);
-    // the TMEM-staged runs (if the span fits) for TVD, JSD and RKL, where they
-    // measured faster: TVD 94.7 % against 70.1 % of the HBM peak, JSD 71.6 % against
-    // 63.0 %, RKL 95.1 % against 86.4 % (65536 x 32000 bf16); FKL and CE, at 90.9 %
-    // and 96.3 % on the per-row kernel, measured slower on an earlier form of them
-    const bool tm_path = aligned && !accepted && (kind == OSD_TVD || kind == OSD_JSD || (kTmRkl && kind == OSD_RKL));
+    // the TMEM-staged runs (if the span fits) for TVD, JSD, RKL and FKL, where they
+    // measured faster: TVD 95.1 % against 70.1 % of the HBM peak, JSD 71.9 % against
+    // 63.0 %, RKL 95.5 % against 86.4 %, FKL 100.6 % against 90.9 % of the measured
+    // copy bandwidth (65536 x 32000 bf16); CE stays at 96.3 % on the per-row kernel.
+    // Rows chosen by verification stay on the per-row kernel: on the runs, 32 rows
+    // of 32000 took 12.8 against 10.4 us, and 256 of 128256 no less time
+    const bool tm_path = aligned && !accepted &&
+                         (kind == OSD_TVD || kind == OSD_JSD || (kTmRkl && kind == OSD_RKL) || kind == OSD_FKL);
     int csize = 1, span = V;
     // JSD, with the most work per entry, stages best in longer spans on the per-row
     // kernel; the TMEM-staged runs take the 32 KB spans for every kind.  (At
@@ -1609,6 +1725,14 @@ static osd_status distill_run(const void* draft_logits, const void* target_logit
     // (measured 6-12 % less latency at 4 and 128 rows of 32000)
     if (static_cast<long long>(G) * P <= device_sms()) span_bytes /= 2;
     if (!row_span_shape(V, es, span_bytes, kDistMaxCluster, kDistMaxSmem, &csize, &span))
+        return OSD_ERR_UNSUPPORTED;
+    // on the TMEM-staged runs, rows that need more than 8 spans of the target size
+    // take up to 16 CTAs: spans that fit 64 columns of tensor memory and six CTAs
+    // an SM instead of 128 columns and two (2048 x 128256 bf16: FKL 77.7 against
+    // 75.6 %, RKL 71.5 against 67.9 %, TVD 71.8 against 65.0 %, JSD 55.3 against
+    // 54.3 %); the per-row kernel keeps at most 8 (measured no faster)
+    if (tm_path && csize == kDistMaxCluster && size_t(span) * 2 * es > span_bytes &&
+        !row_span_shape(V, es, span_bytes, kDistMaxClusterWide, kDistMaxSmem, &csize, &span))
         return OSD_ERR_UNSUPPORTED;
     const long long rows = static_cast<long long>(G) * P;
     if (rows * csize > INT_MAX) return OSD_ERR_UNSUPPORTED;

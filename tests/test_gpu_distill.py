@@ -274,3 +274,58 @@ def test_single_row_ragged_tail(osd, kind, V):
         lr, gr = _oracle(z, t, None, kind, 0.4, tau=tau)
         skip = _tvd_ambiguous(z, t, tau) if kind == "tvd" else None
         check_distill(lg, gg, lr, gr, np.ones(1, bool), skip)
+
+
+MASK_PATTERNS = ["random40", "none", "all", "last_only", "first_and_last"]
+
+
+@pytest.mark.parametrize("kind", ["rkl", "jsd", "tvd"])
+@pytest.mark.parametrize("pattern", MASK_PATTERNS)
+def test_masked_rows_every_pattern(osd, kind, pattern):
+    """Masked launches on the TMEM-staged runs of rows: every active row must match
+    the oracle and every masked-out row keep loss 0 and its untouched gradient,
+    for 1003 rows (runs of 8, pairs and single rows, the last run ragged) with
+    40 %, none, all, only the last, or only the first and last rows active."""
+    N, V = 1003, 4000
+    spec = W.DistillSpec(N, V, torch.bfloat16, 2.0, "draft+noise", 1.5, 1.0)
+    inp = W.distill_inputs(spec, seed=501)
+    z, t = inp["draft"], inp["target"]
+    mask = torch.zeros(N, dtype=torch.uint8)
+    if pattern == "random40":
+        g = torch.Generator().manual_seed(502)
+        mask[torch.randperm(N, generator=g)[: round(0.4 * N)]] = 1
+    elif pattern == "all":
+        mask[:] = 1
+    elif pattern == "last_only":
+        mask[-1] = 1
+    elif pattern == "first_and_last":
+        mask[0] = 1
+        mask[-1] = 1
+    lg, gg = _run(osd, z, t, mask, kind, 0.5)
+    lr, gr = _oracle(z, t, mask, kind, 0.5)
+    skip = _tvd_ambiguous(z, t) if kind == "tvd" else None
+    rep = check_distill(lg, gg, lr, gr, mask.numpy() == 1, skip)
+    print(f"{kind} {pattern}: {rep}")
+
+
+@pytest.mark.parametrize("kind", ["rkl", "jsd", "tvd"])
+def test_masked_rows_unaligned_mask_and_few_rows(osd, kind):
+    """A mask view that starts off a 16-byte boundary, and launches with fewer
+    rows than resident clusters (each row a run of its own), masked or not."""
+    dev = torch.device("cuda")
+    for N, off in ((300, 1), (5, 0), (5, 3)):
+        spec = W.DistillSpec(N, 4000, torch.bfloat16, 2.0, "draft+noise", 1.5, 1.0)
+        inp = W.distill_inputs(spec, seed=600 + N + off)
+        z, t = inp["draft"], inp["target"]
+        g = torch.Generator().manual_seed(601 + N)
+        mask = (torch.rand(N, generator=g) < 0.5).to(torch.uint8)
+        mask[0] = 1
+        big = torch.zeros(N + 16, dtype=torch.uint8, device=dev)
+        big[off:off + N] = mask.to(dev)
+        md = big[off:off + N]
+        dl = torch.full((N, 4000), float("nan"), dtype=torch.float32, device=dev)
+        loss, gg = osd.osd_distill(z.to(dev), t.to(dev), md, kind, 0.5, dlogits=dl)
+        torch.cuda.synchronize()
+        lr, gr = _oracle(z, t, mask, kind, 0.5)
+        skip = _tvd_ambiguous(z, t) if kind == "tvd" else None
+        check_distill(loss.cpu().numpy(), gg.cpu().numpy(), lr, gr, mask.numpy() == 1, skip)
