@@ -75,8 +75,15 @@ def test_verify_matches_oracle(osd, B, k, V, dtype, T):
     print(f"B={B} k={k} V={V} {dtype} T={T}: {rep}")
 
 
-@pytest.mark.parametrize("B,k,V,dtype", [(16, 3, 1, torch.float32), (32, 4, 1001, torch.bfloat16),
-                                         (12, 5, 32000, torch.bfloat16), (9, 2, 40000, torch.float32)])
+GREEDY_CASES = [
+    (16, 3, 1, torch.float32), (32, 4, 1001, torch.bfloat16), (9, 2, 40000, torch.float32),
+    (12, 5, 32000, torch.bfloat16), (38, 7, 32768, torch.bfloat16), (7, 3, 4096, torch.bfloat16),
+    (5, 1, 40, torch.float32), (20, 5, 16000, torch.float32), (39, 7, 32768, torch.bfloat16),
+    (4, 8, 32000, torch.bfloat16),
+]
+
+
+@pytest.mark.parametrize("B,k,V,dtype", GREEDY_CASES)
 def test_greedy_matches_oracle(osd, B, k, V, dtype):
     spec = W.VerifySpec(B, k, V, dtype, 2.0, 1.0, 0.3, 0.0)
     inp = W.verify_inputs(spec, seed=99 + V)
@@ -93,6 +100,18 @@ def test_greedy_matches_oracle(osd, B, k, V, dtype):
     dev = torch.device("cuda")
     res2 = osd.osd_verify(None, inp["target"].to(dev), inp["greedy_tokens"].to(dev), None, 0.0)
     assert torch.equal(res2.out_tokens, res.out_tokens)
+    # draft tokens outside [0, V) mark their sequence bad; the others are unaffected
+    if B >= 3:
+        bad = inp["greedy_tokens"].clone()
+        bad[1, 0] = V
+        bad[2, k - 1] = -1
+        res3 = osd.osd_verify(None, inp["target"].to(dev), bad.to(dev), None, 0.0)
+        torch.cuda.synchronize()
+        ref3 = oracle.verify(inp["draft"], inp["target"], bad, inp["uniforms"], 0.0)
+        np.testing.assert_array_equal(res3.accepted.cpu().numpy(), ref3["accepted"])
+        np.testing.assert_array_equal(res3.out_tokens.cpu().numpy(), ref3["out_tokens"])
+        np.testing.assert_array_equal(res3.mismatch_mask.cpu().numpy(), ref3["mismatch_mask"])
+        assert res3.accepted[1].item() == -1 and res3.accepted[2].item() == -1
 
 
 @pytest.mark.parametrize("B,V", [(16, 5000), (160, 8192)])
