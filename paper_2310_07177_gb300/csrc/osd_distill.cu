@@ -256,11 +256,23 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
     const int rank = (csize > 1) ? static_cast<int>(cluster_rank()) : 0;
     long long row = blockIdx.x / csize;  // the launch row; from here on, the output row
     long long g, pp;
+    const int V = p.V;
+    const int e0 = rank * p.span;
+    const int n = min(p.span, V - e0);
+    In* zs = reinterpret_cast<In*>(dsm);
+    In* ts = zs + p.span;
+    bool issued = false;  // accepted mode: the span's copies went out before the slot count
     if (p.accepted) {
         // sequence b = row keeps position a = accepted[b] when a < k (the first rejected
         // draft token); the output slot counts the active sequences before it
         const int b = static_cast<int>(row), a = p.accepted[b];
         const bool active = a >= 0 && a < p.k;
+        if (active) {  // the copies first: the count below runs while they are in flight
+            stage_span_issue<In, kAligned>(zs, ts, static_cast<const In*>(p.draft) + b * p.dsg + a * p.dsp + e0,
+                                           static_cast<const In*>(p.target) + b * p.tsg + a * p.tsp + e0, n,
+                                           &bar, &s_err);
+            issued = true;
+        }
         int2 cnt = make_int2(0, 0);  // (active before b, active in total)
         for (int i = tid; i < p.G; i += kT) {
             const int ai = p.accepted[i];
@@ -292,14 +304,10 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
     }
     const In* zrow = static_cast<const In*>(p.draft) + g * p.dsg + pp * p.dsp;
     const In* trow = static_cast<const In*>(p.target) + g * p.tsg + pp * p.tsp;
-    const int V = p.V;
-    const int e0 = rank * p.span;
-    const int n = min(p.span, V - e0);
-    In* zs = reinterpret_cast<In*>(dsm);
-    In* ts = zs + p.span;
 
     // ---- stage the span of both rows in shared memory
-    const int err_local = stage_span<In, kAligned, kT>(zs, ts, zrow + e0, trow + e0, n, &bar, &s_err);
+    const int err_local = issued ? stage_span_land<In, kAligned, kT>(zs, ts, zrow + e0, trow + e0, n, &bar, &s_err)
+                                 : stage_span<In, kAligned, kT>(zs, ts, zrow + e0, trow + e0, n, &bar, &s_err);
 
     // ---- pass 0: this thread's maxima, and the chunk where each first appears
     float mz = kNegInf, mt = kNegInf;

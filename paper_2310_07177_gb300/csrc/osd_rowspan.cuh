@@ -61,6 +61,43 @@ __device__ __forceinline__ int stage_span(In* zs, In* ts, const In* zsrc, const 
     return *s_err;
 }
 
+// stage_span in two halves, for a caller with other work to do while the copies
+// fly: stage_span_issue (thread 0 initialises `bar` and issues the bulk copies;
+// a block barrier must come before any other thread waits on `bar`), then
+// stage_span_land (the ragged tail by plain loads, the bounded wait, a block
+// barrier; returns non-zero, for every thread, when the wait gave up).
+template <typename In, bool kAligned>
+__device__ __forceinline__ void stage_span_issue(In* zs, In* ts, const In* zsrc, const In* tsrc, int n,
+                                                 uint64_t* bar, int* s_err) {
+    if (threadIdx.x == 0) *s_err = 0;
+    if constexpr (kAligned) {
+        const uint32_t bytes = static_cast<uint32_t>(n * sizeof(In)) & ~15u;
+        if (threadIdx.x == 0 && bytes) {
+            mbar_init(bar, 1);
+            mbar_arrive_expect_tx(bar, 2 * bytes);
+            bulk_g2s(zs, zsrc, bytes, bar);
+            bulk_g2s(ts, tsrc, bytes, bar);
+        }
+    }
+}
+template <typename In, bool kAligned, int kT = kRowThreads>
+__device__ __forceinline__ int stage_span_land(In* zs, In* ts, const In* zsrc, const In* tsrc, int n, uint64_t* bar,
+                                               int* s_err) {
+    const int tid = threadIdx.x;
+    const uint32_t bytes = kAligned ? (static_cast<uint32_t>(n * sizeof(In)) & ~15u) : 0u;
+    const int nb = static_cast<int>(bytes / sizeof(In));
+    for (int e = nb + tid; e < n; e += kT) {
+        copy_raw(zs + e, zsrc + e);
+        copy_raw(ts + e, tsrc + e);
+    }
+    if (bytes && !mbar_wait_bounded(bar, 0, kStageWaitNs)) {
+        atomicOr(s_err, 1);
+        mbar_wait_bounded(bar, 0, kStageWaitNs);  // give copies in flight a last chance to land
+    }
+    __syncthreads();
+    return *s_err;
+}
+
 // Visit this thread's entries of a staged span in chunks of one 16-byte vector
 // (or single entries on the element-wise path).  Clamping (to -1e30, see Elem)
 // happens on the packed words.  f(z[], t[], count_tag, j0, zmax, tmax, ninf,
