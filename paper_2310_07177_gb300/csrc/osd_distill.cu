@@ -743,8 +743,7 @@ constexpr int kTmThreads = 128;  // one warp per tensor-memory lane quarter
 constexpr int kTmG = 2;          // chunk slots per round of tensor-memory loads
 constexpr int kTmRows = 8;       // rows per cluster run
 constexpr int kTmJsdG = 1;       // JSD's passes 2 and 3: one chunk slot per round (no spills at 72 registers)
-constexpr bool kTmRkl = true;     // RKL on these runs too
-constexpr int kTmRklG = 1;       // RKL pass 1: one chunk slot per round (no spills at 72 registers)
+constexpr int kTmMomG = 1;       // RKL and FKL pass 1: one chunk slot per round (no spills at 72 registers)
 constexpr int kTmMaxChunks = 4096;  // 16-byte chunks per span (<= 256 columns; longer spans stage as above)
 
 struct TmShape {
@@ -1276,7 +1275,7 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                 bool ninf = false, rinf = false;
                 const float Mz = gz == kNegInf ? 0.f : __fmul_rn(gz, c), Mt = gt == kNegInf ? 0.f : __fmul_rn(gt, c);
                 const float2 gz2 = f2(gz), tp2 = f2(tp);
-                sweep_tm<In, false, false, false, true, false, kTmRklG>(tw, tsh, nv, tail, tz, tt,
+                sweep_tm<In, false, false, false, true, false, kTmMomG>(tw, tsh, nv, tail, tz, tt,
                     [&](const float* z, const float* t, auto tag, int, float, float, bool cninf, uint4&, uint4&) {
                         constexpr int kCnt = decltype(tag)::value;
                         if (kCnt == 1 || cninf) {  // element-wise, with the guards a -inf needs
@@ -1721,7 +1720,7 @@ static osd_status distill_run(const void* draft_logits, const void* target_logit
     // Rows chosen by verification stay on the per-row kernel: on the runs, 32 rows
     // of 32000 took 12.8 against 10.4 us, and 256 of 128256 no less time
     const bool tm_path = aligned && !accepted &&
-                         (kind == OSD_TVD || kind == OSD_JSD || (kTmRkl && kind == OSD_RKL) || kind == OSD_FKL);
+                         (kind == OSD_TVD || kind == OSD_JSD || kind == OSD_RKL || kind == OSD_FKL);
     int csize = 1, span = V;
     // JSD, with the most work per entry, stages best in longer spans on the per-row
     // kernel; the TMEM-staged runs take the 32 KB spans for every kind.  (At
