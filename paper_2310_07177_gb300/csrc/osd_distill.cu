@@ -1093,15 +1093,24 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
         // ---- pass 0: this warp's maxima (JSD: clamped logits kept; RKL: with the
         // target logit at the draft maximum)
         float mz = kNegInf, mt = kNegInf, tp = kNegInf;
+        // RKL: the raw words of the chunk that first raised this thread's draft maximum
+        // (or the tail entry's target logit), scanned for the pivot once the pass is done
+        [[maybe_unused]] uint4 pz = make_uint4(0u, 0u, 0u, 0u), pt = pz;
+        [[maybe_unused]] bool piv_tail = false;
         sweep_tm<In, kJsd, kJsd, true, false, kJsd>(tw, tsh, nv, tail, tz, tt,
-            [&](const float* z, const float* t, auto tag, int, float cz, float ct, bool, uint4&, uint4&) {
+            [&](const float*, const float* t, auto tag, int, float cz, float ct, bool, uint4& zr, uint4& tr) {
                 if constexpr (kRkl) {
                     constexpr int kCnt = decltype(tag)::value;
                     if (cz > mz) {
                         mz = cz;
-#pragma unroll
-                        for (int e = kCnt - 1; e >= 0; --e)
-                            if (z[e] == cz) tp = t[e];
+                        if constexpr (kCnt == 1) {
+                            piv_tail = true;
+                            tp = t[0];
+                        } else {
+                            piv_tail = false;
+                            pz = zr;
+                            pt = tr;
+                        }
                     }
                 } else {
                     mz = fmaxf(mz, cz);
@@ -1109,6 +1118,14 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                 mt = fmaxf(mt, ct);
             });
         if constexpr (kRkl) {
+            if (!piv_tail && mz != kNegInf) {  // the first entry of the saved chunk that holds mz
+                float z[kVec], t[kVec];
+                Elem<In>::unpack(pz, z);
+                Elem<In>::unpack(pt, t);
+#pragma unroll
+                for (int e = kVec - 1; e >= 0; --e)
+                    if (z[e] == mz) tp = t[e];
+            }
             const float2 pv = warp_max_pivot(mz, tp);
             mz = pv.x;
             tp = pv.y;
