@@ -1146,8 +1146,12 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
             float2 Ez2 = f2(0.f), Et2 = f2(0.f);
             const float Mz = mz == kNegInf ? 0.f : __fmul_rn(mz, c), Mt = mt == kNegInf ? 0.f : __fmul_rn(mt, c);
             sweep_tm<In, false, false, false, false, false>(tw, tsh, nv, tail, tz, tt,
-                [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4&, uint4&) {
+                [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4& zr, uint4& tr) {
                     constexpr int kCnt = decltype(tag)::value;
+                    // JSD's bf16 chunks take x - m straight from the packed words (the
+                    // mixed-precision subtract, exact here as the unpacked one is)
+                    constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && kJsd;
+                    const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw4[4] = {tr.x, tr.y, tr.z, tr.w};
                     if constexpr (kCnt == 1) {
                         Ez2.x += kFold ? ex2(fmaf(z[0], c, -Mz)) : ex2((z[0] - mz) * c);
                         Et2.x += kFold ? ex2(fmaf(t[0], c, -Mt)) : ex2((t[0] - mt) * c);
@@ -1155,8 +1159,14 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
 #pragma unroll
                         for (int e = 0; e < kCnt; e += 2) {
                             const float2 zz = make_float2(z[e], z[e + 1]), tt2 = make_float2(t[e], t[e + 1]);
-                            const float2 a = kFold ? fma2(zz, f2(c), f2(-Mz)) : mul2(sub2(zz, f2(mz)), f2(c));
-                            const float2 b = kFold ? fma2(tt2, f2(c), f2(-Mt)) : mul2(sub2(tt2, f2(mt)), f2(c));
+                            float2 a, b;
+                            if constexpr (kRaw) {
+                                a = mul2(bf16x2_minus(zw[e / 2], mz), f2(c));
+                                b = mul2(bf16x2_minus(tw4[e / 2], mt), f2(c));
+                            } else {
+                                a = kFold ? fma2(zz, f2(c), f2(-Mz)) : mul2(sub2(zz, f2(mz)), f2(c));
+                                b = kFold ? fma2(tt2, f2(c), f2(-Mt)) : mul2(sub2(tt2, f2(mt)), f2(c));
+                            }
                             Ez2 = add2(Ez2, make_float2(ex2(a.x), ex2(a.y)));
                             Et2 = add2(Et2, make_float2(ex2(b.x), ex2(b.y)));
                         }
@@ -1199,7 +1209,7 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                     sweep_tm<In, false, false, false, false, kTvd, kJsd ? kTmJsdG : kTmG>(tw, tsh, nv, tail, tz, tt,
                         [&](const float* z, const float* t, auto tag, int, float, float, bool, uint4& zr, uint4& tr) {
                             constexpr int kCnt = decltype(tag)::value;
-                            constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && kTvd;
+                            constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8;
                             const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw4[4] = {tr.x, tr.y, tr.z, tr.w};
                             [[maybe_unused]] float qs[kCnt];
 #pragma unroll
@@ -1396,7 +1406,7 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                 [&](const float* z, const float* t, auto tag, int j0, float, float, bool, uint4& zr, uint4& tr) {
                     constexpr int kCnt = decltype(tag)::value;
                     // RKL's bf16 chunks take x - m from the packed words (mixed-precision subtracts)
-                    constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8 && kMom;
+                    constexpr bool kRaw = sizeof(In) == 2 && kCnt == 8;
                     const uint32_t zw[4] = {zr.x, zr.y, zr.z, zr.w}, tw4[4] = {tr.x, tr.y, tr.z, tr.w};
                     auto zdiff = [&](int e, float m) {
                         if constexpr (kRaw) return bf16x2_minus(zw[e / 2], m);
