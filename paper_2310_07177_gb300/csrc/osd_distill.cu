@@ -913,6 +913,10 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
     constexpr bool kJsd = kKind == OSD_JSD, kTvd = kKind == OSD_TVD, kRkl = kKind == OSD_RKL;
     constexpr bool kFkl = kKind == OSD_FKL;
     constexpr bool kMom = kRkl || kFkl;  // the maxima go round first, then the sums with the loss moment
+    // pass 0 (the maxima) taken while the span moves into tensor memory (JSD and FKL:
+    // 3.6 and 1.6 % faster) or as a sweep of its own after the next row's copy is
+    // issued (RKL and TVD: 1.9 and 2.5 % faster that way)
+    constexpr bool kStage0 = kJsd || kFkl;
     // TVD, RKL: exponent arguments x c - m c as one fma; JSD: logits clamped to -1e30, (x - m) c
     constexpr bool kFold = !kJsd;
     extern __shared__ __align__(128) unsigned char dsm[];
@@ -1061,9 +1065,14 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
             if (rank == 0 && tid == 0) p.loss[row] = __int_as_float(0x7fc00000);
             continue;
         }
-        // ---- this row's span: shared memory (bounded wait) -> tensor memory
+        // ---- this row's span: shared memory (bounded wait) -> tensor memory; JSD and
+        // FKL take pass 0 on the way: this thread's maxima (JSD clamps the logits
+        // first, and tensor memory keeps the clamped words)
         const bool landed = !bytes || mbar_wait_bounded(&bar, phase, kStageWaitNs);
         if (tid == 0 && landed) pending = false;
+        float mz = kNegInf, mt = kNegInf, tp = kNegInf;
+        [[maybe_unused]] uint4 pz = make_uint4(0u, 0u, 0u, 0u), pt = pz;
+        [[maybe_unused]] bool piv_tail = false;
         for (int s0 = 0; s0 < tsh.slots; s0 += kTmG) {
             uint4 zr[kTmG], tr[kTmG];
 #pragma unroll
@@ -1071,6 +1080,14 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                 const int v = tid + kT * (s0 + g);
                 zr[g] = (v < nv) ? lds_v4(zs + v * kVec) : make_uint4(0u, 0u, 0u, 0u);
                 tr[g] = (v < nv) ? lds_v4(ts + v * kVec) : make_uint4(0u, 0u, 0u, 0u);
+                if (kStage0 && v < nv) {
+                    if constexpr (kJsd) {
+                        Elem<In>::clamp_raw(zr[g]);
+                        Elem<In>::clamp_raw(tr[g]);
+                    }
+                    mz = fmaxf(mz, Elem<In>::max_raw(zr[g]));
+                    mt = fmaxf(mt, Elem<In>::max_raw(tr[g]));
+                }
             }
             tm_st8(tw + 4 * s0, zr[0], zr[1]);
             tm_st8(tw + tsh.t_off + 4 * s0, tr[0], tr[1]);
@@ -1078,6 +1095,14 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
         tm_wait_st();
         tz = nz;
         tt = nt;
+        if (kStage0 && tid < tail) {  // the ragged tail entry, last, as a chunk of one
+            if constexpr (kJsd) {
+                tz = Elem<In>::clamp1(tz);
+                tt = Elem<In>::clamp1(tt);
+            }
+            mz = fmaxf(mz, tz);
+            mt = fmaxf(mt, tt);
+        }
         __syncthreads();  // the staging buffer is free
         // ---- the next active row's copy goes in flight while this row is
         // processed; after a copy that gave up (which may still land) none does
@@ -1090,33 +1115,31 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
         }
         const bool werr = __any_sync(0xffffffffu, !landed);
 
-        // ---- pass 0: this warp's maxima (JSD: clamped logits kept; RKL: with the
-        // target logit at the draft maximum)
-        float mz = kNegInf, mt = kNegInf, tp = kNegInf;
-        // RKL: the raw words of the chunk that first raised this thread's draft maximum
-        // (or the tail entry's target logit), scanned for the pivot once the pass is done
-        [[maybe_unused]] uint4 pz = make_uint4(0u, 0u, 0u, 0u), pt = pz;
-        [[maybe_unused]] bool piv_tail = false;
-        sweep_tm<In, kJsd, kJsd, true, false, kJsd>(tw, tsh, nv, tail, tz, tt,
-            [&](const float*, const float* t, auto tag, int, float cz, float ct, bool, uint4& zr, uint4& tr) {
-                if constexpr (kRkl) {
-                    constexpr int kCnt = decltype(tag)::value;
-                    if (cz > mz) {
-                        mz = cz;
-                        if constexpr (kCnt == 1) {
-                            piv_tail = true;
-                            tp = t[0];
-                        } else {
-                            piv_tail = false;
-                            pz = zr;
-                            pt = tr;
+        if constexpr (!kStage0) {
+            // ---- pass 0: this warp's maxima (RKL: the raw words of the chunk that first
+            // raised this thread's draft maximum, or the tail entry's target logit, are
+            // kept and scanned for the pivot once the pass is done)
+            sweep_tm<In, false, false, true, false, false>(tw, tsh, nv, tail, tz, tt,
+                [&](const float*, const float* t, auto tag, int, float cz, float ct, bool, uint4& zr, uint4& tr) {
+                    if constexpr (kRkl) {
+                        constexpr int kCnt = decltype(tag)::value;
+                        if (cz > mz) {
+                            mz = cz;
+                            if constexpr (kCnt == 1) {
+                                piv_tail = true;
+                                tp = t[0];
+                            } else {
+                                piv_tail = false;
+                                pz = zr;
+                                pt = tr;
+                            }
                         }
+                    } else {
+                        mz = fmaxf(mz, cz);
                     }
-                } else {
-                    mz = fmaxf(mz, cz);
-                }
-                mt = fmaxf(mt, ct);
-            });
+                    mt = fmaxf(mt, ct);
+                });
+        }
         if constexpr (kRkl) {
             if (!piv_tail && mz != kNegInf) {  // the first entry of the saved chunk that holds mz
                 float z[kVec], t[kVec];
