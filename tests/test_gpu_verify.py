@@ -62,6 +62,12 @@ CASES = [  # (B, k, V, dtype, T)
     (300, 2, 16384, torch.float32, 0.7),     # exactly one slice
     (150, 4, 49160, torch.bfloat16, 1.3),    # a ragged last slice
     (140, 2, 16392, torch.bfloat16, 0.7),    # a last slice of one 8-entry vector
+    # a single sequence: one cluster (the one-launch path where the rows are 16-byte aligned)
+    (1, 1, 1, torch.float32, 1.0),
+    (1, 5, 7, torch.bfloat16, 0.7),
+    (1, 5, 32000, torch.bfloat16, 1.0),
+    (1, 8, 128256, torch.bfloat16, 0.7),
+    (1, 3, 32000, torch.float32, 1.3),
 ]
 
 
@@ -79,7 +85,7 @@ GREEDY_CASES = [
     (16, 3, 1, torch.float32), (32, 4, 1001, torch.bfloat16), (9, 2, 40000, torch.float32),
     (12, 5, 32000, torch.bfloat16), (38, 7, 32768, torch.bfloat16), (7, 3, 4096, torch.bfloat16),
     (5, 1, 40, torch.float32), (20, 5, 16000, torch.float32), (39, 7, 32768, torch.bfloat16),
-    (4, 8, 32000, torch.bfloat16),
+    (4, 8, 32000, torch.bfloat16), (1, 5, 32000, torch.bfloat16), (1, 1, 1, torch.float32),
 ]
 
 
