@@ -1248,8 +1248,10 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                                 }
                                 const float2 pj = make_float2(ex2(u.x), ex2(u.y)), qj = make_float2(ex2(v.x), ex2(v.y));
                                 if constexpr (kJsd) {
-                                    const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
-                                    const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
+                                    // m plus the smallest normal: equal to m above about 2^-102, and
+                                    // never 0, so that no lg2 of it is -inf (one FMA, no max)
+                                    const float2 m = fma2(pj, f2(beta), fma2(qj, f2(1.f - beta), f2(kMinNormal)));
+                                    const float2 lm = make_float2(lg2(m.x), lg2(m.y));
                                     const float2 pw = two ? pj : make_float2(pj.x, 0.f);
                                     const float2 qw = two ? qj : make_float2(qj.x, 0.f);
                                     A2 = fma2(pw, sub2(u, lm), A2);
@@ -1461,8 +1463,8 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
                         } else {
                             const float2 u = fma2(tdiff(e, gt), f2(c), cus);
                             const float2 pj = make_float2(ex2(u.x), ex2(u.y));
-                            const float2 m = fma2(pj, f2(beta), mul2(qj, f2(1.f - beta)));
-                            const float2 lm = make_float2(lg2(fmaxf(m.x, kMinNormal)), lg2(fmaxf(m.y, kMinNormal)));
+                            const float2 m = fma2(pj, f2(beta), fma2(qj, f2(1.f - beta), f2(kMinNormal)));
+                            const float2 lm = make_float2(lg2(m.x), lg2(m.y));
                             gg = mul2(qj, sub2(sub2(v, lm), f2(sa)));
                         }
                         gr[e] = gg.x;
