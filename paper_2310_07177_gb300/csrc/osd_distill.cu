@@ -1689,10 +1689,12 @@ static cudaError_t tm_launch_shape(int span, int csize, TmLaunch* out) {
         attr.val.clusterDim.z = 1;
         cfg.attrs = &attr;
         cfg.numAttrs = 1;
+        // a failed query leaves the estimate above (the error is not sticky; clear it)
         int n = 0;
-        e = cudaOccupancyMaxActiveClusters(&n, tm_cluster_probe, &cfg);
-        if (e != cudaSuccess) return e;
-        if (n >= 1) clusters = std::min(clusters, n);
+        if (cudaOccupancyMaxActiveClusters(&n, tm_cluster_probe, &cfg) == cudaSuccess && n >= 1)
+            clusters = std::min(clusters, n);
+        else
+            (void)cudaGetLastError();
     }
     {
         std::lock_guard<std::mutex> lock(mu);
