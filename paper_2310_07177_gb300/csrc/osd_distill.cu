@@ -1721,9 +1721,9 @@ static cudaError_t launch_distill_tm(const DistParams& dp, long long rows, cudaS
     // before them in pairs).  With runs of 8 throughout, 6554 rows over about 228
     // resident clusters left some clusters 32 rows and others 24.  The long runs
     // are 8 rows from 16 K rows on, 4 from 8 K, else 2: with few rows per cluster
-    // more, shorter runs did better than one wave of long ones (256 rows of 128256
-    // over 47 resident 16-CTA clusters: runs of 2, 67.6 us; one wave of runs of 6,
-    // 71.7 us), the 16 CTAs of a row waiting on each other twice a row.
+    // more, shorter runs did better than one wave of long ones (a call of 256 rows
+    // of 128256 over the 47 resident 16-CTA clusters: runs of 2, 67.6 us; one wave of
+    // runs of 6, 71.7 us), the 16 CTAs of a row waiting on each other twice a row.
     const long long K = tl.clusters;
     const long long ones = std::min(rows, K);
     const long long twos = std::min(rows - ones, 2 * K);
