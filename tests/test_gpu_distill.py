@@ -329,3 +329,28 @@ def test_masked_rows_unaligned_mask_and_few_rows(osd, kind):
         lr, gr = _oracle(z, t, mask, kind, 0.5)
         skip = _tvd_ambiguous(z, t) if kind == "tvd" else None
         check_distill(loss.cpu().numpy(), gg.cpu().numpy(), lr, gr, mask.numpy() == 1, skip)
+
+
+def test_concurrent_flushes_on_two_streams(osd):
+    """Two buffer flushes on the TMEM-staged runs in flight at once on two streams
+    (RKL beside TVD, FKL beside JSD): their clusters share the SMs and tensor memory,
+    and every CTA's shared-memory request keeps the resident CTAs within the SM's 512
+    columns, so each flush gives exactly the results it gives alone."""
+    dev = torch.device("cuda")
+    spec = W.DistillSpec(1024, 32000, torch.bfloat16, 2.0, "draft+noise", 2.0, 1.0)
+    a = W.distill_inputs(spec, seed=701, device=dev)
+    b = W.distill_inputs(spec, seed=702, device=dev)
+    for ka, kb in (("rkl", "tvd"), ("fkl", "jsd")):
+        ref_a = osd.osd_distill(a["draft"], a["target"], None, ka, 0.5)
+        ref_b = osd.osd_distill(b["draft"], b["target"], None, kb, 0.5)
+        torch.cuda.synchronize()
+        s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+        s1.wait_stream(torch.cuda.current_stream())
+        s2.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s1):
+            out_a = osd.osd_distill(a["draft"], a["target"], None, ka, 0.5, stream=s1)
+        with torch.cuda.stream(s2):
+            out_b = osd.osd_distill(b["draft"], b["target"], None, kb, 0.5, stream=s2)
+        torch.cuda.synchronize()
+        for ref, out in ((ref_a, out_a), (ref_b, out_b)):
+            assert torch.equal(ref[0], out[0]) and torch.equal(ref[1], out[1])
