@@ -198,6 +198,31 @@ def test_extreme_and_neg_inf_logits(osd):
         check_distill(lg, gg, lr, gr, np.ones(5, bool), skip)
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("tau", [1.0, 0.7])
+def test_logits_far_above_the_first_chunks(osd, dtype, tau):
+    """TVD and JSD sum against a reference taken from each thread's first chunk; a
+    logit far above it later in the row (or a row whose first chunks are all -inf)
+    must give the same result as the true maxima."""
+    g0 = torch.Generator().manual_seed(31)
+    N, V = 6, 32000
+    z = torch.randn(N, V, generator=g0) * 2
+    t = torch.randn(N, V, generator=g0) * 2
+    z[0, V - 1] = 80.0                       # a late spike in the draft row
+    t[1, 31000] = 50.0                       # ... in the target row only
+    z[2, :4096] = float("-inf")              # every first chunk of the span is -inf
+    t[2, :4096] = float("-inf")
+    t[3] = z[3]                              # identical rows with a late spike in both
+    z[3, 20000] = t[3, 20000] = 70.0
+    z[4, 9000:9100] = 45.0                   # a late plateau
+    z, t = z.to(dtype), t.to(dtype)
+    for kind in KINDS:
+        lg, gg = _run(osd, z, t, None, kind, 0.3, tau=tau)
+        lr, gr = _oracle(z, t, None, kind, 0.3, tau=tau)
+        skip = _tvd_ambiguous(z, t, tau) if kind == "tvd" else None
+        check_distill(lg, gg, lr, gr, np.ones(N, bool), skip)
+
+
 def test_invalid_arguments_are_rejected(osd):
     dev = torch.device("cuda")
     z = torch.zeros(2, 16, device=dev)
