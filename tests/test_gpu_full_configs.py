@@ -33,9 +33,9 @@ def osd():
     return pkg
 
 
-def _flush(osd, cfg, kind, beta):
-    spec = W.DISTILL[cfg]
-    inp = W.distill_inputs(spec, seed=W.seed_for(cfg), device="cuda")
+def _flush(osd, workload, kind, beta):
+    spec = W.DISTILL[workload]
+    inp = W.distill_inputs(spec, seed=W.seed_for(workload), device="cuda")
     z, t, mask = inp["draft"], inp["target"], inp["mask"]
     dl = torch.full((spec.N, spec.V), float("nan"), device="cuda")
     status = torch.full((1,), -1, dtype=torch.int32, device="cuda")
@@ -44,11 +44,11 @@ def _flush(osd, cfg, kind, beta):
     assert status.item() == 0
     active = None if mask is None else mask.cpu().numpy() == 1
     rep = distill_parity(z, t, active, loss, g, kind, beta)
-    print(f"config {cfg} {kind}: {rep}")
+    print(f"flush {spec.N} x {spec.V} {kind}: {rep}")
     return spec, rep
 
 
-def test_config3_jsd_every_row(osd):
+def test_masked_flush_jsd_every_row(osd):
     spec, rep = _flush(osd, 3, "jsd", 0.5)
     n_on = int(round(spec.active_frac * spec.N))
     assert rep["rows"] == n_on == 6554
@@ -56,7 +56,7 @@ def test_config3_jsd_every_row(osd):
 
 
 @pytest.mark.parametrize("kind", ["rkl", "tvd"])
-def test_config4_every_row(osd, kind):
+def test_flush_65536_rows_every_row(osd, kind):
     spec, rep = _flush(osd, 4, kind, 0.5)
     assert rep["rows"] == spec.N == 65536 and rep["inactive_rows"] == 0
 
@@ -72,17 +72,17 @@ def large_vocab(osd):
     return spec, inp, res, ref
 
 
-def test_config5_verify_every_sequence(large_vocab):
+def test_large_vocab_verify_every_sequence(large_vocab):
     spec, inp, res, ref = large_vocab
     rep = check_verify(res, ref, spec.k, spec.V)
     worst = check_margins(res, ref)
     assert rep["sequences"] == spec.B == 256
     acc = res.accepted.cpu().numpy()
-    print(f"config 5 verify: {rep}, accept-ratio error max {worst:.3g}, "
+    print(f"verify B=256 k=8 V=128256: {rep}, accept-ratio error max {worst:.3g}, "
           f"mean accepted {acc.mean():.3f}, rejecting sequences {int((acc < spec.k).sum())}")
 
 
-def test_config5_chain_every_rejected_row(osd, large_vocab):
+def test_large_vocab_fkl_chain_every_rejected_row(osd, large_vocab):
     """osd_verify's mismatch mask drives forward-KL distillation of the [B, k]
     draft rows against the target[:, :k] view on the same stream."""
     spec, inp, res, ref = large_vocab
@@ -95,10 +95,10 @@ def test_config5_chain_every_rejected_row(osd, large_vocab):
     rep = distill_parity(inp["draft"].reshape(-1, V), inp["target"][:, :k].reshape(-1, V), active,
                          loss.reshape(-1), g.reshape(-1, V), "fkl", 0.5)
     assert rep["rows"] + rep["inactive_rows"] == B * k
-    print(f"config 5 verify -> FKL chain: {rep}")
+    print(f"verify B=256 k=8 V=128256 -> FKL chain: {rep}")
 
 
-def test_config5_distill_accepted_every_row(osd, large_vocab):
+def test_large_vocab_distill_accepted_every_row(osd, large_vocab):
     """The same rows chosen on the device from the accepted counts and compacted."""
     spec, inp, res, ref = large_vocab
     B, k, V = spec.B, spec.k, spec.V
@@ -119,4 +119,4 @@ def test_config5_distill_accepted_every_row(osd, large_vocab):
     rep = distill_parity(inp["draft"][bi, ai], inp["target"][bi, ai], None, rej.loss[:n], rej.dlogits[:n],
                          "fkl", 0.5)
     assert (rej.loss[n:] == 0).all() and torch.isnan(rej.dlogits[n:]).all()
-    print(f"config 5 osd_distill_accepted: {rep}, slots beyond the count {B - n}")
+    print(f"V=128256 osd_distill_accepted: {rep}, slots beyond the count {B - n}")
