@@ -743,7 +743,7 @@ __global__ void __launch_bounds__(kT) distill_kernel(DistParams p) {
 // hardware schedules the runs like any grid (no assumption on how many
 // clusters are resident), and masked-out rows of a run cost one mask read.
 // 16-byte-aligned rows; TVD, JSD, RKL and FKL (CE, which needs no second
-// exchange, stays on the per-row kernel, at 96 % of the HBM peak there).  A row
+// exchange, stays on the per-row kernel, at 97 % of the HBM peak there).  A row
 // costs one CTA barrier (the staging buffer is free) and two exchanges within
 // the cluster: TVD and JSD exchange the normalisers, then the sums of pass 2;
 // RKL and FKL the maxima (RKL with its pivot), then the sums and the moment.
@@ -923,14 +923,14 @@ __global__ void __launch_bounds__(kTmThreads, 7) distill_tm_kernel(DistParams p,
     constexpr bool kJsd = kKind == OSD_JSD, kTvd = kKind == OSD_TVD, kRkl = kKind == OSD_RKL;
     constexpr bool kFkl = kKind == OSD_FKL;
     constexpr bool kMom = kRkl || kFkl;  // the maxima go round first, then the sums with the loss moment
-    // pass 0 (the maxima) taken while the span moves into tensor memory (FKL: 1.6 %
-    // faster) or as a sweep of its own after the next row's copy is issued (RKL: 1.9 %
-    // faster that way)
+    // work done while the span moves into tensor memory: FKL's pass 0 (the maxima; 1.6 %
+    // faster than a sweep of its own), JSD's clamp and its first-chunk maxima (below).
+    // RKL keeps pass 0 as a sweep after the next row's copy is issued (1.9 % faster that way)
     constexpr bool kStage0 = kJsd || kFkl;
     // TVD and JSD need no pass 0: they sum against a reference taken while staging from
     // each thread's first chunk only (the warp's largest such logit); a warp whose sums
     // come out too large for that (a reference far below a later logit) takes its true
-    // maxima and sums again.  At 65536 x 32000 bf16: TVD 94.9 -> 98.5 %, JSD 80.2 -> 81.3 %
+    // maxima and sums again.  At 65536 x 32000 bf16: TVD 94.9 -> 98.5 %, JSD 80.2 -> 81.2 %
     // of the copy bandwidth
     constexpr bool kRef = kTvd || kJsd;
     // TVD, RKL: exponent arguments x c - m c as one fma; JSD: logits clamped to -1e30, (x - m) c
